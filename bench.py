@@ -1,0 +1,370 @@
+"""Benchmark: draft+verify steps/s of the speculative-decoding hot path on GB300.
+
+One step = one osprey_draft_step (extend row + a K-token chain through the
+drafter, LM head sampled on chip) + one osprey_verify over the workload's
+synthetic target/draft logits, captured in one CUDA graph.  Inputs are seeded
+synthetic data shaped like the workload (weights bf16 ~ N(0, 0.02^2)).
+
+Default workload: Qwen3-8B-shaped drafter (d=1024, 1 layer, 16/8 heads, hd 128,
+FFN 3072, vocab 151936), batch 1, K=7, context 2048, temperature 1.
+
+Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
+the same workload instead (a deliberately slow float64 program).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
+from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: E402
+
+# dram__bytes_read.sum + dram__bytes_write.sum of one LM-head launch, from an
+# ncu capture of this workload; valid only for the draft.cu it was taken on.
+LM_TRAFFIC = {"draft_cu_sha256": None, "bytes_per_launch": None}
+
+
+def _sha(path):
+    with open(path, "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()
+
+
+def parse():
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", default="osprey", choices=["osprey", "reference"])
+    p.add_argument("--workload", default=BENCH_WORKLOAD, choices=sorted(WORKLOADS))
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    return p.parse_args()
+
+
+def make_inputs(wl, rank=0):
+    sh = wl.shape
+    seed = wl.seed + 1000 * rank
+    ctx = syn.make_contexts(wl, seed + 17)
+    w = syn.make_weights(sh, seed)
+    kv = syn.make_kv_prefix(sh, ctx, wl.n_new + wl.K, seed + 1)
+    di = syn.make_draft_inputs(sh, wl.batch, wl.n_new, wl.K, seed + 2)
+    vi = syn.make_verify_inputs(sh.vocab, wl.batch, wl.K, wl.temperature, wl.sigma_p, seed + 3)
+    return ctx, w, kv, di, vi
+
+
+def algorithmic_bytes(wl, ctx):
+    """Bytes the method must touch per step (no L2 reuse credited)."""
+    sh = wl.shape
+    B, K = wl.batch, wl.K
+    w_step = sh.weight_bytes_per_step()
+    kv_row = 2 * sh.n_layers * sh.n_kv_heads * sh.head_dim * 2           # K and V, bf16, all layers
+    # chain step k attends over ctx + n_new + k positions (extend row: ctx + 1 with n_new = 1)
+    kv = sum(kv_row * (int(c) + wl.n_new + k) for c in ctx for k in range(K))
+    draft = K * w_step + 2 * sh.d_model * sh.feat_dim + kv + B * wl.n_new * sh.feat_dim * 2
+    s = 4 if wl.logits_dtype == "f32" else 2
+    verify = B * (K + 1) * sh.vocab * s + B * K * sh.vocab * s
+    lm_launch = sh.vocab * sh.d_model * 2 * 1 + 2 * sh.d_model
+    return {"draft": draft, "verify": verify, "lm_head_launch": lm_launch}
+
+
+class ClockSampler:
+    """nvidia-smi clocks and throttle reasons while the timed region runs."""
+    Q = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index, self.rows, self.proc = index, [], None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
+                                          "--format=csv,noheader,nounits", "-lms", "100"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except OSError:
+            self.proc = None
+        return self
+
+    def _read(self):
+        for line in self.proc.stdout:
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) == 7:
+                self.rows.append(parts)
+
+    def __exit__(self, *a):
+        if self.proc:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self):
+        if not self.rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
+        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
+        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[3 + i].lower() == "active"})
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(self.rows)}
+
+
+def peaks():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            p = json.load(f)
+        return float(p["hbm_gbs"]), "measured"
+    except (OSError, KeyError, ValueError):
+        return 6800.0, "fallback"
+
+
+def cpu_baseline(wl, ctx, w, kv, di, vi, budget_s=10.0):
+    """The oracle as it stands on the host cores: whole steps of the same workload."""
+    import torch
+    from oracle import drafter as od
+    from oracle import verify as ov
+    t0 = time.perf_counter()
+    W = od.widen_weights(w)
+    setup = time.perf_counter() - t0
+    n, t_run = 0, 0.0
+    while True:
+        t1 = time.perf_counter()
+        od.draft_step(w, wl.shape, kv["k_rows"], kv["v_rows"], ctx, di["tokens"], di["feats"], di["n_new"], wl.K,
+                      wl.temperature, di["u_draft"], widened=W)
+        ov.verify(vi["target_logits"], vi["draft_logits"], vi["draft_tokens"], wl.temperature, vi["u_accept"],
+                  vi["u_sample"])
+        t_run += time.perf_counter() - t1
+        n += 1
+        if t_run > budget_s or n >= 50:
+            break
+    cores = torch.get_num_threads()
+    return {"value": n / t_run, "unit": "steps/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} full step(s) (draft K={wl.K} + verify) of {wl.name}, float64 numpy; "
+                      f"weights widened once ({setup:.1f}s, untimed); {os.cpu_count()} host cores visible"}
+
+
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    wl = WORKLOADS[args.workload]
+    ctx, w, kv, di, vi = make_inputs(wl)
+    from oracle import drafter as od
+    from oracle import verify as ov
+    import torch
+    W = od.widen_weights(w)
+
+    def step():
+        od.draft_step(w, wl.shape, kv["k_rows"], kv["v_rows"], ctx, di["tokens"], di["feats"], di["n_new"], wl.K,
+                      wl.temperature, di["u_draft"], widened=W)
+        ov.verify(vi["target_logits"], vi["draft_logits"], vi["draft_tokens"], wl.temperature, vi["u_accept"],
+                  vi["u_sample"])
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    dt = time.perf_counter() - t0
+    v = args.steps / dt
+    cores = torch.get_num_threads()
+    print(json.dumps({
+        "impl": "reference", "metric": "draft+verify steps/s", "value": v, "unit": "steps/s", "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": config_of(wl, ctx),
+        "cpu_baseline": {"value": v, "unit": "steps/s", "cores": cores, "kind": "oracle",
+                         "sample": f"whole steps of {wl.name} on the host cores"},
+        "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }))
+
+
+def config_of(wl, ctx):
+    sh = wl.shape
+    return {"workload": wl.name, "batch": wl.batch, "K": wl.K, "ctx": [int(ctx.min()), int(ctx.max())],
+            "vocab": sh.vocab, "d_model": sh.d_model, "layers": sh.n_layers,
+            "heads": f"{sh.n_q_heads}/{sh.n_kv_heads}x{sh.head_dim}", "ffn": sh.ffn_dim,
+            "temperature": wl.temperature, "logits": wl.logits_dtype, "weights": "bf16",
+            "l2": "flushed (256 MB write) before every timed step", "parallelism": "replicas"}
+
+
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_09338_gb300 import binding as ob
+    from paper_2609_09338_gb300.session import DraftSession, VerifyBuffers
+
+    wl = WORKLOADS[args.workload]
+    sh, B, K, T = wl.shape, wl.batch, wl.K, wl.temperature
+    ctx, w, kv, di, vi = make_inputs(wl, rank)
+    dev = "cuda"
+    sess = DraftSession(sh, w, kv["page_table"], kv["n_pages"], K, wl.n_new)
+    sess.append(ctx, kv["k_rows"], kv["v_rows"])
+    torch.cuda.synchronize()
+    assert int(sess.status.item()) == 0
+    seq0 = sess.kv.seq_len.clone()
+    T_ = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    d_in = {"n_new": T_(di["n_new"]), "tokens": T_(di["tokens"]), "feats": ob.to_device_bf16(di["feats"]),
+            "u_draft": T_(di["u_draft"])}
+    if wl.logits_dtype == "f32":
+        v_in = {"target": T_(vi["target_logits"]), "draft": T_(vi["draft_logits"])}
+    else:
+        v_in = {"target": ob.to_device_bf16(syn.bf16_bits(vi["target_logits"])),
+                "draft": ob.to_device_bf16(syn.bf16_bits(vi["draft_logits"]))}
+    v_in.update({"tokens": T_(vi["draft_tokens"]), "u_accept": T_(vi["u_accept"]), "u_sample": T_(vi["u_sample"])})
+    out = sess.draft_buffers()
+    vb = VerifyBuffers(B, K, sh.vocab)
+    ob.osprey_probe_enable(sess.ctx, K)
+    stream = torch.cuda.Stream()
+
+    def step():
+        sess.kv.seq_len.copy_(seq0)
+        sess.draft(d_in["n_new"], d_in["tokens"], d_in["feats"], T, d_in["u_draft"], out)
+        vb.run(v_in["target"], v_in["draft"] if T > 0 else None, v_in["tokens"], T, v_in["u_accept"],
+               v_in["u_sample"])
+
+    # eager warm-up, then capture one step in a graph
+    with torch.cuda.stream(stream):
+        step()
+    torch.cuda.synchronize()
+    graph = torch.cuda.CUDAGraph()
+    n0 = ob.osprey_launch_count()
+    with torch.cuda.graph(graph, stream=stream):
+        step()
+    launches_per_step = ob.osprey_launch_count() - n0
+    torch.cuda.synchronize()
+    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    for _ in range(max(args.warmup, 3)):
+        flush.zero_()
+        graph.replay()
+    torch.cuda.synchronize()
+    assert int(sess.status.item()) == 0 and int(vb.status.item()) == 0
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    lm_ms = []
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clk:
+        with torch.cuda.stream(stream):
+            for i in range(args.steps):
+                flush.zero_()
+                starts[i].record(stream)
+                graph.replay()
+                ends[i].record(stream)
+                ends[i].synchronize()
+                lm_ms.extend(ob.osprey_probe_read(sess.ctx, K))
+        torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    ms = sum(step_ms) / len(step_ms)
+    if world > 1:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+
+    # verify alone (same inputs, L2 flushed): verify GB/s
+    vgraph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(vgraph, stream=stream):
+        vb.run(v_in["target"], v_in["draft"] if T > 0 else None, v_in["tokens"], T, v_in["u_accept"], v_in["u_sample"])
+    vs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ve = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            flush.zero_()
+            vs[i].record(stream)
+            vgraph.replay()
+            ve[i].record(stream)
+    torch.cuda.synchronize()
+    v_ms = sum(s.elapsed_time(e) for s, e in zip(vs, ve)) / args.steps
+
+    # end to end: inputs from pinned host memory, results back to the host
+    h_in = {k: v.cpu().pin_memory() for k, v in {**d_in, **v_in}.items()}
+    h_out = {"draft_tokens": torch.empty_like(out["draft_tokens"], device="cpu").pin_memory(),
+             "out_tokens": torch.empty_like(vb.out_tokens, device="cpu").pin_memory(),
+             "n_accepted": torch.empty_like(vb.n_accepted, device="cpu").pin_memory()}
+    dst = {**d_in, **v_in}
+    es, ee = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)], \
+        [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            flush.zero_()
+            es[i].record(stream)
+            for k, v in h_in.items():
+                dst[k].copy_(v, non_blocking=True)
+            graph.replay()
+            h_out["draft_tokens"].copy_(out["draft_tokens"], non_blocking=True)
+            h_out["out_tokens"].copy_(vb.out_tokens, non_blocking=True)
+            h_out["n_accepted"].copy_(vb.n_accepted, non_blocking=True)
+            ee[i].record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = sum(s.elapsed_time(e) for s, e in zip(es, ee)) / args.steps
+    h2d = sum(v.numel() * v.element_size() for v in h_in.values())
+    d2h = sum(v.numel() * v.element_size() for v in h_out.values())
+
+    nb = algorithmic_bytes(wl, ctx)
+    peak, peak_kind = peaks()
+    lm_mean_ms = sum(lm_ms) / len(lm_ms)
+    lm_gbs = nb["lm_head_launch"] / (lm_mean_ms * 1e-3) / 1e9
+    sha = _sha(os.path.join(ROOT, "paper_2609_09338_gb300", "csrc", "draft.cu"))
+    traffic = LM_TRAFFIC["bytes_per_launch"] if LM_TRAFFIC["draft_cu_sha256"] == sha else None
+    acc_len = float(vb.n_accepted.float().mean().item()) + 1.0
+
+    if rank == 0:
+        res = {
+            "metric": "draft+verify steps/s", "value": world * 1e3 / ms, "unit": "steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": config_of(wl, ctx),
+            "drafted_tokens_per_s": world * B * K * 1e3 / ms,
+            "verify_gbs": nb["verify"] / (v_ms * 1e-3) / 1e9,
+            "verify_us": v_ms * 1e3,
+            "draft_step_bytes": nb["draft"],
+            "step_hbm_frac": (nb["draft"] + nb["verify"]) / (ms * 1e-3) / 1e9 / peak,
+            "synthetic_al": acc_len,
+            "roofline": {"kernel": "lm_head_kernel (fused final RMSNorm + LM-head GEMV + online softmax)",
+                         "bound": "hbm", "achieved": lm_gbs, "peak": peak, "unit": "GB/s",
+                         "frac": lm_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
+                         "bytes_per_launch": nb["lm_head_launch"], "mean_launch_us": lm_mean_ms * 1e3,
+                         "launches_timed": len(lm_ms)},
+            "e2e": {"value": world * 1e3 / e2e_ms, "unit": "steps/s", "h2d_bytes_per_step": h2d,
+                    "d2h_bytes_per_step": d2h},
+            "gpu_launches": launches_per_step * args.steps,
+            "clocks": clk.summary(),
+        }
+        if not args.no_cpu_baseline:
+            res["cpu_baseline"] = cpu_baseline(wl, ctx, w, kv, di, vi)
+        print(json.dumps(res))
+    if world > 1:
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,203 @@
+/*
+ * osprey.h - C ABI of the speculative-decoding hot path (draft step + verify)
+ * for Osprey-style drafters on one NVIDIA GB300 (sm_103a).
+ *
+ * The path, after the paper:
+ *   - Sec. 3.1: a drafter q proposes K tokens after a prefix; the frozen target p
+ *     verifies them in one pass with the standard speculative-sampling rule
+ *     (Leviathan et al.), which Osprey does not modify.
+ *   - Sec. 3.3, Eq. 1: c_t = W_c [h_low; h_mid; h_high] projects three target
+ *     hidden states into the drafter width and feeds every attention layer.
+ *   - Sec. 3.3, Eq. 2-3: each layer's QKV projection reads [c_{t-1}; z_t]
+ *     through W~_qkv = [W_ctx  W_qkv] (context columns first).
+ *   - Sec. 3.4: inside a chain the drafter's own hidden state (the last layer's
+ *     residual output, before the final norm) takes the context slot.
+ *   - Sec. 4 (inference settings): chain drafting with topk = 1.
+ *
+ * Conventions for every entry point:
+ *   - All tensor arguments are DEVICE pointers owned by the caller and borrowed
+ *     for the duration of the (asynchronous) call.  The library allocates no
+ *     device memory on these paths; scratch comes from a caller workspace.
+ *   - Work is enqueued on `stream` (a cudaStream_t; NULL = legacy default
+ *     stream) and returns before it completes.  Nothing is synchronised.
+ *   - The return value is OSPREY_OK or a negative OSPREY_ERR_* code.  Argument
+ *     errors the host can see are reported before anything is launched;
+ *     osprey_last_error() then holds a message (thread-local).
+ *   - Errors only the device can see (a token id out of range, a sequence whose
+ *     pages cannot hold the rows) are written to the caller's int32
+ *     `dev_status` word (first error wins; it is never cleared by the library:
+ *     the caller zeroes it).  The affected sequence's outputs are filled with
+ *     -1 / 0 and the other sequences are unaffected.
+ *   - A workspace must be zero-filled once before its first use (the kernels
+ *     leave their counters at zero again when they finish).  A workspace must
+ *     not be shared by calls that can run at the same time.
+ *   - bf16 is IEEE-754 binary32 truncated to its top 16 bits (round to nearest
+ *     even by the producer); all row-major, no padding.
+ */
+#ifndef OSPREY_H
+#define OSPREY_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define OSPREY_MAX_LAYERS 8
+
+enum {
+    OSPREY_OK = 0,
+    OSPREY_ERR_INVALID_ARG = -1, /* null pointer, bad count, bad enum */
+    OSPREY_ERR_SHAPE = -2,       /* a dimension the kernels do not support */
+    OSPREY_ERR_DTYPE = -3,       /* unknown logits dtype */
+    OSPREY_ERR_CAPACITY = -4,    /* pages or workspace too small */
+    OSPREY_ERR_CUDA = -5,        /* a CUDA runtime call failed */
+    OSPREY_ERR_TIMEOUT = -6      /* reserved for bounded device waits */
+};
+
+enum { OSPREY_F32 = 0, OSPREY_BF16 = 1 };
+
+/* Drafter shape.  d_model, head_dim and feat_dim multiples of 256, 64 and 256;
+ * n_q_heads a multiple of n_kv_heads; ffn_dim a multiple of 256.
+ * rms_eps: RMSNorm epsilon (1e-6).  rope_theta: rotary base (rotate-half
+ * convention, angle pos * theta^(-2i/head_dim)). */
+typedef struct osprey_config {
+    int32_t d_model, n_layers, n_q_heads, n_kv_heads, head_dim, ffn_dim, vocab, feat_dim;
+    int32_t page_size; /* KV page length in positions; must be 16 */
+    float rms_eps, rope_theta;
+} osprey_config;
+
+/* Drafter weights, bf16, device, borrowed for the context's lifetime.
+ *   W_c        [d][feat_dim]                 Eq. 1, no bias
+ *   embed      [vocab][d]
+ *   final_norm [d]
+ *   lm_head    [vocab][d]
+ * per layer l < n_layers:
+ *   attn_norm  [d]
+ *   W_qkv      [(Hq + 2 Hkv) head_dim][2 d]  Eq. 2: columns 0..d-1 read the
+ *              context slot (c or the fed-back hidden state), d..2d-1 read
+ *              RMSNorm(x); rows are Q heads, then K heads, then V heads
+ *   W_o        [d][Hq head_dim]
+ *   ffn_norm   [d]
+ *   W_gate, W_up [ffn][d];  W_down [d][ffn]                                  */
+typedef struct osprey_weights {
+    const void *W_c, *embed, *final_norm, *lm_head;
+    const void *attn_norm[OSPREY_MAX_LAYERS], *W_qkv[OSPREY_MAX_LAYERS], *W_o[OSPREY_MAX_LAYERS];
+    const void *ffn_norm[OSPREY_MAX_LAYERS], *W_gate[OSPREY_MAX_LAYERS], *W_up[OSPREY_MAX_LAYERS];
+    const void *W_down[OSPREY_MAX_LAYERS];
+} osprey_weights;
+
+/* Paged drafter KV cache (bf16, device, caller-owned).
+ *   k_pages, v_pages [n_layers][n_pages][n_kv_heads][page_size][head_dim]
+ *   page_table [B][max_pages_per_seq] int32: position t of sequence b lives in
+ *              page page_table[b][t / page_size], slot t % page_size
+ *   seq_len    [B] int32: committed positions of each sequence                */
+typedef struct osprey_kv {
+    void *k_pages, *v_pages;
+    int32_t *page_table, *seq_len;
+    int32_t max_pages_per_seq, n_pages;
+} osprey_kv;
+
+typedef struct osprey_ctx osprey_ctx;
+
+/* Thread-local message for the last error returned on this thread ("" if none). */
+const char *osprey_last_error(void);
+
+/* Validate the shape and weight pointers and make a context (host memory only).
+ * Errors: INVALID_ARG (null), SHAPE (unsupported dimension). */
+int osprey_create(const osprey_config *cfg, const osprey_weights *w, osprey_ctx **out);
+void osprey_destroy(osprey_ctx *ctx);
+
+/* Bytes of workspace osprey_draft_step needs for a batch of B sequences, chains
+ * of K tokens, up to max_new extend rows per sequence and page tables of
+ * max_pages_per_seq pages.  0 on bad arguments. */
+size_t osprey_draft_workspace_bytes(const osprey_ctx *ctx, int B, int K, int max_new,
+                                    int max_pages_per_seq);
+
+/* Write K/V rows into the paged cache after each sequence's committed length
+ * and advance seq_len (the prefix fill of a draft session).
+ *   n_rows [B] int32 (device): rows for sequence b, summing to total_rows
+ *   k_rows, v_rows [n_layers][total_rows][n_kv_heads][head_dim] bf16 (keys
+ *   already rotated), rows of sequence b after those of sequences < b.
+ * Device errors: CAPACITY (rows past the page table or a page id outside
+ * [0, n_pages)), INVALID_ARG (n_rows negative or not summing to total_rows);
+ * such a sequence is left untouched. */
+int osprey_kv_append(const osprey_ctx *ctx, const osprey_kv *kv, int B, const int32_t *n_rows,
+                     int64_t total_rows, const void *k_rows, const void *v_rows,
+                     int32_t *dev_status, void *stream);
+
+/* One draft call: extend, then a K-token chain (Sec. 3.1, Eq. 1-3, Sec. 3.4).
+ *   n_new  [B] int32 (device), 1 <= n_new[b] <= max_new: extend rows of b
+ *   tokens [B][max_new] int32: extend row j is token tokens[b][j] at position
+ *          seq_len[b] + j ...
+ *   feats  [B][max_new][feat_dim] bf16: ... paired with the concatenated target
+ *          hidden states of the previous position (Eq. 2 pairs x_t with c_{t-1})
+ *   temperature: draft distribution q = softmax(logits / T); T == 0 is greedy
+ *          (argmax, lowest id on ties)
+ *   u_draft [B][K] float in [0,1): token k is the smallest id j with
+ *          u * S < C_j (C the inclusive cumulative of exp(logits/T - M) over ids
+ *          in ascending order, S its total)
+ * Outputs (device):
+ *   draft_tokens [B][K] int32
+ *   draft_qx     [B][K] float, q(token) (1 for greedy); may be NULL
+ *   draft_stats  [B][K][2] float, (M, log S) of logits/T (of logits when
+ *                greedy); may be NULL
+ *   draft_logits [B][K][vocab] float, raw logits; NULL to keep them on chip
+ * Effects: the extend rows' K/V are committed and seq_len[b] += n_new[b]; the
+ * chain rows' K/V are written speculatively after them (not committed; the
+ * next call's extend rows overwrite them).  The pages must hold
+ * seq_len[b] + n_new[b] + K - 1 positions (else dev_status = CAPACITY and the
+ * sequence is skipped: tokens -1, seq_len unchanged).
+ * Host errors: INVALID_ARG, SHAPE, CAPACITY (workspace_bytes too small). */
+int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
+                      const int32_t *n_new, const int32_t *tokens, const void *feats,
+                      float temperature, const float *u_draft, int32_t *draft_tokens,
+                      float *draft_qx, float *draft_stats, float *draft_logits,
+                      void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
+
+/* Bytes of workspace osprey_verify needs.  0 on bad arguments. */
+size_t osprey_verify_workspace_bytes(int B, int K, int V);
+
+/* Speculative-sampling verification of B chains of K draft tokens (Sec. 3.1).
+ *   logits_dtype: OSPREY_F32 or OSPREY_BF16 for both logits arrays
+ *   target_logits [B][K+1][V], draft_logits [B][K][V] (may be NULL iff T == 0)
+ *   draft_tokens [B][K] int32 in [0, V)
+ *   temperature: p_i = softmax(target_i / T), q_i = softmax(draft_i / T);
+ *          T == 0 is greedy: accept while argmax p_i == token_i, then emit
+ *          argmax p_r (raw logits, lowest id on ties)
+ *   u_accept [B][K]: accept token i iff u_accept[i] < p_i(x_i) / q_i(x_i)
+ *   u_sample [B][K+1]: the token emitted at the first rejected position r is
+ *          drawn from norm(max(0, p_r - q_r)) (r < K) or from p_K (all
+ *          accepted) by the same inverse CDF as osprey_draft_step, at
+ *          u_sample[r]
+ * Outputs (device):
+ *   out_tokens [B][K+1] int32: accepted tokens, then the emitted one, then -1
+ *   n_accepted [B] int32
+ *   flags [B][K+1] uint8: bit 3 = the residual had no mass in float32 and p_r
+ *          was sampled instead; bit 4 = the inverse-CDF point fell past the last
+ *          cumulative sum after rounding and the last token with mass was taken
+ *   probs [B][K][2] float: (p_i(x_i), q_i(x_i)); may be NULL (greedy: unused)
+ * Device errors: INVALID_ARG for a draft token outside [0, V) (that sequence
+ * gets n_accepted 0 and out_tokens -1). */
+int osprey_verify(int B, int K, int V, int logits_dtype, const void *target_logits,
+                  const void *draft_logits, const int32_t *draft_tokens, float temperature,
+                  const float *u_accept, const float *u_sample, int32_t *out_tokens,
+                  int32_t *n_accepted, uint8_t *flags, float *probs, void *workspace,
+                  size_t workspace_bytes, int32_t *dev_status, void *stream);
+
+/* ---- measurement hooks (not part of the method) ------------------------------
+ * osprey_probe_enable: make n_slots pairs of timing events in the context (n = 0
+ * releases them).  While enabled, osprey_draft_step records pair k around its
+ * k-th LM-head launch (k < n_slots), also under stream capture (as external
+ * event nodes).  osprey_probe_read writes the elapsed milliseconds of the first
+ * n pairs after the caller has synchronised.  osprey_launch_count: kernels the
+ * library has launched (or captured) in this process. */
+int osprey_probe_enable(osprey_ctx *ctx, int n_slots);
+int osprey_probe_read(osprey_ctx *ctx, float *ms, int n);
+int64_t osprey_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* OSPREY_H */

@@ -1,0 +1,433 @@
+// C ABI: argument validation, workspace layout and launch sequencing.
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+
+#include "draft.cuh"
+#include "internal.h"
+#include "osprey.h"
+
+namespace osp {
+
+static std::atomic<long long> g_launches{0};
+void count_launch(int n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+static thread_local char g_err[512] = "";
+
+static int fail(int code, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof g_err, fmt, ap);
+    va_end(ap);
+    return code;
+}
+
+static int cuda_fail(cudaError_t e, const char *what) {
+    return fail(OSPREY_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+static size_t align256(size_t x) { return (x + 255) & ~(size_t)255; }
+
+}  // namespace osp
+
+using namespace osp;
+
+struct osprey_ctx {
+    osprey_config cfg;
+    osprey_weights w;
+    Dims dim;
+    int sms;
+    double inv_freq[64];
+    int n_probe;
+    cudaEvent_t *probe_begin, *probe_end;
+};
+
+extern "C" const char *osprey_last_error(void) { return g_err; }
+extern "C" int64_t osprey_launch_count(void) { return g_launches.load(); }
+
+static bool is_pow2_multiple(int x, int m) { return x > 0 && x % m == 0; }
+
+extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, osprey_ctx **out) {
+    g_err[0] = 0;
+    if (!cfg || !w || !out) return fail(OSPREY_ERR_INVALID_ARG, "null argument");
+    *out = nullptr;
+    const osprey_config &c = *cfg;
+    if (c.n_layers < 1 || c.n_layers > OSPREY_MAX_LAYERS)
+        return fail(OSPREY_ERR_SHAPE, "n_layers must be in 1..%d", OSPREY_MAX_LAYERS);
+    if (!is_pow2_multiple(c.d_model, 256)) return fail(OSPREY_ERR_SHAPE, "d_model must be a multiple of 256");
+    if (c.head_dim != 64 && c.head_dim != 128) return fail(OSPREY_ERR_SHAPE, "head_dim must be 64 or 128");
+    if (c.n_kv_heads < 1 || c.n_q_heads < c.n_kv_heads || c.n_q_heads % c.n_kv_heads)
+        return fail(OSPREY_ERR_SHAPE, "n_q_heads must be a positive multiple of n_kv_heads");
+    const int G = c.n_q_heads / c.n_kv_heads;
+    if (G != 1 && G != 2 && G != 4 && G != 8) return fail(OSPREY_ERR_SHAPE, "n_q_heads/n_kv_heads must be 1, 2, 4 or 8");
+    if ((c.n_q_heads * c.head_dim) % 256) return fail(OSPREY_ERR_SHAPE, "n_q_heads*head_dim must be a multiple of 256");
+    if (!is_pow2_multiple(c.ffn_dim, 256)) return fail(OSPREY_ERR_SHAPE, "ffn_dim must be a multiple of 256");
+    if (!is_pow2_multiple(c.feat_dim, 256)) return fail(OSPREY_ERR_SHAPE, "feat_dim must be a multiple of 256");
+    if (c.feat_dim > 100 * 1024) return fail(OSPREY_ERR_SHAPE, "feat_dim above 102400 is not supported");
+    if (c.vocab < 1) return fail(OSPREY_ERR_SHAPE, "vocab must be positive");
+    if (c.page_size != 16) return fail(OSPREY_ERR_SHAPE, "page_size must be 16");
+    if (!(c.rms_eps > 0.f) || !(c.rope_theta > 1.f)) return fail(OSPREY_ERR_INVALID_ARG, "rms_eps and rope_theta must be positive");
+    if (!w->W_c || !w->embed || !w->final_norm || !w->lm_head) return fail(OSPREY_ERR_INVALID_ARG, "null weight pointer");
+    for (int l = 0; l < c.n_layers; ++l)
+        if (!w->attn_norm[l] || !w->W_qkv[l] || !w->W_o[l] || !w->ffn_norm[l] || !w->W_gate[l] ||
+            !w->W_up[l] || !w->W_down[l])
+            return fail(OSPREY_ERR_INVALID_ARG, "null weight pointer in layer %d", l);
+    const void *ptrs[] = {w->W_c, w->embed, w->final_norm, w->lm_head};
+    for (const void *p : ptrs)
+        if ((uintptr_t)p % 16) return fail(OSPREY_ERR_INVALID_ARG, "weights must be 16-byte aligned");
+    osprey_ctx *ctx = new (std::nothrow) osprey_ctx();
+    if (!ctx) return fail(OSPREY_ERR_INVALID_ARG, "out of host memory");
+    ctx->cfg = c;
+    ctx->w = *w;
+    ctx->dim = Dims{c.d_model, c.n_layers, c.n_q_heads, c.n_kv_heads, c.head_dim, c.ffn_dim,
+                    c.vocab, c.feat_dim, c.page_size, c.rms_eps};
+    for (int i = 0; i < c.head_dim / 2; ++i)
+        ctx->inv_freq[i] = std::pow((double)c.rope_theta, -2.0 * i / c.head_dim);
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e == cudaSuccess) e = draft_set_attributes();
+    if (e != cudaSuccess) {
+        delete ctx;
+        return cuda_fail(e, "device query");
+    }
+    *out = ctx;
+    return OSPREY_OK;
+}
+
+static void probe_release(osprey_ctx *ctx) {
+    for (int i = 0; i < ctx->n_probe; ++i) {
+        cudaEventDestroy(ctx->probe_begin[i]);
+        cudaEventDestroy(ctx->probe_end[i]);
+    }
+    delete[] ctx->probe_begin;
+    delete[] ctx->probe_end;
+    ctx->probe_begin = ctx->probe_end = nullptr;
+    ctx->n_probe = 0;
+}
+
+extern "C" void osprey_destroy(osprey_ctx *ctx) {
+    if (!ctx) return;
+    probe_release(ctx);
+    delete ctx;
+}
+
+extern "C" int osprey_probe_enable(osprey_ctx *ctx, int n) {
+    if (!ctx || n < 0) return fail(OSPREY_ERR_INVALID_ARG, "bad probe arguments");
+    probe_release(ctx);
+    if (n == 0) return OSPREY_OK;
+    ctx->probe_begin = new cudaEvent_t[n];
+    ctx->probe_end = new cudaEvent_t[n];
+    for (int i = 0; i < n; ++i) {
+        cudaError_t e = cudaEventCreate(&ctx->probe_begin[i]);
+        if (e == cudaSuccess) e = cudaEventCreate(&ctx->probe_end[i]);
+        if (e != cudaSuccess) {
+            ctx->n_probe = i;
+            probe_release(ctx);
+            return cuda_fail(e, "cudaEventCreate");
+        }
+        ctx->n_probe = i + 1;
+    }
+    return OSPREY_OK;
+}
+
+extern "C" int osprey_probe_read(osprey_ctx *ctx, float *ms, int n) {
+    if (!ctx || !ms || n < 0 || n > ctx->n_probe) return fail(OSPREY_ERR_INVALID_ARG, "bad probe read");
+    for (int i = 0; i < n; ++i) {
+        cudaError_t e = cudaEventElapsedTime(&ms[i], ctx->probe_begin[i], ctx->probe_end[i]);
+        if (e != cudaSuccess) return cuda_fail(e, "cudaEventElapsedTime");
+    }
+    return OSPREY_OK;
+}
+
+static cudaError_t probe_record(cudaEvent_t ev, cudaStream_t s) {
+    cudaStreamCaptureStatus st = cudaStreamCaptureStatusNone;
+    cudaError_t e = cudaStreamIsCapturing(s, &st);
+    if (e != cudaSuccess) return e;
+    return st == cudaStreamCaptureStatusActive ? cudaEventRecordWithFlags(ev, s, cudaEventRecordExternal)
+                                               : cudaEventRecord(ev, s);
+}
+
+// ------------------------------------------------------------------ workspace
+static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int max_pages,
+                           DraftWs *ws, void *base) {
+    const Dims &D = ctx->dim;
+    const long long R_ext = (long long)B * max_new;
+    const int max_ctx = max_pages * D.P;
+    const int ns = std::max(attn_splits((int)R_ext, D.Hkv, max_ctx, ctx->sms),
+                            attn_splits(B, D.Hkv, max_ctx, ctx->sms));
+    const int lm_warps = lm_blocks(D.V, ctx->sms) * 8;
+    size_t off = 0;
+    auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
+    size_t o_valid = take(4ull * B), o_pos0 = take(4ull * B), o_nn = take(4ull * B);
+    size_t o_at = take(4ull * R_ext * D.Hkv), o_lt = take(4ull * B);
+    size_t o_xe = take(4ull * R_ext * D.d), o_se = take(2ull * R_ext * D.d);
+    size_t o_xc = take(4ull * B * D.d), o_sc = take(2ull * B * D.d);
+    size_t o_q = take(4ull * R_ext * D.Hq * D.hd);
+    size_t o_ap = take(4ull * R_ext * D.Hq * ns * (D.hd + 2));
+    size_t o_ao = take(2ull * R_ext * D.Hq * D.hd);
+    size_t o_fh = take(2ull * R_ext * D.F);
+    size_t o_ls = take(16ull * B * lm_warps);
+    if (ws && base) {
+        char *p = (char *)base;
+        ws->seq_valid = (int *)(p + o_valid);
+        ws->seq_pos0 = (int *)(p + o_pos0);
+        ws->seq_nnew = (int *)(p + o_nn);
+        ws->attn_ticket = (int *)(p + o_at);
+        ws->lm_ticket = (int *)(p + o_lt);
+        ws->x_ext = (float *)(p + o_xe);
+        ws->s_ext = (uint16_t *)(p + o_se);
+        ws->x_chain = (float *)(p + o_xc);
+        ws->s_chain = (uint16_t *)(p + o_sc);
+        ws->q = (float *)(p + o_q);
+        ws->attn_part = (float *)(p + o_ap);
+        ws->attn_out = (uint16_t *)(p + o_ao);
+        ws->ffn_h = (uint16_t *)(p + o_fh);
+        ws->lm_stats = (float4 *)(p + o_ls);
+        ws->n_splits_max = ns;
+        ws->lm_warps_max = lm_warps;
+    }
+    (void)K;
+    return off;
+}
+
+static bool draft_args_ok(const osprey_ctx *ctx, int B, int K, int max_new, int max_pages) {
+    return ctx && B >= 1 && B <= 65535 && K >= 1 && K <= 64 && max_new >= 1 && max_new <= 64 &&
+           max_pages >= 1 && (long long)max_pages * ctx->dim.P < (1LL << 30);
+}
+
+extern "C" size_t osprey_draft_workspace_bytes(const osprey_ctx *ctx, int B, int K, int max_new,
+                                               int max_pages_per_seq) {
+    if (!draft_args_ok(ctx, B, K, max_new, max_pages_per_seq)) return 0;
+    return draft_layout(ctx, B, K, max_new, max_pages_per_seq, nullptr, nullptr);
+}
+
+// ------------------------------------------------------------------ kv append
+extern "C" int osprey_kv_append(const osprey_ctx *ctx, const osprey_kv *kv, int B, const int32_t *n_rows,
+                                int64_t total_rows, const void *k_rows, const void *v_rows,
+                                int32_t *dev_status, void *stream) {
+    g_err[0] = 0;
+    if (!ctx || !kv) return fail(OSPREY_ERR_INVALID_ARG, "null context or kv");
+    if (B == 0) return OSPREY_OK;
+    if (B < 0 || B > 4096) return fail(OSPREY_ERR_INVALID_ARG, "B must be in 0..4096");
+    if (total_rows < 0) return fail(OSPREY_ERR_INVALID_ARG, "total_rows must be >= 0");
+    if (!n_rows || !kv->k_pages || !kv->v_pages || !kv->page_table || !kv->seq_len)
+        return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
+    if (total_rows > 0 && (!k_rows || !v_rows)) return fail(OSPREY_ERR_INVALID_ARG, "null rows");
+    if (kv->max_pages_per_seq < 1 || kv->n_pages < 1) return fail(OSPREY_ERR_INVALID_ARG, "empty page pool");
+    if (((uintptr_t)k_rows | (uintptr_t)v_rows | (uintptr_t)kv->k_pages | (uintptr_t)kv->v_pages) % 16)
+        return fail(OSPREY_ERR_INVALID_ARG, "K/V buffers must be 16-byte aligned");
+    KvAppendArgs a{};
+    a.k_pages = kv->k_pages;
+    a.v_pages = kv->v_pages;
+    a.page_table = kv->page_table;
+    a.seq_len = kv->seq_len;
+    a.n_rows = n_rows;
+    a.k_rows = k_rows;
+    a.v_rows = v_rows;
+    a.total_rows = total_rows;
+    a.B = B;
+    a.L = ctx->dim.L;
+    a.Hkv = ctx->dim.Hkv;
+    a.hd = ctx->dim.hd;
+    a.P = ctx->dim.P;
+    a.max_pages = kv->max_pages_per_seq;
+    a.n_pages = kv->n_pages;
+    a.status = dev_status;
+    cudaError_t e = launch_kv_append(a, (cudaStream_t)stream);
+    return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "kv_append launch");
+}
+
+// ------------------------------------------------------------------ draft step
+extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
+                                 const int32_t *n_new, const int32_t *tokens, const void *feats,
+                                 float temperature, const float *u_draft, int32_t *draft_tokens,
+                                 float *draft_qx, float *draft_stats, float *draft_logits,
+                                 void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                 void *stream) {
+    g_err[0] = 0;
+    if (!ctx || !kv) return fail(OSPREY_ERR_INVALID_ARG, "null context or kv");
+    if (B == 0) return OSPREY_OK;
+    if (!draft_args_ok(ctx, B, K, max_new, kv->max_pages_per_seq))
+        return fail(OSPREY_ERR_INVALID_ARG, "B in 1..65535, K and max_new in 1..64, max_pages_per_seq >= 1 required");
+    if (!(temperature >= 0.f) || !std::isfinite(temperature))
+        return fail(OSPREY_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+    if (!n_new || !tokens || !feats || !draft_tokens || !workspace || !kv->k_pages || !kv->v_pages ||
+        !kv->page_table || !kv->seq_len)
+        return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
+    if (temperature > 0.f && !u_draft) return fail(OSPREY_ERR_INVALID_ARG, "u_draft is required when temperature > 0");
+    if (kv->n_pages < 1) return fail(OSPREY_ERR_INVALID_ARG, "empty page pool");
+    if (((uintptr_t)feats | (uintptr_t)workspace) % 16)
+        return fail(OSPREY_ERR_INVALID_ARG, "feats and workspace must be 16-byte aligned");
+    DraftWs ws{};
+    const size_t need = draft_layout(ctx, B, K, max_new, kv->max_pages_per_seq, &ws, workspace);
+    if (workspace_bytes < need)
+        return fail(OSPREY_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
+
+    cudaStream_t s = (cudaStream_t)stream;
+    const Dims &D = ctx->dim;
+    const osprey_weights &W = ctx->w;
+    const size_t layer_pages = (size_t)kv->n_pages * D.Hkv * D.P * D.hd;
+    const int max_ctx = kv->max_pages_per_seq * D.P;
+    cudaError_t e;
+
+    PrepArgs pa{B, K, max_new, kv->max_pages_per_seq, kv->n_pages, D.P, D.V,
+                kv->seq_len, n_new, tokens, kv->page_table,
+                ws.seq_valid, ws.seq_pos0, ws.seq_nnew, draft_tokens, dev_status};
+    if ((e = launch_prepare(pa, s)) != cudaSuccess) return cuda_fail(e, "prepare launch");
+
+    GemvArgs g{};
+    g.dim = D;
+    g.map = RowMap{ws.seq_valid, ws.seq_pos0, ws.seq_nnew, max_new, 0};
+    g.R = B * max_new;
+    g.W = (const uint16_t *)W.W_c;
+    g.embed = (const uint16_t *)W.embed;
+    g.tokens = tokens;
+    g.feats = (const uint16_t *)feats;
+    g.max_new = max_new;
+    g.x = ws.x_ext;
+    g.s = ws.s_ext;
+    g.page_table = kv->page_table;
+    g.max_pages = kv->max_pages_per_seq;
+    g.n_pages = kv->n_pages;
+    for (int i = 0; i < D.hd / 2; ++i) g.inv_freq[i] = ctx->inv_freq[i];
+    if ((e = launch_gemv(G_FEAT, g, gemv_rg(G_FEAT, D, g.R), ctx->sms, s)) != cudaSuccess)
+        return cuda_fail(e, "feature projection launch");
+
+    for (int step = 0; step < K; ++step) {
+        const bool ext = step == 0;
+        const int rows_per_seq = ext ? max_new : 1;
+        const int R = B * rows_per_seq;
+        RowMap map{ws.seq_valid, ws.seq_pos0, ws.seq_nnew, rows_per_seq, step};
+        float *x = ext ? ws.x_ext : ws.x_chain;
+        uint16_t *sb = ext ? ws.s_ext : ws.s_chain;
+        const int ns = attn_splits(R, D.Hkv, max_ctx, ctx->sms);
+        for (int l = 0; l < D.L; ++l) {
+            g.map = map;
+            g.R = R;
+            g.x = x;
+            g.s = sb;
+            g.W = (const uint16_t *)W.W_qkv[l];
+            g.gain = (const uint16_t *)W.attn_norm[l];
+            g.q = ws.q;
+            g.k_pages = (uint16_t *)kv->k_pages + l * layer_pages;
+            g.v_pages = (uint16_t *)kv->v_pages + l * layer_pages;
+            if ((e = launch_gemv(G_QKV, g, gemv_rg(G_QKV, D, R), ctx->sms, s)) != cudaSuccess)
+                return cuda_fail(e, "qkv launch");
+            AttnArgs at{};
+            at.dim = D;
+            at.map = map;
+            at.R = R;
+            at.n_splits = ns;
+            at.split_len = attn_split_len(max_ctx, ns);
+            at.q = ws.q;
+            at.k_pages = g.k_pages;
+            at.v_pages = g.v_pages;
+            at.page_table = kv->page_table;
+            at.max_pages = kv->max_pages_per_seq;
+            at.part = ws.attn_part;
+            at.out = ws.attn_out;
+            at.ticket = ws.attn_ticket;
+            if ((e = launch_attn(at, s)) != cudaSuccess) return cuda_fail(e, "attention launch");
+            g.W = (const uint16_t *)W.W_o[l];
+            g.xin_bf = ws.attn_out;
+            if ((e = launch_gemv(G_OPROJ, g, gemv_rg(G_OPROJ, D, R), ctx->sms, s)) != cudaSuccess)
+                return cuda_fail(e, "o-proj launch");
+            g.W = (const uint16_t *)W.W_gate[l];
+            g.W2 = (const uint16_t *)W.W_up[l];
+            g.gain = (const uint16_t *)W.ffn_norm[l];
+            g.out_bf = ws.ffn_h;
+            if ((e = launch_gemv(G_GATEUP, g, gemv_rg(G_GATEUP, D, R), ctx->sms, s)) != cudaSuccess)
+                return cuda_fail(e, "gate/up launch");
+            g.W = (const uint16_t *)W.W_down[l];
+            g.xin_bf = ws.ffn_h;
+            if ((e = launch_gemv(G_DOWN, g, gemv_rg(G_DOWN, D, R), ctx->sms, s)) != cudaSuccess)
+                return cuda_fail(e, "down launch");
+        }
+        LmArgs lm{};
+        lm.dim = D;
+        lm.map = map;
+        lm.B = B;
+        lm.K = K;
+        lm.step = step;
+        lm.max_new = max_new;
+        lm.W = (const uint16_t *)W.lm_head;
+        lm.gain = (const uint16_t *)W.final_norm;
+        lm.embed = (const uint16_t *)W.embed;
+        lm.x_in = x;
+        lm.src_is_ext = ext;
+        lm.x_chain = ws.x_chain;
+        lm.s_chain = ws.s_chain;
+        lm.temperature = temperature;
+        lm.u_draft = u_draft;
+        lm.tokens = draft_tokens;
+        lm.qx = draft_qx;
+        lm.stats = draft_stats;
+        lm.logits = draft_logits;
+        lm.warp_stats = ws.lm_stats;
+        lm.ticket = ws.lm_ticket;
+        const int blocks = lm_blocks(D.V, ctx->sms);
+        lm.warps_total = blocks * 8;
+        int rg = 1;
+        while (rg < B && rg < 8) rg <<= 1;
+        const bool probe = step < ctx->n_probe;
+        if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
+            return cuda_fail(e, "probe record");
+        if ((e = launch_lm(lm, rg, blocks, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
+        if (probe && (e = probe_record(ctx->probe_end[step], s)) != cudaSuccess)
+            return cuda_fail(e, "probe record");
+    }
+    return OSPREY_OK;
+}
+
+// ------------------------------------------------------------------ verify
+extern "C" size_t osprey_verify_workspace_bytes(int B, int K, int V) {
+    if (B < 1 || K < 1 || K > 15 || V < 1) return 0;
+    return verify_workspace_layout(B, K, V, nullptr, nullptr);
+}
+
+extern "C" int osprey_verify(int B, int K, int V, int logits_dtype, const void *target_logits,
+                             const void *draft_logits, const int32_t *draft_tokens, float temperature,
+                             const float *u_accept, const float *u_sample, int32_t *out_tokens,
+                             int32_t *n_accepted, uint8_t *flags, float *probs, void *workspace,
+                             size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    g_err[0] = 0;
+    if (B == 0) return OSPREY_OK;
+    if (B < 0 || K < 1 || K > 15 || V < 1)
+        return fail(OSPREY_ERR_INVALID_ARG, "B >= 0, K in 1..15 and V >= 1 required");
+    if (logits_dtype != OSPREY_F32 && logits_dtype != OSPREY_BF16)
+        return fail(OSPREY_ERR_DTYPE, "logits_dtype must be OSPREY_F32 or OSPREY_BF16");
+    if (!(temperature >= 0.f) || !std::isfinite(temperature))
+        return fail(OSPREY_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+    if (!target_logits || !draft_tokens || !out_tokens || !n_accepted || !flags || !workspace)
+        return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
+    if (temperature > 0.f && (!draft_logits || !u_accept || !u_sample))
+        return fail(OSPREY_ERR_INVALID_ARG, "draft_logits, u_accept and u_sample are required when temperature > 0");
+    if ((long long)V * (K + 1) * B > (1LL << 40)) return fail(OSPREY_ERR_SHAPE, "logits too large");
+    if ((long long)((V + 8191) / 8192) * (K + 1) * B >= (1LL << 31))
+        return fail(OSPREY_ERR_SHAPE, "too many (sequence, row, chunk) blocks");
+    VerifyArgs a{};
+    const size_t need = verify_workspace_layout(B, K, V, &a, workspace);
+    if (workspace_bytes < need)
+        return fail(OSPREY_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
+    a.B = B;
+    a.K = K;
+    a.V = V;
+    a.dtype = logits_dtype;
+    a.temperature = temperature;
+    a.target = target_logits;
+    a.draft = draft_logits;
+    a.tokens = draft_tokens;
+    a.u_accept = u_accept;
+    a.u_sample = u_sample;
+    a.out_tokens = out_tokens;
+    a.n_accepted = n_accepted;
+    a.flags = flags;
+    a.probs = probs;
+    a.status = dev_status;
+    cudaError_t e = launch_verify(a, (cudaStream_t)stream);
+    return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "verify launch");
+}

@@ -1,0 +1,732 @@
+// Draft step on CUDA cores: HBM-bound GEMV kernels with fused prologues and
+// epilogues, split-KV GQA decode attention over the paged cache, and an LM
+// head that samples on chip.
+//
+// Per chain step and layer (Sec. 3.3 Eq. 1-3, Sec. 3.4):
+//   qkv     z = RMSNorm(x); [q;k;v] = W~_qkv [s; z]; rotary on q,k; k,v -> pages
+//   attn    split-KV partial softmax per (row, KV head, split); the last split
+//           block of a (row, KV head) merges the partials
+//   oproj   x += W_o attn
+//   gateup  h = silu(W_gate n) * (W_up n), n = RMSNorm(x)
+//   down    x += W_down h
+// then lm_head: logits = W_lm RMSNorm(x_L) by warp ranges of the vocabulary,
+// each warp keeping (max, sum exp) and argmax of its range; the last block
+// picks the range that holds u * S, recomputes only that range's logits and
+// scans them in id order.  The logits never leave the chip unless asked for.
+#include <math.h>
+
+#include "common.cuh"
+#include "draft.cuh"
+#include "internal.h"
+
+namespace osp {
+
+constexpr int GT = 256;          // threads per GEMV / LM-head block
+constexpr int GW = GT / 32;      // warps per block
+constexpr int AT = 128;          // threads per attention block
+
+// ---------------------------------------------------------------------------
+// One warp computes TR dot products of length Kd (weights streamed from HBM,
+// 16 bytes per lane per load, NB loads per row in flight) against RG bf16
+// activation rows held in shared memory.  Every (row, activation) pair is
+// accumulated in the same order (ascending k, fmaf) whatever TR, NB and RG are,
+// so a recomputed logit is bitwise equal to the first one.
+template <int TR, int RG, int NB>
+__device__ __forceinline__ void warp_dot(const uint16_t *const (&w)[TR], const uint16_t *xs, int Kd,
+                                         float (&acc)[TR][RG]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int t = 0; t < TR; ++t)
+#pragma unroll
+        for (int r = 0; r < RG; ++r) acc[t][r] = 0.f;
+    for (int base = 0; base < Kd; base += NB * 256) {
+        uint4 wv[TR][NB];
+#pragma unroll
+        for (int i = 0; i < NB; ++i) {
+            const int k = base + i * 256 + lane * 8;
+#pragma unroll
+            for (int t = 0; t < TR; ++t)
+                wv[t][i] = (base + i * 256 < Kd) ? ld_stream(w[t] + k) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int i = 0; i < NB; ++i) {
+            if (base + i * 256 < Kd) {
+                const int k = base + i * 256 + lane * 8;
+                float wf[TR][8];
+#pragma unroll
+                for (int t = 0; t < TR; ++t) unpack8(wv[t][i], wf[t]);
+#pragma unroll
+                for (int r = 0; r < RG; ++r) {
+                    float xf[8];
+                    unpack8(*(const uint4 *)(xs + (size_t)r * Kd + k), xf);
+#pragma unroll
+                    for (int t = 0; t < TR; ++t)
+#pragma unroll
+                        for (int e = 0; e < 8; ++e) acc[t][r] = fmaf(wf[t][e], xf[e], acc[t][r]);
+                }
+            }
+        }
+    }
+#pragma unroll
+    for (int t = 0; t < TR; ++t)
+#pragma unroll
+        for (int r = 0; r < RG; ++r) acc[t][r] = warp_sum(acc[t][r]);
+}
+
+// ---- prologue helpers -------------------------------------------------------------
+// dst[k] = bf16(src[k]) for a bf16 row (or zeros when src is null).
+__device__ __forceinline__ void stage_copy(uint16_t *dst, const uint16_t *src, int n) {
+    for (int c = threadIdx.x; c < n / 8; c += blockDim.x)
+        ((uint4 *)dst)[c] = src ? *((const uint4 *)src + c) : make_uint4(0, 0, 0, 0);
+}
+
+// dst[k] = bf16(x[k] / sqrt(mean(x^2) + eps) * gain[k]) (zeros when x is null).
+__device__ __forceinline__ void stage_rmsnorm(uint16_t *dst, const float *x, const uint16_t *gain,
+                                              int d, float eps, float *red) {
+    float ss = 0.f;
+    if (x)
+        for (int k = threadIdx.x; k < d; k += blockDim.x) {
+            float v = x[k];
+            ss = fmaf(v, v, ss);
+        }
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        float t = 0.f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+        red[32] = rsqrtf(t / (float)d + eps);
+    }
+    __syncthreads();
+    const float inv = red[32];
+    for (int k = threadIdx.x; k < d; k += blockDim.x)
+        dst[k] = x ? f_to_bf(x[k] * inv * bf_to_f(gain[k])) : (uint16_t)0;
+    __syncthreads();
+}
+
+__device__ __forceinline__ void rope_cs(double inv_freq, int pos, float &c, float &s) {
+    // angle reduced modulo 2*pi in double before the float sin/cos
+    const double turns = (double)pos * inv_freq * 0.15915494309189535;
+    const double frac = turns - floor(turns);
+    sincosf((float)(frac * 6.283185307179586), &s, &c);
+}
+
+// ---------------------------------------------------------------------------
+template <int MODE, int RG>
+__global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
+    extern __shared__ __align__(16) uint16_t xs[];
+    __shared__ float red[33];
+    __shared__ int s_b[RG], s_pos[RG], s_act[RG];
+    const Dims &D = a.dim;
+    const int r0 = blockIdx.y * RG;
+    if (threadIdx.x < RG) {
+        int b = 0, pos = 0;
+        const int r = r0 + threadIdx.x;
+        const bool act = r < a.R && a.map.row(r, b, pos);
+        s_b[threadIdx.x] = b;
+        s_pos[threadIdx.x] = pos;
+        s_act[threadIdx.x] = act;
+    }
+    __syncthreads();
+
+    int Kd, n_tasks;
+    if (MODE == G_FEAT) { Kd = D.feat; n_tasks = D.d; }
+    else if (MODE == G_QKV) { Kd = 2 * D.d; n_tasks = (D.Hq + 2 * D.Hkv) * D.hd / 2; }
+    else if (MODE == G_OPROJ) { Kd = D.Hq * D.hd; n_tasks = D.d; }
+    else if (MODE == G_GATEUP) { Kd = D.d; n_tasks = D.F; }
+    else { Kd = D.F; n_tasks = D.d; }
+
+    // ---- prologue: stage the activation rows (bf16) in shared memory
+    for (int rr = 0; rr < RG; ++rr) {
+        const int r = r0 + rr;
+        const bool act = s_act[rr];
+        uint16_t *row = xs + (size_t)rr * Kd;
+        if (MODE == G_FEAT) {
+            stage_copy(row, act ? a.feats + (size_t)r * D.feat : nullptr, Kd);
+            if (blockIdx.x == 0 && act) {     // residual stream of layer 0 starts at E[x]
+                const uint16_t *e = a.embed + (size_t)a.tokens[r] * D.d;
+                for (int k = threadIdx.x; k < D.d; k += blockDim.x) a.x[(size_t)r * D.d + k] = bf_to_f(e[k]);
+            }
+        } else if (MODE == G_QKV) {
+            stage_copy(row, act ? a.s + (size_t)r * D.d : nullptr, D.d);
+            stage_rmsnorm(row + D.d, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
+        } else if (MODE == G_OPROJ) {
+            stage_copy(row, act ? a.xin_bf + (size_t)r * Kd : nullptr, Kd);
+        } else if (MODE == G_GATEUP) {
+            stage_rmsnorm(row, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
+        } else {
+            stage_copy(row, act ? a.xin_bf + (size_t)r * Kd : nullptr, Kd);
+        }
+    }
+    __syncthreads();
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    for (int task = blockIdx.x * GW + warp; task < n_tasks; task += gridDim.x * GW) {
+        if (MODE == G_QKV || MODE == G_GATEUP) {
+            const uint16_t *w[2];
+            int h = 0, i = 0;
+            if (MODE == G_QKV) {
+                h = task / (D.hd / 2);
+                i = task % (D.hd / 2);
+                w[0] = a.W + ((size_t)h * D.hd + i) * Kd;
+                w[1] = a.W + ((size_t)h * D.hd + i + D.hd / 2) * Kd;
+            } else {
+                w[0] = a.W + (size_t)task * Kd;
+                w[1] = a.W2 + (size_t)task * Kd;
+            }
+            float acc[2][RG];
+            warp_dot<2, RG, 8>(w, xs, Kd, acc);
+#pragma unroll
+            for (int rr = 0; rr < RG; ++rr) {
+                if (lane != rr || !s_act[rr]) continue;
+                const int r = r0 + rr;
+                if (MODE == G_GATEUP) {
+                    const float g = acc[0][rr], u = acc[1][rr];
+                    a.out_bf[(size_t)r * D.F + task] = f_to_bf(g / (1.f + expf(-g)) * u);
+                } else {
+                    const int b = s_b[rr], pos = s_pos[rr];
+                    float x1 = acc[0][rr], x2 = acc[1][rr];
+                    if (h < D.Hq + D.Hkv) {       // rotary on q and k (rotate-half pairs)
+                        float c, s;
+                        rope_cs(a.inv_freq[i], pos, c, s);
+                        const float y1 = x1 * c - x2 * s, y2 = x2 * c + x1 * s;
+                        x1 = y1;
+                        x2 = y2;
+                    }
+                    if (h < D.Hq) {
+                        float *q = a.q + (size_t)r * D.Hq * D.hd + (size_t)h * D.hd;
+                        q[i] = x1;
+                        q[i + D.hd / 2] = x2;
+                    } else {
+                        const bool is_k = h < D.Hq + D.Hkv;
+                        const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
+                        const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
+                        uint16_t *dst = (is_k ? a.k_pages : a.v_pages) +
+                                        (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * D.hd;
+                        dst[i] = f_to_bf(x1);
+                        dst[i + D.hd / 2] = f_to_bf(x2);
+                    }
+                }
+            }
+        } else {
+            const uint16_t *w[1] = {a.W + (size_t)task * Kd};
+            float acc[1][RG];
+            warp_dot<1, RG, 16>(w, xs, Kd, acc);
+#pragma unroll
+            for (int rr = 0; rr < RG; ++rr) {
+                if (lane != rr || !s_act[rr]) continue;
+                const int r = r0 + rr;
+                if (MODE == G_FEAT) a.s[(size_t)r * D.d + task] = f_to_bf(acc[0][rr]);
+                else a.x[(size_t)r * D.d + task] += acc[0][rr];   // residual add (oproj, down)
+            }
+        }
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Split-KV GQA decode attention.  Block (split, kv head, row); 4 warps take the
+// split's pages round-robin.  HD/8 lanes share one key (8 dims, 16 bytes each).
+template <int HD, int G>
+__global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
+    constexpr int LPK = HD / 8;
+    constexpr int KPL = 32 / LPK;
+    constexpr int NIT = 16 / KPL;     // loads per page (16 positions)
+    __shared__ float sm_m[AT / 32][G], sm_l[AT / 32][G];
+    __shared__ float sm_acc[AT / 32][G][HD];
+    const Dims &D = a.dim;
+    const int split = blockIdx.x, kvh = blockIdx.y, r = blockIdx.z;
+    int b, pos;
+    if (!a.map.row(r, b, pos)) return;
+    const int n_keys = pos + 1;
+    const int k_begin = split * a.split_len;
+    const int k_end = min(n_keys, k_begin + a.split_len);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int kg = lane / LPK, dl = (lane % LPK) * 8;
+    const float scale = rsqrtf((float)HD);
+
+    float q[G][8], acc[G][8], m_run[G], l[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+        const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dl;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) { q[g][e] = qp[e] * scale; acc[g][e] = 0.f; }
+        m_run[g] = -INFINITY;
+        l[g] = 0.f;
+    }
+    const size_t head_stride = (size_t)D.P * HD;
+    for (int pg = k_begin / D.P + warp; pg * D.P < k_end; pg += AT / 32) {
+        const int page = a.page_table[(size_t)b * a.max_pages + pg];
+        const uint16_t *kb = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
+        const uint16_t *vb = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
+        uint4 kr[NIT], vr[NIT];
+#pragma unroll
+        for (int it = 0; it < NIT; ++it) {
+            const int slot = it * KPL + kg;
+            kr[it] = ld_stream(kb + slot * HD + dl);
+            vr[it] = ld_stream(vb + slot * HD + dl);
+        }
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            float sc[NIT];
+            float mx = -INFINITY;
+#pragma unroll
+            for (int it = 0; it < NIT; ++it) {
+                float kf[8];
+                unpack8(kr[it], kf);
+                float p = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) p = fmaf(q[g][e], kf[e], p);
+#pragma unroll
+                for (int o = LPK / 2; o; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
+                const int key = pg * D.P + it * KPL + kg;
+                sc[it] = key < k_end ? p : -INFINITY;
+                mx = fmaxf(mx, sc[it]);
+            }
+#pragma unroll
+            for (int o = LPK; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            const float m_new = fmaxf(m_run[g], mx);
+            const float corr = __expf(m_run[g] - m_new);
+            l[g] *= corr;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[g][e] *= corr;
+#pragma unroll
+            for (int it = 0; it < NIT; ++it) {
+                const float p = __expf(sc[it] - m_new);
+                float vf[8];
+                unpack8(vr[it], vf);
+                l[g] += p;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p, vf[e], acc[g][e]);
+            }
+            m_run[g] = m_new;
+        }
+    }
+    // merge the key groups of the warp, then the warps of the block
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+#pragma unroll
+        for (int o = LPK; o < 32; o <<= 1) {
+            l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[g][e] += __shfl_xor_sync(0xffffffffu, acc[g][e], o);
+        }
+        if (lane < LPK) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) sm_acc[warp][g][dl + e] = acc[g][e];
+        }
+        if (lane == 0) { sm_m[warp][g] = m_run[g]; sm_l[warp][g] = l[g]; }
+    }
+    __syncthreads();
+    const int Hq = D.Hq;
+    for (int idx = threadIdx.x; idx < G * HD; idx += AT) {
+        const int g = idx / HD, dim = idx % HD;
+        float M = -INFINITY;
+        for (int w = 0; w < AT / 32; ++w) M = fmaxf(M, sm_m[w][g]);
+        float num = 0.f, den = 0.f;
+        if (M != -INFINITY)
+            for (int w = 0; w < AT / 32; ++w) {
+                const float f = __expf(sm_m[w][g] - M);
+                num = fmaf(f, sm_acc[w][g][dim], num);
+                den = fmaf(f, sm_l[w][g], den);
+            }
+        float *pp = a.part + (((size_t)r * Hq + kvh * G + g) * a.n_splits + split) * (HD + 2);
+        pp[2 + dim] = num;
+        if (dim == 0) { pp[0] = M; pp[1] = den; }
+    }
+    if (!arrive_last(a.ticket + (size_t)r * D.Hkv + kvh, a.n_splits)) return;
+    for (int idx = threadIdx.x; idx < G * HD; idx += AT) {
+        const int g = idx / HD, dim = idx % HD;
+        const float *pp = a.part + ((size_t)r * Hq + kvh * G + g) * a.n_splits * (HD + 2);
+        float M = -INFINITY;
+        for (int s = 0; s < a.n_splits; ++s) M = fmaxf(M, __ldcg(pp + (size_t)s * (HD + 2)));
+        float num = 0.f, den = 0.f;
+        for (int s = 0; s < a.n_splits; ++s) {
+            const float ms = __ldcg(pp + (size_t)s * (HD + 2));
+            if (ms == -INFINITY) continue;
+            const float f = __expf(ms - M);
+            num = fmaf(f, __ldcg(pp + (size_t)s * (HD + 2) + 2 + dim), num);
+            den = fmaf(f, __ldcg(pp + (size_t)s * (HD + 2) + 1), den);
+        }
+        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = f_to_bf(num / den);
+    }
+}
+
+// ---------------------------------------------------------------------------
+// LM head + on-chip sampling.
+__device__ __forceinline__ void warp_range(int V, int warps_total, int gw, int &lo, int &hi) {
+    lo = (int)(((long long)V * gw) / warps_total);
+    hi = (int)(((long long)V * (gw + 1)) / warps_total);
+}
+
+template <int RG>
+__device__ void lm_sample(const LmArgs &a, int b, int rr, int src_row, const uint16_t *xs,
+                          float *ybuf) {
+    __shared__ MS shm[GW];
+    __shared__ AM sha[GW];
+    __shared__ float sh_scan[33];
+    __shared__ int s_pick, s_last, s_tok;
+    __shared__ float s_before, s_before_last, s_e;
+    const Dims &D = a.dim;
+    const int V = D.V, Wt = a.warps_total;
+    const bool greedy = a.temperature == 0.f;
+    const float invT = greedy ? 1.f : 1.f / a.temperature;
+    const float4 *st = a.warp_stats + (size_t)b * Wt;
+    const int per = (Wt + GT - 1) / GT;
+    const int e0 = threadIdx.x * per, e1 = min(Wt, e0 + per);
+
+    MS ms{-INFINITY, 0.f};
+    AM am{-INFINITY, 0x7fffffff};
+    for (int e = e0; e < e1; ++e) {
+        const float4 v = __ldcg(st + e);
+        ms = ms_combine(ms, MS{v.x, v.y});
+        am = am_combine(am, AM{v.z, __float_as_int(v.w)});
+    }
+    const MS tot = block_ms(ms, shm);
+    const AM best = block_am(am, sha);
+    const float M = tot.m;
+    int token;
+    float qx, S;
+    if (greedy) {
+        token = best.i;
+        qx = 1.f;
+        S = tot.s;
+    } else {
+        // contributions of the warp ranges, in id order
+        float mine = 0.f;
+        for (int e = e0; e < e1; ++e) {
+            const float4 v = __ldcg(st + e);
+            mine += v.x == -INFINITY ? 0.f : v.y * __expf(v.x - M);
+        }
+        float Ssum;
+        const float ex = block_excl_scan(mine, sh_scan, &Ssum);
+        S = Ssum;
+        const float t = a.u_draft[(size_t)b * a.K + a.step] * S;
+        if (threadIdx.x == 0) { s_pick = 0x7fffffff; s_last = -1; }
+        __syncthreads();
+        float run = ex;
+        int found = 0x7fffffff, lastpos = -1;
+        float before = 0.f, before_last = 0.f;
+        for (int e = e0; e < e1; ++e) {
+            const float4 v = __ldcg(st + e);
+            const float c = v.x == -INFINITY ? 0.f : v.y * __expf(v.x - M);
+            if (c > 0.f) { lastpos = e; before_last = run; }
+            if (found == 0x7fffffff && c > 0.f && t < run + c) { found = e; before = run; }
+            run += c;
+        }
+        atomicMin(&s_pick, found);
+        atomicMax(&s_last, lastpos);
+        __syncthreads();
+        if (found != 0x7fffffff && found == s_pick) s_before = before;
+        if (s_pick == 0x7fffffff && lastpos >= 0 && lastpos == s_last) s_before_last = before_last;
+        __syncthreads();
+        const int pick = s_pick != 0x7fffffff ? s_pick : s_last;
+        const float cbefore = s_pick != 0x7fffffff ? s_before : s_before_last;
+        // recompute the chosen range's logits (same arithmetic as the first pass)
+        int lo, hi;
+        warp_range(V, Wt, pick, lo, hi);
+        const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+        for (int n = lo + warp; n < hi; n += GW) {
+            const uint16_t *w[1] = {a.W + (size_t)n * D.d};
+            float acc[1][RG];
+            warp_dot<1, RG, 16>(w, xs, D.d, acc);
+            if (lane == 0) ybuf[n - lo] = acc[0][rr] * invT;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            float run2 = cbefore;
+            int tok = -1, lastp = -1;
+            float etok = 0.f, elast = 0.f;
+            for (int base = lo; base < hi && tok < 0; base += 32) {
+                const int n = base + lane;
+                const float e = n < hi ? __expf(ybuf[n - lo] - M) : 0.f;
+                const float inc = warp_incl_scan(e) + run2;
+                const unsigned hit = __ballot_sync(0xffffffffu, n < hi && e > 0.f && t < inc);
+                const unsigned pos = __ballot_sync(0xffffffffu, n < hi && e > 0.f);
+                if (pos) {
+                    const int l2 = 31 - __clz(pos);
+                    lastp = base + l2;
+                    elast = __shfl_sync(0xffffffffu, e, l2);
+                }
+                if (hit) {
+                    const int l2 = __ffs(hit) - 1;
+                    tok = base + l2;
+                    etok = __shfl_sync(0xffffffffu, e, l2);
+                }
+                run2 = __shfl_sync(0xffffffffu, inc, 31);
+            }
+            if (lane == 0) {
+                if (tok < 0) { tok = lastp >= 0 ? lastp : lo; etok = elast; }
+                s_tok = tok;
+                s_e = etok;
+            }
+        }
+        __syncthreads();
+        token = s_tok;
+        qx = s_e / S;
+    }
+    if (threadIdx.x == 0) {
+        a.tokens[(size_t)b * a.K + a.step] = token;
+        if (a.qx) a.qx[(size_t)b * a.K + a.step] = qx;
+        if (a.stats) {
+            a.stats[((size_t)b * a.K + a.step) * 2 + 0] = M;
+            a.stats[((size_t)b * a.K + a.step) * 2 + 1] = logf(S);
+        }
+    }
+    if (a.step + 1 < a.K) {
+        // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[token]
+        const float *xl = a.x_in + (size_t)src_row * D.d;
+        for (int k = threadIdx.x; k < D.d; k += blockDim.x)
+            a.s_chain[(size_t)b * D.d + k] = f_to_bf(xl[k]);
+        __syncthreads();
+        const uint16_t *e = a.embed + (size_t)token * D.d;
+        for (int k = threadIdx.x; k < D.d; k += blockDim.x)
+            a.x_chain[(size_t)b * D.d + k] = bf_to_f(e[k]);
+    }
+    __syncthreads();
+}
+
+template <int RG>
+__global__ void __launch_bounds__(GT) lm_head_kernel(const LmArgs a) {
+    extern __shared__ __align__(16) uint16_t xs[];   // [RG][d] bf16, then the range's logits
+    __shared__ float red[33];
+    __shared__ int s_src[RG], s_act[RG];
+    const Dims &D = a.dim;
+    const int b0 = blockIdx.y * RG;
+    if (threadIdx.x < RG) {
+        const int b = b0 + threadIdx.x;
+        const bool act = b < a.B && a.map.valid[b];
+        s_act[threadIdx.x] = act;
+        s_src[threadIdx.x] = act ? (a.src_is_ext ? b * a.max_new + a.map.nnew[b] - 1 : b) : 0;
+    }
+    __syncthreads();
+    for (int rr = 0; rr < RG; ++rr)
+        stage_rmsnorm(xs + (size_t)rr * D.d, s_act[rr] ? a.x_in + (size_t)s_src[rr] * D.d : nullptr,
+                      a.gain, D.d, D.eps, red);
+    float *ybuf = (float *)(xs + (size_t)RG * D.d);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int gw = blockIdx.x * GW + warp;
+    int lo, hi;
+    warp_range(D.V, a.warps_total, gw, lo, hi);
+    const float invT = a.temperature == 0.f ? 1.f : 1.f / a.temperature;
+    float m[RG], s[RG], bv[RG];
+    int bi[RG];
+#pragma unroll
+    for (int rr = 0; rr < RG; ++rr) { m[rr] = -INFINITY; s[rr] = 0.f; bv[rr] = -INFINITY; bi[rr] = 0x7fffffff; }
+    auto consume = [&](int n, int rr, float z) {
+        if (a.logits && lane == 0 && s_act[rr])
+            a.logits[((size_t)(b0 + rr) * a.K + a.step) * D.V + n] = z;
+        const float y = z * invT;
+        if (y > m[rr]) { s[rr] = s[rr] * __expf(m[rr] - y) + 1.f; m[rr] = y; }
+        else s[rr] += __expf(y - m[rr]);
+        if (z > bv[rr]) { bv[rr] = z; bi[rr] = n; }
+    };
+    int n = lo;
+    for (; n + 4 <= hi; n += 4) {
+        const uint16_t *w[4] = {a.W + (size_t)n * D.d, a.W + (size_t)(n + 1) * D.d,
+                                a.W + (size_t)(n + 2) * D.d, a.W + (size_t)(n + 3) * D.d};
+        float acc[4][RG];
+        warp_dot<4, RG, 4>(w, xs, D.d, acc);
+#pragma unroll
+        for (int t = 0; t < 4; ++t)
+#pragma unroll
+            for (int rr = 0; rr < RG; ++rr) consume(n + t, rr, acc[t][rr]);
+    }
+    for (; n < hi; ++n) {
+        const uint16_t *w[1] = {a.W + (size_t)n * D.d};
+        float acc[1][RG];
+        warp_dot<1, RG, 16>(w, xs, D.d, acc);
+#pragma unroll
+        for (int rr = 0; rr < RG; ++rr) consume(n, rr, acc[0][rr]);
+    }
+    if (lane == 0) {
+#pragma unroll
+        for (int rr = 0; rr < RG; ++rr)
+            if (b0 + rr < a.B)
+                a.warp_stats[(size_t)(b0 + rr) * a.warps_total + gw] =
+                    make_float4(m[rr], s[rr], bv[rr], __int_as_float(bi[rr]));
+    }
+    if (!arrive_last(a.ticket + blockIdx.y, gridDim.x)) return;
+    for (int rr = 0; rr < RG; ++rr)
+        if (s_act[rr]) lm_sample<RG>(a, b0 + rr, rr, s_src[rr], xs, ybuf);
+}
+
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(128) prepare_kernel(const PrepArgs a) {
+    __shared__ int ok, code;
+    const int b = blockIdx.x;
+    const int L0 = a.seq_len[b], nn = a.n_new[b];
+    if (threadIdx.x == 0) {
+        const bool n_ok = nn >= 1 && nn <= a.max_new;
+        const bool cap = L0 >= 0 && (long long)L0 + nn + a.K - 1 <= (long long)a.max_pages * a.P;
+        ok = n_ok && cap;
+        code = !n_ok ? OSPREY_ERR_INVALID_ARG : (!cap ? OSPREY_ERR_CAPACITY : 0);
+    }
+    __syncthreads();
+    if (ok) {
+        const int npages = (L0 + nn + a.K - 1 + a.P - 1) / a.P;
+        for (int pg = threadIdx.x; pg < npages; pg += blockDim.x) {
+            const int page = a.page_table[(size_t)b * a.max_pages + pg];
+            if (page < 0 || page >= a.n_pages) { ok = 0; atomicCAS(&code, 0, OSPREY_ERR_CAPACITY); }
+        }
+        for (int j = threadIdx.x; j < nn; j += blockDim.x) {
+            const int t = a.tokens[(size_t)b * a.max_new + j];
+            if (t < 0 || t >= a.V) { ok = 0; atomicCAS(&code, 0, OSPREY_ERR_INVALID_ARG); }
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        a.valid[b] = ok;
+        a.pos0[b] = L0;
+        a.nnew[b] = nn;
+        if (ok) a.seq_len[b] = L0 + nn;
+        else set_status(a.status, code);
+    }
+    if (!ok)
+        for (int k = threadIdx.x; k < a.K; k += blockDim.x) a.draft_tokens[(size_t)b * a.K + k] = -1;
+}
+
+// ---------------------------------------------------------------------------
+// host side
+
+int attn_splits(int R, int Hkv, int max_ctx, int sms) {
+    auto cdiv = [](long long x, long long y) { return (int)((x + y - 1) / y); };
+    int want = cdiv(4LL * sms, (long long)R * Hkv);
+    int by_len = cdiv(max_ctx, 1024);
+    int s = want > by_len ? want : by_len;
+    int cap = cdiv(max_ctx, 32);
+    if (s > cap) s = cap;
+    return s < 1 ? 1 : s;
+}
+
+int attn_split_len(int max_ctx, int n_splits) {
+    int len = (max_ctx + n_splits - 1) / n_splits;
+    return (len + 15) / 16 * 16;
+}
+
+int lm_blocks(int V, int sms) {
+    int want = 2 * sms;
+    int cap = (V + GW * 16 - 1) / (GW * 16);   // at least ~16 rows per warp range
+    return want < cap ? want : (cap < 1 ? 1 : cap);
+}
+
+static int gemv_kd(GemvMode mode, const Dims &d) {
+    switch (mode) {
+    case G_FEAT: return d.feat;
+    case G_QKV: return 2 * d.d;
+    case G_OPROJ: return d.Hq * d.hd;
+    case G_GATEUP: return d.d;
+    default: return d.F;
+    }
+}
+
+int gemv_rg(GemvMode mode, const Dims &d, int R) {
+    int rg = 1;
+    while (rg < R && rg < 8) rg <<= 1;
+    const size_t limit = 200 * 1024;
+    while (rg > 1 && (size_t)rg * gemv_kd(mode, d) * 2 > limit) rg >>= 1;
+    return rg;
+}
+
+size_t gemv_smem(GemvMode mode, const Dims &d, int rg) { return (size_t)rg * gemv_kd(mode, d) * 2; }
+
+template <int MODE>
+static cudaError_t launch_gemv_m(const GemvArgs &a, int rg, int sms, cudaStream_t s) {
+    const Dims &D = a.dim;
+    int n_tasks;
+    if (MODE == G_QKV) n_tasks = (D.Hq + 2 * D.Hkv) * D.hd / 2;
+    else if (MODE == G_GATEUP) n_tasks = D.F;
+    else n_tasks = D.d;
+    int blocks = (n_tasks + GW - 1) / GW;
+    if (blocks > 4 * sms) blocks = 4 * sms;
+    const int groups = (a.R + rg - 1) / rg;
+    const size_t smem = gemv_smem((GemvMode)MODE, D, rg);
+    dim3 grid(blocks, groups);
+    switch (rg) {
+    case 1: gemv_kernel<MODE, 1><<<grid, GT, smem, s>>>(a); break;
+    case 2: gemv_kernel<MODE, 2><<<grid, GT, smem, s>>>(a); break;
+    case 4: gemv_kernel<MODE, 4><<<grid, GT, smem, s>>>(a); break;
+    default: gemv_kernel<MODE, 8><<<grid, GT, smem, s>>>(a); break;
+    }
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaStream_t s) {
+    switch (mode) {
+    case G_FEAT: return launch_gemv_m<G_FEAT>(a, rg, sms, s);
+    case G_QKV: return launch_gemv_m<G_QKV>(a, rg, sms, s);
+    case G_OPROJ: return launch_gemv_m<G_OPROJ>(a, rg, sms, s);
+    case G_GATEUP: return launch_gemv_m<G_GATEUP>(a, rg, sms, s);
+    default: return launch_gemv_m<G_DOWN>(a, rg, sms, s);
+    }
+}
+
+cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s) {
+    dim3 grid(a.n_splits, a.dim.Hkv, a.R);
+    const int G = a.dim.Hq / a.dim.Hkv;
+    if (a.dim.hd == 128) {
+        switch (G) {
+        case 1: attn_kernel<128, 1><<<grid, AT, 0, s>>>(a); break;
+        case 2: attn_kernel<128, 2><<<grid, AT, 0, s>>>(a); break;
+        case 4: attn_kernel<128, 4><<<grid, AT, 0, s>>>(a); break;
+        default: attn_kernel<128, 8><<<grid, AT, 0, s>>>(a); break;
+        }
+    } else {
+        switch (G) {
+        case 1: attn_kernel<64, 1><<<grid, AT, 0, s>>>(a); break;
+        case 2: attn_kernel<64, 2><<<grid, AT, 0, s>>>(a); break;
+        case 4: attn_kernel<64, 4><<<grid, AT, 0, s>>>(a); break;
+        default: attn_kernel<64, 8><<<grid, AT, 0, s>>>(a); break;
+        }
+    }
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_lm(const LmArgs &a, int rg, int blocks, cudaStream_t s) {
+    const int groups = (a.B + rg - 1) / rg;
+    const int range_max = (a.dim.V + a.warps_total - 1) / a.warps_total + 1;
+    const size_t smem = (size_t)rg * a.dim.d * 2 + (size_t)range_max * 4;
+    dim3 grid(blocks, groups);
+    switch (rg) {
+    case 1: lm_head_kernel<1><<<grid, GT, smem, s>>>(a); break;
+    case 2: lm_head_kernel<2><<<grid, GT, smem, s>>>(a); break;
+    case 4: lm_head_kernel<4><<<grid, GT, smem, s>>>(a); break;
+    default: lm_head_kernel<8><<<grid, GT, smem, s>>>(a); break;
+    }
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s) {
+    prepare_kernel<<<a.B, 128, 0, s>>>(a);
+    count_launch();
+    return cudaGetLastError();
+}
+
+template <int MODE>
+static cudaError_t set_gemv_attr() {
+    const int mx = 227 * 1024;
+    cudaError_t e;
+    if ((e = cudaFuncSetAttribute(gemv_kernel<MODE, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
+    if ((e = cudaFuncSetAttribute(gemv_kernel<MODE, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
+    if ((e = cudaFuncSetAttribute(gemv_kernel<MODE, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
+    return cudaFuncSetAttribute(gemv_kernel<MODE, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+}
+
+cudaError_t draft_set_attributes() {
+    cudaError_t e;
+    if ((e = set_gemv_attr<G_FEAT>())) return e;
+    if ((e = set_gemv_attr<G_QKV>())) return e;
+    if ((e = set_gemv_attr<G_OPROJ>())) return e;
+    if ((e = set_gemv_attr<G_GATEUP>())) return e;
+    if ((e = set_gemv_attr<G_DOWN>())) return e;
+    const int mx = 227 * 1024;
+    if ((e = cudaFuncSetAttribute(lm_head_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
+    if ((e = cudaFuncSetAttribute(lm_head_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
+    if ((e = cudaFuncSetAttribute(lm_head_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
+    return cudaFuncSetAttribute(lm_head_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+}
+
+}  // namespace osp

@@ -1,0 +1,128 @@
+// Draft-step kernel interface (CUDA-core GEMV path for up to 8 rows per group).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "osprey.h"
+
+namespace osp {
+
+struct Dims {
+    int d, L, Hq, Hkv, hd, F, V, feat, P;
+    float eps;
+};
+
+// Workspace views of one draft call.
+struct DraftWs {
+    int *seq_valid, *seq_pos0, *seq_nnew;  // [B]
+    int *attn_ticket;                      // [R_ext * Hkv]
+    int *lm_ticket;                        // [groups]
+    float *x_ext;                          // [B*max_new][d]  residual stream, extend rows
+    uint16_t *s_ext;                       // [B*max_new][d]  context slot (c), bf16
+    float *x_chain;                        // [B][d]          residual stream, chain rows
+    uint16_t *s_chain;                     // [B][d]          context slot (fed-back x_L), bf16
+    float *q;                              // [R_ext][Hq*hd]  rotated queries
+    float *attn_part;                      // [R_ext][Hq][n_splits][hd+2]
+    uint16_t *attn_out;                    // [R_ext][Hq*hd]
+    uint16_t *ffn_h;                       // [R_ext][F]
+    float4 *lm_stats;                      // [B][lm_warps]
+    int n_splits_max, lm_warps_max;
+};
+
+// Which rows a launch works on: extend rows (step 0, rows_per_seq = max_new,
+// row r = b*max_new + j, active for j < n_new[b]) or the chain row of step k
+// (rows_per_seq = 1, row r = b, position pos0 + n_new + k - 1).
+struct RowMap {
+    const int *valid, *pos0, *nnew;
+    int rows_per_seq, step;
+    __device__ __forceinline__ bool row(int r, int &b, int &pos) const {
+        b = r / rows_per_seq;
+        const int j = r - b * rows_per_seq;
+        if (!valid[b]) return false;
+        const int nn = nnew[b];
+        if (step == 0) {
+            if (j >= nn) return false;
+            pos = pos0[b] + j;
+        } else {
+            pos = pos0[b] + nn + step - 1;
+        }
+        return true;
+    }
+};
+
+struct GemvArgs {
+    Dims dim;
+    RowMap map;
+    int R;                        // rows of this step (B * rows_per_seq)
+    const uint16_t *W, *W2;       // weight matrix (and the up matrix for gate/up)
+    const uint16_t *gain;         // RMSNorm gain of the prologue (qkv, gate/up)
+    const uint16_t *embed;        // feature projection: embedding gather
+    const int32_t *tokens;        // [B][max_new]
+    const uint16_t *feats;        // [B][max_new][feat]
+    int max_new;
+    float *x;                     // residual stream of this step
+    uint16_t *s;                  // context slot of this step
+    const uint16_t *xin_bf;       // bf16 activation input (attn_out / ffn_h)
+    uint16_t *out_bf;             // bf16 output (s_ext / ffn_h / attn partial input)
+    float *q;                     // rotated queries
+    uint16_t *k_pages, *v_pages;  // this layer's pages
+    const int32_t *page_table;
+    int max_pages, n_pages;
+    double inv_freq[64];          // theta^(-2i/hd)
+};
+
+struct AttnArgs {
+    Dims dim;
+    RowMap map;
+    int R, n_splits, split_len;
+    const float *q;
+    const uint16_t *k_pages, *v_pages;
+    const int32_t *page_table;
+    int max_pages;
+    float *part;
+    uint16_t *out;
+    int *ticket;
+};
+
+struct LmArgs {
+    Dims dim;
+    RowMap map;
+    int B, K, step, max_new;
+    const uint16_t *W, *gain, *embed;
+    const float *x_in;            // residual of the step's rows (x_ext or x_chain)
+    int src_is_ext;               // extend step: read row b*max_new + n_new[b] - 1
+    float *x_chain;
+    uint16_t *s_chain;
+    float temperature;
+    const float *u_draft;
+    int32_t *tokens;
+    float *qx, *stats, *logits;
+    float4 *warp_stats;
+    int *ticket;
+    int warps_total;              // gridDim.x * 8 (stats entries per row)
+};
+
+struct PrepArgs {
+    int B, K, max_new, max_pages, n_pages, P, V;
+    int32_t *seq_len;
+    const int32_t *n_new, *tokens, *page_table;
+    int *valid, *pos0, *nnew;
+    int32_t *draft_tokens;
+    int32_t *status;
+};
+
+enum GemvMode { G_FEAT = 0, G_QKV = 1, G_OPROJ = 2, G_GATEUP = 3, G_DOWN = 4 };
+
+cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s);
+cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaStream_t s);
+cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s);
+cudaError_t launch_lm(const LmArgs &a, int rg, int blocks, cudaStream_t s);
+int attn_splits(int R, int Hkv, int max_ctx, int sms);
+int attn_split_len(int max_ctx, int n_splits);
+int lm_blocks(int V, int sms);
+size_t gemv_smem(GemvMode mode, const Dims &d, int rg);
+int gemv_rg(GemvMode mode, const Dims &d, int R);
+cudaError_t draft_set_attributes();
+
+}  // namespace osp

@@ -1,0 +1,50 @@
+// Launchers shared between the C-ABI translation unit and the kernel units.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "osprey.h"
+
+namespace osp {
+
+// Counts every kernel the library launches (or captures), for measurement.
+void count_launch(int n = 1);
+
+// ---------------------------------------------------------------- verify
+struct VerifyArgs {
+    int B, K, V, dtype;
+    float temperature;
+    const void *target, *draft;
+    const int32_t *tokens;
+    const float *u_accept, *u_sample;
+    int32_t *out_tokens, *n_accepted;
+    uint8_t *flags;
+    float *probs;
+    int32_t *status;
+    // workspace views
+    void *part;     // [B][K+1][nch] 16-byte partials
+    void *dec;      // [B] decisions
+    void *csum;     // [B][nch] float2 chunk sums
+    int *ticket1;   // [B]
+    int *ticket2;   // [B]
+    int nch;
+};
+size_t verify_workspace_layout(int B, int K, int V, VerifyArgs *a, void *base);
+cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s);
+
+// ---------------------------------------------------------------- kv append
+struct KvAppendArgs {
+    void *k_pages, *v_pages;
+    const int32_t *page_table;
+    int32_t *seq_len;
+    const int32_t *n_rows;
+    const void *k_rows, *v_rows;
+    int64_t total_rows;
+    int B, L, Hkv, hd, P, max_pages, n_pages;
+    int32_t *status;
+};
+cudaError_t launch_kv_append(const KvAppendArgs &a, cudaStream_t s);
+
+}  // namespace osp

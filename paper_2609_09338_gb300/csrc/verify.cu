@@ -1,0 +1,413 @@
+// Speculative-sampling verification (Sec. 3.1: the unmodified rule of
+// Leviathan et al.) as two streaming kernels.
+//
+// verify_stats: one block per (vocab chunk, row i, sequence b) reads the chunk
+//   of target row i and, for i < K, of draft row i exactly once with 16-byte
+//   coalesced loads, and publishes (max, sum exp) of logits/T for both (argmax
+//   in greedy mode).  The last block of a sequence to finish (atomic ticket, no
+//   waiting) combines the partials into the row normalisers, evaluates
+//   p_i(x_i), q_i(x_i), runs the acceptance chain and fixes the decision row r.
+// verify_sample (sampled mode only): one block per (vocab chunk, sequence)
+//   re-reads only row r and sums the weights max(0, p_r - q_r) (or p_K for the
+//   bonus) per chunk; the last block picks the chunk holding u * S and scans it
+//   in id order for the token.
+#include <float.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+
+namespace osp {
+
+constexpr int VT = 256;                 // threads per block
+constexpr int VCHUNK = 8192;            // logits of one row per block
+constexpr int VPER = VCHUNK / VT;       // logits per thread
+
+struct Decision {
+    int r;          // first rejected position (K = all accepted), -1 = invalid sequence
+    float Mp, Sp;   // normalisers of target row r (logits / T)
+    float Mq, Sq;   // of draft row r (r < K)
+    int pad[3];
+};
+
+template <typename T> struct Vec;
+template <> struct Vec<float> { static constexpr int W = 4; };
+template <> struct Vec<uint16_t> { static constexpr int W = 8; };
+
+__device__ __forceinline__ float to_f(float x) { return x; }
+__device__ __forceinline__ float to_f(uint16_t x) { return bf_to_f(x); }
+
+// Element index of value j (0..VPER-1) of this thread inside its chunk: the
+// thread's vectors are strided across the block so every load is coalesced.
+template <typename T, bool VEC>
+__device__ __forceinline__ int chunk_index(int j) {
+    constexpr int W = VEC ? Vec<T>::W : 1;
+    return ((j / W) * VT + threadIdx.x) * W + (j % W);
+}
+
+// Load this thread's VPER values of a chunk; positions past V read -inf.
+template <typename T, bool VEC>
+__device__ __forceinline__ void load_chunk(const T *row, int start, int V, float (&f)[VPER]) {
+    if (VEC) {
+        constexpr int W = Vec<T>::W;
+        constexpr int NV = VPER / W;
+        uint4 raw[NV];
+#pragma unroll
+        for (int it = 0; it < NV; ++it) {
+            int e = start + (it * VT + threadIdx.x) * W;
+            raw[it] = e < V ? ld_stream(row + e) : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int it = 0; it < NV; ++it) {
+            int e = start + (it * VT + threadIdx.x) * W;
+            if (W == 4) {
+                f[it * 4 + 0] = __uint_as_float(raw[it].x);
+                f[it * 4 + 1] = __uint_as_float(raw[it].y);
+                f[it * 4 + 2] = __uint_as_float(raw[it].z);
+                f[it * 4 + 3] = __uint_as_float(raw[it].w);
+            } else {
+                float g[8];
+                unpack8(raw[it], g);
+#pragma unroll
+                for (int j = 0; j < 8; ++j) f[it * 8 + j] = g[j];
+            }
+            if (e >= V) {
+#pragma unroll
+                for (int j = 0; j < W; ++j) f[it * W + j] = -INFINITY;
+            }
+        }
+    } else {
+#pragma unroll
+        for (int j = 0; j < VPER; ++j) {
+            int e = start + j * VT + threadIdx.x;
+            f[j] = e < V ? to_f(row[e]) : -INFINITY;
+        }
+    }
+}
+
+template <typename T, bool VEC>
+__device__ __forceinline__ int elem_index(int start, int j) {
+    return VEC ? start + chunk_index<T, true>(j) : start + j * VT + threadIdx.x;
+}
+
+__device__ __forceinline__ MS thread_ms(const float (&f)[VPER], float invT) {
+    float m = -INFINITY;
+#pragma unroll
+    for (int j = 0; j < VPER; ++j) m = fmaxf(m, f[j] * invT);
+    if (m == -INFINITY) return {m, 0.f};
+    float s = 0.f;
+#pragma unroll
+    for (int j = 0; j < VPER; ++j) s += __expf(f[j] * invT - m);
+    return {m, s};
+}
+
+__device__ __forceinline__ float ld_logit(const void *base, int dtype, size_t idx) {
+    return dtype == OSPREY_F32 ? __ldg((const float *)base + idx)
+                               : bf_to_f(__ldg((const uint16_t *)base + idx));
+}
+
+// The last block of sequence b: combine the partials of all K+1 rows, run the
+// acceptance chain and write everything but the token emitted at r.
+template <bool GREEDY>
+__device__ void decide(const VerifyArgs &a, int b) {
+    __shared__ float sMp[16], sSp[16], sMq[16], sSq[16];
+    __shared__ int sAm[16];
+    const int K = a.K, V = a.V, nch = a.nch;
+    const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const float4 *part = (const float4 *)a.part + (size_t)b * (K + 1) * nch;
+    for (int i = w; i <= K; i += VT / 32) {
+        if (GREEDY) {
+            AM am{-INFINITY, 0x7fffffff};
+            for (int c = lane; c < nch; c += 32) {
+                float4 p = __ldcg(part + (size_t)i * nch + c);
+                am = am_combine(am, AM{p.x, __float_as_int(p.y)});
+            }
+            am = warp_am(am);
+            if (lane == 0) sAm[i] = am.i;
+        } else {
+            MS p{-INFINITY, 0.f}, q{-INFINITY, 0.f};
+            for (int c = lane; c < nch; c += 32) {
+                float4 v = __ldcg(part + (size_t)i * nch + c);
+                p = ms_combine(p, MS{v.x, v.y});
+                q = ms_combine(q, MS{v.z, v.w});
+            }
+            p = warp_ms(p);
+            q = warp_ms(q);
+            if (lane == 0) {
+                sMp[i] = p.m; sSp[i] = p.s; sMq[i] = q.m; sSq[i] = q.s;
+            }
+        }
+    }
+    __syncthreads();
+    if (threadIdx.x != 0) return;
+    const int32_t *x = a.tokens + (size_t)b * K;
+    int32_t *out = a.out_tokens + (size_t)b * (K + 1);
+    uint8_t *fl = a.flags + (size_t)b * (K + 1);
+    Decision *dec = (Decision *)a.dec + b;
+    bool ok = true;
+    for (int i = 0; i < K; ++i) ok &= (x[i] >= 0 && x[i] < V);
+    for (int i = 0; i <= K; ++i) fl[i] = 0;
+    if (!ok) {
+        set_status(a.status, OSPREY_ERR_INVALID_ARG);
+        for (int i = 0; i <= K; ++i) out[i] = -1;
+        a.n_accepted[b] = 0;
+        dec->r = -1;
+        return;
+    }
+    int r = K;
+    if (GREEDY) {
+        for (int i = 0; i < K; ++i)
+            if (sAm[i] != x[i]) { r = i; break; }
+        for (int i = 0; i < r; ++i) out[i] = x[i];
+        out[r] = sAm[r];
+    } else {
+        const float invT = 1.f / a.temperature;
+        for (int i = 0; i < K; ++i) {
+            size_t rowp = ((size_t)b * (K + 1) + i) * V, rowq = ((size_t)b * K + i) * V;
+            float px = expf(ld_logit(a.target, a.dtype, rowp + x[i]) * invT - sMp[i]) / sSp[i];
+            float qx = expf(ld_logit(a.draft, a.dtype, rowq + x[i]) * invT - sMq[i]) / sSq[i];
+            if (a.probs) {
+                a.probs[((size_t)b * K + i) * 2 + 0] = px;
+                a.probs[((size_t)b * K + i) * 2 + 1] = qx;
+            }
+            if (r == K && !(a.u_accept[(size_t)b * K + i] < px / qx)) r = i;
+        }
+        for (int i = 0; i < r; ++i) out[i] = x[i];
+        out[r] = -1;  // written by verify_sample
+        dec->r = r;
+        dec->Mp = sMp[r]; dec->Sp = sSp[r];
+        dec->Mq = r < K ? sMq[r] : 0.f;
+        dec->Sq = r < K ? sSq[r] : 1.f;
+    }
+    for (int i = r + 1; i <= K; ++i) out[i] = -1;
+    a.n_accepted[b] = r;
+}
+
+template <typename T, bool VEC, bool GREEDY>
+__global__ void __launch_bounds__(VT) verify_stats(VerifyArgs a) {
+    __shared__ MS shm[VT / 32];
+    __shared__ AM sha[VT / 32];
+    // flattened grid: x = (b * (K+1) + i) * nch + c
+    const int K = a.K, V = a.V;
+    const int c = (int)(blockIdx.x % a.nch);
+    const int i = (int)((blockIdx.x / a.nch) % (K + 1));
+    const int b = (int)(blockIdx.x / ((unsigned)a.nch * (K + 1)));
+    const int start = c * VCHUNK;
+    const T *zp = (const T *)a.target + ((size_t)b * (K + 1) + i) * V;
+    float4 *part = (float4 *)a.part + ((size_t)b * (K + 1) + i) * a.nch + c;
+    if (GREEDY) {
+        float f[VPER];
+        load_chunk<T, VEC>(zp, start, V, f);
+        AM am{-INFINITY, 0x7fffffff};
+#pragma unroll
+        for (int j = 0; j < VPER; ++j) am = am_combine(am, AM{f[j], elem_index<T, VEC>(start, j)});
+        am = block_am(am, sha);
+        if (threadIdx.x == 0) *part = make_float4(am.v, __int_as_float(am.i), 0.f, 0.f);
+    } else {
+        const float invT = 1.f / a.temperature;
+        float f[VPER], g[VPER];
+        load_chunk<T, VEC>(zp, start, V, f);
+        const bool has_q = i < K;
+        if (has_q) load_chunk<T, VEC>((const T *)a.draft + ((size_t)b * K + i) * V, start, V, g);
+        MS p = block_ms(thread_ms(f, invT), shm);
+        MS q{-INFINITY, 0.f};
+        if (has_q) q = block_ms(thread_ms(g, invT), shm);
+        if (threadIdx.x == 0) *part = make_float4(p.m, p.s, q.m, q.s);
+    }
+    if (arrive_last(a.ticket1 + b, a.nch * (K + 1))) decide<GREEDY>(a, b);
+}
+
+// Weight of id e in the decision row's draw: max(0, p - q) (residual) or p.
+__device__ __forceinline__ float sample_weight(float zp, float zq, const Decision &d, float invT,
+                                               bool residual, bool use_p) {
+    float p = __expf(zp * invT - d.Mp) * (1.f / d.Sp);
+    if (use_p || !residual) return p;
+    float q = __expf(zq * invT - d.Mq) * (1.f / d.Sq);
+    return fmaxf(0.f, p - q);
+}
+
+template <typename T, bool VEC>
+__global__ void __launch_bounds__(VT) verify_sample(VerifyArgs a) {
+    __shared__ float sh[33];
+    __shared__ float2 shs[VT / 32];
+    __shared__ int s_chunk, s_tok, s_flag;
+    __shared__ float s_t, s_before;
+    const int K = a.K, V = a.V, nch = a.nch;
+    const int c = (int)(blockIdx.x % nch), b = (int)(blockIdx.x / nch);
+    const Decision d = ((const Decision *)a.dec)[b];   // written by verify_stats
+    const float invT = 1.f / a.temperature;
+    const bool valid = d.r >= 0;
+    const int r = valid ? d.r : 0;
+    const bool residual = r < K;
+    const T *zp = (const T *)a.target + ((size_t)b * (K + 1) + r) * V;
+    const T *zq = residual ? (const T *)a.draft + ((size_t)b * K + r) * V : zp;
+    const int start = c * VCHUNK;
+    float2 *csum = (float2 *)a.csum + (size_t)b * nch;
+    if (valid) {
+        float f[VPER], g[VPER];
+        load_chunk<T, VEC>(zp, start, V, f);
+        if (residual) load_chunk<T, VEC>(zq, start, V, g);
+        float sw = 0.f, sp = 0.f;
+#pragma unroll
+        for (int j = 0; j < VPER; ++j) {
+            if (f[j] == -INFINITY) continue;
+            sw += sample_weight(f[j], residual ? g[j] : 0.f, d, invT, residual, false);
+            sp += sample_weight(f[j], 0.f, d, invT, false, true);
+        }
+        sw = warp_sum(sw);
+        sp = warp_sum(sp);
+        if ((threadIdx.x & 31) == 0) shs[threadIdx.x >> 5] = make_float2(sw, sp);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float2 t = make_float2(0.f, 0.f);
+            for (int w = 0; w < VT / 32; ++w) { t.x += shs[w].x; t.y += shs[w].y; }
+            csum[c] = t;
+        }
+    }
+    if (!arrive_last(a.ticket2 + b, nch) || !valid) return;
+
+    // ---- last block: choose the chunk, then the id inside it (ascending ids)
+    if (threadIdx.x < 32) {
+        const int lane = threadIdx.x;
+        float tot_w = 0.f;
+        for (int base = 0; base < nch; base += 32) {
+            float v = base + lane < nch ? __ldcg(&csum[base + lane].x) : 0.f;
+            tot_w += warp_sum(v);
+        }
+        const bool fallback = !(tot_w > 0.f) || !isfinite(tot_w);
+        float S = 0.f;
+        for (int base = 0; base < nch; base += 32) {
+            float v = base + lane < nch ? (fallback ? __ldcg(&csum[base + lane].y)
+                                                    : __ldcg(&csum[base + lane].x)) : 0.f;
+            S += warp_sum(v);
+        }
+        const float t = a.u_sample[(size_t)b * (K + 1) + r] * S;
+        float run = 0.f;
+        int chunk = -1, last_pos = 0;
+        float before = 0.f;
+        for (int base = 0; base < nch && chunk < 0; base += 32) {
+            float v = base + lane < nch ? (fallback ? __ldcg(&csum[base + lane].y)
+                                                    : __ldcg(&csum[base + lane].x)) : 0.f;
+            float inc = warp_incl_scan(v) + run;
+            unsigned hit = __ballot_sync(0xffffffffu, base + lane < nch && t < inc);
+            unsigned pos = __ballot_sync(0xffffffffu, base + lane < nch && v > 0.f);
+            if (pos) last_pos = base + 31 - __clz(pos);
+            if (hit) {
+                int l = __ffs(hit) - 1;
+                chunk = base + l;
+                before = __shfl_sync(0xffffffffu, inc - v, l);
+            }
+            run = __shfl_sync(0xffffffffu, inc, 31);
+        }
+        if (lane == 0) {
+            s_flag = fallback ? 8 : 0;
+            if (chunk < 0) {   // u*S past the last cumulative sum after rounding
+                chunk = last_pos;
+                s_flag |= 16;
+                before = 0.f;
+                for (int k2 = 0; k2 < chunk; ++k2)
+                    before += fallback ? __ldcg(&csum[k2].y) : __ldcg(&csum[k2].x);
+            }
+            s_chunk = chunk;
+            s_t = t;
+            s_before = before;
+            s_tok = 0x7fffffff;
+        }
+    }
+    __syncthreads();
+    const bool fallback = s_flag & 8;
+    // each thread scans a contiguous run of ids inside the chosen chunk
+    const int cs = s_chunk * VCHUNK;
+    const int e0 = cs + threadIdx.x * VPER;
+    float wv[VPER];
+    float mine = 0.f;
+#pragma unroll
+    for (int j = 0; j < VPER; ++j) {
+        int e = e0 + j;
+        float w = 0.f;
+        if (e < V) {
+            float zpv = to_f(zp[e]);
+            float zqv = residual ? to_f(zq[e]) : 0.f;
+            w = sample_weight(zpv, zqv, d, invT, residual, fallback);
+        }
+        wv[j] = w;
+        mine += w;
+    }
+    float total;
+    float ex = block_excl_scan(mine, sh, &total);
+    float run = s_before + ex;
+    int found = 0x7fffffff, lastpos = -1;
+#pragma unroll
+    for (int j = 0; j < VPER; ++j) {
+        run += wv[j];
+        if (found == 0x7fffffff && wv[j] > 0.f && s_t < run) found = e0 + j;
+        if (wv[j] > 0.f) lastpos = e0 + j;
+    }
+    atomicMin(&s_tok, found);
+    __syncthreads();
+    if (s_tok == 0x7fffffff) {   // rounding left u*S past this chunk: last id with weight
+        __shared__ int s_last;
+        if (threadIdx.x == 0) s_last = -1;
+        __syncthreads();
+        atomicMax(&s_last, lastpos);
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            s_tok = s_last >= 0 ? s_last : cs;
+            s_flag |= 16;
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) {
+        a.out_tokens[(size_t)b * (K + 1) + r] = s_tok;
+        a.flags[(size_t)b * (K + 1) + r] = (uint8_t)s_flag;
+    }
+}
+
+size_t verify_workspace_layout(int B, int K, int V, VerifyArgs *a, void *base) {
+    const int nch = (V + VCHUNK - 1) / VCHUNK;
+    auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
+    size_t off = 0;
+    size_t o_t1 = off; off = al(off + sizeof(int) * B);
+    size_t o_t2 = off; off = al(off + sizeof(int) * B);
+    size_t o_part = off; off = al(off + (size_t)16 * B * (K + 1) * nch);
+    size_t o_dec = off; off = al(off + sizeof(Decision) * B);
+    size_t o_cs = off; off = al(off + (size_t)8 * B * nch);
+    if (a && base) {
+        char *p = (char *)base;
+        a->ticket1 = (int *)(p + o_t1);
+        a->ticket2 = (int *)(p + o_t2);
+        a->part = p + o_part;
+        a->dec = p + o_dec;
+        a->csum = p + o_cs;
+        a->nch = nch;
+    }
+    return off;
+}
+
+template <typename T, bool VEC>
+static cudaError_t launch_t(const VerifyArgs &a, cudaStream_t s) {
+    const unsigned g1 = (unsigned)a.nch * (a.K + 1) * a.B;
+    if (a.temperature == 0.f) {
+        verify_stats<T, VEC, true><<<g1, VT, 0, s>>>(a);
+        count_launch();
+        return cudaGetLastError();
+    }
+    verify_stats<T, VEC, false><<<g1, VT, 0, s>>>(a);
+    count_launch();
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    verify_sample<T, VEC><<<(unsigned)a.nch * a.B, VT, 0, s>>>(a);
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s) {
+    const bool f32 = a.dtype == OSPREY_F32;
+    const int W = f32 ? 4 : 8;
+    bool vec = (a.V % W) == 0 && ((uintptr_t)a.target % 16) == 0 &&
+               (a.draft == nullptr || ((uintptr_t)a.draft % 16) == 0);
+    if (f32) return vec ? launch_t<float, true>(a, s) : launch_t<float, false>(a, s);
+    return vec ? launch_t<uint16_t, true>(a, s) : launch_t<uint16_t, false>(a, s);
+}
+
+}  // namespace osp

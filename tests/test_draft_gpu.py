@@ -1,0 +1,213 @@
+"""CUDA draft step vs the oracle drafter (Sec. 3.3 Eq. 1-3, Sec. 3.4), through the C ABI.
+
+Logits must agree within 2e-2 (bf16 weights and activations, fp32 accumulation).
+Token ids must agree wherever the decision is not within the error of a tie:
+greedy where the oracle's top-2 gap exceeds twice the measured logit error;
+sampled tokens are checked twice - against the inverse CDF of the GPU's own
+logits (band 1e-5) and against the oracle's logits (band from the measured
+error).  The oracle follows the GPU's chain (teacher forcing) so a flagged
+position does not desynchronise the rows after it.
+"""
+from dataclasses import replace
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from oracle import drafter as od  # noqa: E402
+from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
+from paper_2609_09338_gb300.workloads import TINY, WORKLOADS  # noqa: E402
+from parity import gather_positions  # noqa: E402
+
+LOGIT_TOL = 2e-2
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__ as g
+    g.build()
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def run_case(shape, ctx, K, T, seed, n_new=None, max_new=1, zero=False, peaked=False, sample_seqs=None,
+             feats_seed=None):
+    from paper_2609_09338_gb300.binding import to_device_bf16
+    from paper_2609_09338_gb300.session import DraftSession
+    ctx = np.asarray(ctx, np.int32)
+    B = len(ctx)
+    w = syn.make_weights(shape, seed, zero_expansion=zero, peaked_vocab=peaked)
+    kv = syn.make_kv_prefix(shape, ctx, max_new + K, seed + 1)
+    di = syn.make_draft_inputs(shape, B, max_new, K, seed + 2)
+    if feats_seed is not None:
+        di["feats"] = syn.make_draft_inputs(shape, B, max_new, K, feats_seed)["feats"]
+    if n_new is not None:
+        di["n_new"] = np.asarray(n_new, np.int32)
+    sess = DraftSession(shape, w, kv["page_table"], kv["n_pages"], K, max_new)
+    sess.append(ctx, kv["k_rows"], kv["v_rows"])
+    out = sess.draft_buffers(with_logits=True)
+    sess.draft(_dev(di["n_new"]), _dev(di["tokens"]), to_device_bf16(di["feats"]), T, _dev(di["u_draft"]), out)
+    torch.cuda.synchronize()
+    g = {k: (v.cpu().numpy() if v is not None else None) for k, v in out.items()}
+    g["status"] = int(sess.status.item())
+    g["seq_len"] = sess.kv.seq_len.cpu().numpy()
+    g["k_pages"] = sess.kv.k_pages.float().cpu().numpy()
+    g["v_pages"] = sess.kv.v_pages.float().cpu().numpy()
+    del sess
+    return dict(w=w, kv=kv, di=di, ctx=ctx, g=g, shape=shape, K=K, T=T,
+                seqs=list(range(B)) if sample_seqs is None else sample_seqs)
+
+
+def oracle_for(case):
+    """Oracle on the sampled sequences, following the GPU's chain."""
+    idx = case["seqs"]
+    ctx, kv, di = case["ctx"], case["kv"], case["di"]
+    offs = np.concatenate([[0], np.cumsum(ctx)])
+    rows = np.concatenate([np.arange(offs[b], offs[b + 1]) for b in idx]).astype(np.int64)
+    return od.draft_step(case["w"], case["shape"], kv["k_rows"][:, rows], kv["v_rows"][:, rows], ctx[idx],
+                         di["tokens"][idx], di["feats"][idx], di["n_new"][idx], case["K"], case["T"],
+                         di["u_draft"][idx], forced_tokens=case["g"]["draft_tokens"][idx])
+
+
+def check_case(case, o=None, min_checked_frac=0.5):
+    g, K, T, sh = case["g"], case["K"], case["T"], case["shape"]
+    idx = case["seqs"]
+    o = oracle_for(case) if o is None else o
+    assert g["status"] == 0
+    np.testing.assert_array_equal(g["seq_len"], case["ctx"] + case["di"]["n_new"])
+    gl = g["draft_logits"][idx]
+    err = float(np.abs(gl - o["logits"]).max())
+    assert err < LOGIT_TOL, f"logits max abs err {err}"
+    toks = g["draft_tokens"][idx]
+    checked = 0
+    for i, b in enumerate(idx):
+        for k in range(K):
+            if T == 0:
+                if o["margins"][i, k] > 2 * err + 1e-6:
+                    assert toks[i, k] == o["tokens"][i, k], (b, k)
+                    checked += 1
+            else:
+                own = od.sample(gl[i, k].astype(np.float64), T, float(case["di"]["u_draft"][b, k]))
+                if own["margin"] > 1e-5:
+                    assert toks[i, k] == own["token"], (b, k, toks[i, k], own["token"])
+                band = np.expm1(2 * err / T) + 1e-5
+                if o["margins"][i, k] > band:
+                    assert toks[i, k] == o["tokens"][i, k], (b, k)
+                    checked += 1
+    # stats and q(token)
+    if T > 0:
+        np.testing.assert_allclose(g["draft_stats"][idx][..., 0], o["stats"][..., 0], atol=LOGIT_TOL / T)
+        np.testing.assert_allclose(g["draft_stats"][idx][..., 1], o["stats"][..., 1], atol=5e-3)
+        np.testing.assert_allclose(g["draft_qx"][idx], o["qx"], rtol=3 * LOGIT_TOL / T, atol=1e-6)
+    # the K/V the call wrote (committed extend rows and speculative chain rows)
+    for i, b in enumerate(idx):
+        nn = int(case["di"]["n_new"][b])
+        pos = np.arange(case["ctx"][b], case["ctx"][b] + nn + K - 1)
+        for name, pages in (("new_k", g["k_pages"]), ("new_v", g["v_pages"])):
+            got = gather_positions(pages, case["kv"]["page_table"][b], pos)
+            np.testing.assert_allclose(got, o[name][i], atol=2e-2, rtol=1e-2)
+    return checked, len(idx) * K
+
+
+@pytest.mark.parametrize("T", [0.0, 1.0])
+def test_tiny_workload(T):
+    wl = WORKLOADS["tiny-d256-v4096-b1-k4"]
+    case = run_case(wl.shape, [wl.ctx_lo], wl.K, T, wl.seed, peaked=T > 0)
+    checked, total = check_case(case)
+    assert checked >= total - 1
+
+
+def test_tiny_random_head_sampled():
+    """A random LM head spreads q almost uniformly: sampled tokens are checked
+    against the GPU's own logits; logits and K/V against the oracle."""
+    case = run_case(TINY, [40, 3, 77], 4, 1.0, 21)
+    check_case(case)
+
+
+def test_ragged_extend_rows_two_layers():
+    shape = replace(TINY, n_layers=2, n_q_heads=8, n_kv_heads=2)
+    case = run_case(shape, [5, 0, 31, 64], 3, 0.0, 31, n_new=[3, 1, 2, 3], max_new=3)
+    check_case(case)
+
+
+def test_head_dim_128_group_4():
+    shape = replace(TINY, head_dim=128, n_q_heads=8, n_kv_heads=2, d_model=512, vocab=5000)
+    case = run_case(shape, [100, 1000, 17], 5, 0.7, 41, peaked=True)
+    check_case(case)
+
+
+def test_zero_expansion_bitwise_feature_independent():
+    """Eq. 3 on the GPU: zero context columns give bitwise-identical logits,
+    tokens and K/V whatever the target features are."""
+    a = run_case(TINY, [50, 9], 4, 0.0, 51, zero=True)
+    b = run_case(TINY, [50, 9], 4, 0.0, 51, zero=True, feats_seed=999)
+    c = run_case(TINY, [50, 9], 4, 0.0, 51, zero=True, feats_seed=1234)
+    for other in (b, c):
+        np.testing.assert_array_equal(a["g"]["draft_logits"], other["g"]["draft_logits"])
+        np.testing.assert_array_equal(a["g"]["draft_tokens"], other["g"]["draft_tokens"])
+        np.testing.assert_array_equal(a["g"]["k_pages"], other["g"]["k_pages"])
+    d = run_case(TINY, [50, 9], 4, 0.0, 51, zero=False, feats_seed=999)
+    e = run_case(TINY, [50, 9], 4, 0.0, 51, zero=False)
+    assert np.abs(d["g"]["draft_logits"] - e["g"]["draft_logits"]).max() > 1e-3
+    check_case(a)
+
+
+def test_page_table_permutation_is_bitwise_invariant():
+    a = run_case(TINY, [70, 20], 3, 1.0, 61)
+    b = run_case(TINY, [70, 20], 3, 1.0, 61)
+    np.testing.assert_array_equal(a["g"]["draft_logits"], b["g"]["draft_logits"])
+    # same contents, different physical pages: same outputs bit for bit
+    from paper_2609_09338_gb300.binding import to_device_bf16
+    from paper_2609_09338_gb300.session import DraftSession
+    kv, w, di, ctx = a["kv"], a["w"], a["di"], a["ctx"]
+    perm = np.random.default_rng(0).permutation(kv["n_pages"])
+    sess = DraftSession(TINY, w, perm[kv["page_table"]], kv["n_pages"], 3)
+    sess.append(ctx, kv["k_rows"], kv["v_rows"])
+    out = sess.draft_buffers(with_logits=True)
+    sess.draft(_dev(di["n_new"]), _dev(di["tokens"]), to_device_bf16(di["feats"]), 1.0, _dev(di["u_draft"]), out)
+    torch.cuda.synchronize()
+    np.testing.assert_array_equal(out["draft_logits"].cpu().numpy(), a["g"]["draft_logits"])
+    np.testing.assert_array_equal(out["draft_tokens"].cpu().numpy(), a["g"]["draft_tokens"])
+
+
+def test_capacity_violation_skips_only_that_sequence():
+    from paper_2609_09338_gb300.binding import to_device_bf16
+    from paper_2609_09338_gb300.session import DraftSession
+    ctx = np.array([30, 12], np.int32)
+    K = 4
+    w = syn.make_weights(TINY, 71)
+    kv = syn.make_kv_prefix(TINY, ctx, 1 + K, 72)
+    di = syn.make_draft_inputs(TINY, 2, 1, K, 73)
+    sess = DraftSession(TINY, w, kv["page_table"], kv["n_pages"], K)
+    sess.append(ctx, kv["k_rows"], kv["v_rows"])
+    # push sequence 0 to the end of its pages
+    fill = np.array([sess.kv.max_pages * 16 - 30 - 2, 0], np.int32)
+    rows = syn.make_kv_prefix(TINY, fill, 0, 74)
+    sess.append(fill, rows["k_rows"], rows["v_rows"])
+    out = sess.draft_buffers()
+    sess.draft(_dev(di["n_new"]), _dev(di["tokens"]), to_device_bf16(di["feats"]), 0.0, _dev(di["u_draft"]), out)
+    torch.cuda.synchronize()
+    assert int(sess.status.item()) == -4
+    t = out["draft_tokens"].cpu().numpy()
+    assert (t[0] == -1).all() and (t[1] >= 0).all()
+    np.testing.assert_array_equal(sess.kv.seq_len.cpu().numpy(), [30 + fill[0], 13])
+
+
+@pytest.mark.parametrize("name,T,sample", [
+    ("qwen3-8b-d1024-v151936-b1-k7", 0.0, None),
+    ("qwen3-8b-d1024-v151936-b1-k7", 1.0, None),
+    ("qwen3-8b-d1024-v151936-b32-k7", 1.0, [0, 13, 31]),
+    ("qwen3-8b-d1024-v151936-b32-k7", 0.0, [5]),
+    ("llama70b-d2048-v128256-b16-k7", 0.7, [0, 15]),
+    ("large-vocab-d1024-v200064-b64-k8", 1.0, [7, 63]),
+])
+def test_workload_full_size(name, T, sample):
+    """Each workload at its full size; the oracle checks sampled sequences."""
+    wl = WORKLOADS[name]
+    ctx = syn.make_contexts(wl)
+    case = run_case(wl.shape, ctx, wl.K, T, wl.seed, sample_seqs=sample)
+    check_case(case)

@@ -1,0 +1,177 @@
+"""CUDA verify kernels vs the oracle (Sec. 3.1 acceptance rule), through the C ABI."""
+import json
+import os
+
+import numpy as np
+import pytest
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+from oracle import verify as ov  # noqa: E402
+from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
+from paper_2609_09338_gb300.workloads import WORKLOADS  # noqa: E402
+from parity import check_verify  # noqa: E402
+
+GOLD = json.load(open(os.path.join(os.path.dirname(__file__), "golden", "hand_cases.json")))
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    import __graft_entry__ as g
+    g.build()
+
+
+def _dev(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).cuda()
+
+
+def _bf16(a):
+    from paper_2609_09338_gb300.binding import to_device_bf16
+    return to_device_bf16(syn.bf16_bits(a))
+
+
+def _run(vi, T, dtype="f32"):
+    from paper_2609_09338_gb300.session import VerifyBuffers
+    B, K1, V = vi["target_logits"].shape
+    vb = VerifyBuffers(B, K1 - 1, V)
+    conv = _dev if dtype == "f32" else _bf16
+    vb.run(conv(vi["target_logits"]), conv(vi["draft_logits"]) if T > 0 else None, _dev(vi["draft_tokens"]), T,
+           _dev(vi["u_accept"]), _dev(vi["u_sample"]))
+    torch.cuda.synchronize()
+    assert int(vb.status.item()) == 0
+    return {k: getattr(vb, k).cpu().numpy() for k in ("out_tokens", "n_accepted", "flags", "probs")}
+
+
+def _oracle(vi, T, dtype="f32"):
+    zp, zq = vi["target_logits"], vi["draft_logits"]
+    if dtype == "bf16":
+        zp, zq = syn.bf16_bits(zp), syn.bf16_bits(zq)
+    return ov.verify(zp, zq if T > 0 else None, vi["draft_tokens"], T, vi["u_accept"], vi["u_sample"])
+
+
+CASES = [
+    # V, B, K, T, sigma, dtype   (small: several chunks and a ragged tail)
+    (4096, 1, 4, 1.0, 0.7, "f32"),
+    (4096, 1, 4, 0.0, 0.7, "f32"),
+    (20000, 7, 3, 1.0, 0.7, "f32"),
+    (20000, 7, 3, 0.7, 0.5, "bf16"),
+    (20003, 5, 2, 1.0, 0.7, "f32"),      # V not a multiple of 8: scalar-load path
+    (20003, 5, 2, 0.0, 0.7, "bf16"),
+    (16, 64, 1, 1.0, 0.7, "f32"),
+    (8191, 3, 15, 1.0, 0.7, "f32"),      # maximum chain length
+]
+
+
+@pytest.mark.parametrize("V,B,K,T,sigma,dtype", CASES)
+def test_verify_matches_oracle(V, B, K, T, sigma, dtype):
+    vi = syn.make_verify_inputs(V, B, K, T, sigma, seed=V + B + K)
+    g = _run(vi, T, dtype)
+    o = _oracle(vi, T, dtype)
+    check_verify(g["out_tokens"], g["n_accepted"], o, K)
+    if T > 0:
+        np.testing.assert_allclose(g["probs"][..., 0], o["p_x"], atol=1e-5)
+        np.testing.assert_allclose(g["probs"][..., 1], o["q_x"], atol=1e-5)
+    assert (g["flags"] & 8).sum() == 0
+
+
+@pytest.mark.parametrize("name", [n for n in WORKLOADS if not n.startswith("tiny")])
+def test_verify_workload_shapes(name):
+    """Every workload's verify at full size, fp32 and (large vocab) bf16 logits."""
+    wl = WORKLOADS[name]
+    vi = syn.make_verify_inputs(wl.shape.vocab, wl.batch, wl.K, wl.temperature, wl.sigma_p, seed=wl.seed + 3)
+    for dtype in (("f32", "bf16") if wl.shape.vocab > 200000 else ("f32",)):
+        g = _run(vi, wl.temperature, dtype)
+        o = _oracle(vi, wl.temperature, dtype)
+        nflag = check_verify(g["out_tokens"], g["n_accepted"], o, wl.K)
+        assert nflag <= max(1, wl.batch // 8)
+        np.testing.assert_allclose(g["probs"][..., 0], o["p_x"], atol=1e-5)
+        # greedy on the same logits
+        g0 = _run(vi, 0.0, dtype)
+        o0 = _oracle(vi, 0.0, dtype)
+        check_verify(g0["out_tokens"], g0["n_accepted"], o0, wl.K)
+
+
+def test_identical_drafter_accepts_everything():
+    rng = np.random.default_rng(5)
+    B, K, V = 6, 7, 151936
+    zq = rng.standard_normal((B, K, V), dtype=np.float32) * 3
+    zp = np.concatenate([zq, rng.standard_normal((B, 1, V), dtype=np.float32)], 1)
+    vi = {"target_logits": zp, "draft_logits": zq, "draft_tokens": rng.integers(0, V, (B, K)).astype(np.int32),
+          "u_accept": rng.random((B, K), dtype=np.float32), "u_sample": rng.random((B, K + 1), dtype=np.float32)}
+    g = _run(vi, 1.0)
+    assert (g["n_accepted"] == K).all()
+    np.testing.assert_array_equal(g["probs"][..., 0], g["probs"][..., 1])   # p/q exactly 1
+    o = _oracle(vi, 1.0)
+    check_verify(g["out_tokens"], g["n_accepted"], o, K)
+
+
+def test_dyadic_grid_bit_exact():
+    """The dyadic V=16 rows on 64-point grids of both uniforms: every GPU outcome
+    equals the oracle's (all boundaries are 1/128 away from the grid points)."""
+    gd = GOLD["dyadic_verify"]
+    rng = np.random.default_rng(3)
+    q0 = np.asarray(gd["q_counts"], float)[rng.permutation(16)] / 64
+    p0 = np.asarray(gd["p_counts"], float)[rng.permutation(16)] / 64
+    p1 = np.asarray(gd["p_counts"], float)[rng.permutation(16)] / 64
+    N = 64
+    grid = (np.arange(N) + 0.5) / N
+    X, UA, US = [a.ravel() for a in np.meshgrid(np.arange(16), grid, grid, indexing="ij")]
+    B = X.size
+    vi = {"target_logits": np.broadcast_to(np.log(np.stack([p0, p1])).astype(np.float32), (B, 2, 16)).copy(),
+          "draft_logits": np.broadcast_to(np.log(q0).astype(np.float32)[None, None], (B, 1, 16)).copy(),
+          "draft_tokens": X[:, None].astype(np.int32), "u_accept": UA[:, None].astype(np.float32),
+          "u_sample": np.stack([US, US], 1).astype(np.float32)}
+    g = _run(vi, 1.0)
+    o = _oracle(vi, 1.0)
+    assert not o["flags"].any()
+    np.testing.assert_array_equal(g["n_accepted"], o["n_accepted"])
+    np.testing.assert_array_equal(g["out_tokens"], o["out_tokens"])
+    w = q0[X] / (N * N)
+    np.testing.assert_allclose(np.bincount(g["out_tokens"][:, 0], weights=w, minlength=16), p0, atol=1e-9)
+
+
+def test_chi_square_emission_is_p():
+    """10^6 seeded trials on V=16: the emitted token at position 0 follows p_0,
+    and at position 1 (given acceptance at 0) follows p_1."""
+    from scipy.stats import chisquare
+    rng = np.random.default_rng(99)
+    V, B = 16, 1_000_000
+    zq = rng.standard_normal((2, V)).astype(np.float32) * 1.5
+    zp = np.concatenate([zq + 0.8 * rng.standard_normal((2, V)).astype(np.float32),
+                         rng.standard_normal((1, V)).astype(np.float32)])
+    q = np.exp(zq.astype(np.float64)); q /= q.sum(-1, keepdims=True)
+    p = np.exp(zp.astype(np.float64)); p /= p.sum(-1, keepdims=True)
+    x = np.stack([rng.choice(V, B, p=q[0]), rng.choice(V, B, p=q[1])], 1).astype(np.int32)
+    vi = {"target_logits": np.broadcast_to(zp, (B, 3, V)).copy(), "draft_logits": np.broadcast_to(zq, (B, 2, V)).copy(),
+          "draft_tokens": x, "u_accept": rng.random((B, 2), dtype=np.float32),
+          "u_sample": rng.random((B, 3), dtype=np.float32)}
+    g = _run(vi, 1.0)
+    e0 = np.bincount(g["out_tokens"][:, 0], minlength=V)
+    assert chisquare(e0, B * p[0]).pvalue > 1e-3
+    acc = g["n_accepted"] >= 1
+    e1 = np.bincount(g["out_tokens"][acc, 1], minlength=V)
+    assert chisquare(e1, acc.sum() * p[1]).pvalue > 1e-3
+
+
+def test_bad_draft_token_sets_status_and_spares_others():
+    from paper_2609_09338_gb300.session import VerifyBuffers
+    vi = syn.make_verify_inputs(4096, 3, 2, 1.0, 0.7, seed=1)
+    vi["draft_tokens"][1, 1] = 4096
+    vb = VerifyBuffers(3, 2, 4096)
+    vb.run(_dev(vi["target_logits"]), _dev(vi["draft_logits"]), _dev(vi["draft_tokens"]), 1.0,
+           _dev(vi["u_accept"]), _dev(vi["u_sample"]))
+    torch.cuda.synchronize()
+    assert int(vb.status.item()) == -1
+    assert vb.n_accepted[1].item() == 0 and (vb.out_tokens[1] == -1).all()
+    ok = vi.copy()
+    o = _oracle({k: (v[[0, 2]] if hasattr(v, "shape") else v) for k, v in ok.items()}, 1.0)
+    check_verify(vb.out_tokens.cpu().numpy()[[0, 2]], vb.n_accepted.cpu().numpy()[[0, 2]], o, 2)
+
+
+def test_repeat_calls_are_deterministic():
+    vi = syn.make_verify_inputs(151936, 4, 7, 1.0, 0.7, seed=17)
+    a = _run(vi, 1.0)
+    b = _run(vi, 1.0)
+    for k in a:
+        np.testing.assert_array_equal(a[k], b[k])
