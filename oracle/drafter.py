@@ -16,6 +16,9 @@ What it computes, in the paper's order and notation:
   pre-norm blocks with RMSNorm, rotary position embedding (rotate-half
   convention), grouped-query attention, SwiGLU MLP, a final RMSNorm and the LM
   head; layer 0's residual stream starts from the token embedding E[x_t].
+* The drafter's KV cache holds bf16 values (paged serving cache, Sec. 4
+  inference settings): each new K/V row is rounded to bf16 when it is cached,
+  and attention reads the cached values.
 * Sampling of each draft token from q = softmax(logits / T) by inverse CDF
   over token ids in ascending order, or argmax (lowest id on ties) when T = 0;
   the chain is drafted with topk = 1 (Sec. 4, inference settings).
@@ -27,7 +30,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from .bf16 import widen
+from .bf16 import round_to_bf16, widen
 
 
 # --------------------------------------------------------------------------
@@ -135,7 +138,8 @@ def forward_row(W: dict, shape, cache: _SeqCache, token: int, s: np.ndarray, pos
         q = qkv[: Hq * hd].reshape(Hq, hd)
         k = qkv[Hq * hd: (Hq + Hkv) * hd].reshape(Hkv, hd)
         v = qkv[(Hq + Hkv) * hd:].reshape(Hkv, hd)
-        q, k = rope(q, pos, theta), rope(k, pos, theta)
+        q, k = rope(q, pos, theta), round_to_bf16(rope(k, pos, theta))
+        v = round_to_bf16(v)
         assert cache.length(l) == pos, "positions must be contiguous"
         cache.k[l].append(k)
         cache.v[l].append(v)
