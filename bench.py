@@ -44,8 +44,8 @@ def _sha(path):
 def parse():
     p = argparse.ArgumentParser()
     p.add_argument("--gpus", type=int, default=1)
-    p.add_argument("--steps", type=int, default=20)
-    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--steps", type=int, default=200)
+    p.add_argument("--warmup", type=int, default=10)
     p.add_argument("--impl", default="osprey", choices=["osprey", "reference"])
     p.add_argument("--workload", default=BENCH_WORKLOAD, choices=sorted(WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
@@ -84,43 +84,50 @@ class ClockSampler:
          "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
          "clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, index):
-        self.index, self.rows, self.proc = index, [], None
+    def __init__(self, index, path):
+        self.index, self.path, self.proc = index, path, None
 
     def __enter__(self):
         try:
+            self.fh = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.Q}",
-                                          "--format=csv,noheader,nounits", "-lms", "100"],
-                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
-            self.t = threading.Thread(target=self._read, daemon=True)
-            self.t.start()
+                                          "--format=csv,noheader,nounits", "-lms", "20"],
+                                         stdout=self.fh, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
         except OSError:
             self.proc = None
         return self
 
-    def _read(self):
-        for line in self.proc.stdout:
-            parts = [x.strip() for x in line.split(",")]
-            if len(parts) == 7:
-                self.rows.append(parts)
-
     def __exit__(self, *a):
         if self.proc:
+            time.sleep(0.1)
             self.proc.terminate()
             try:
                 self.proc.wait(timeout=5)
             except subprocess.TimeoutExpired:
                 self.proc.kill()
+            self.fh.close()
 
     def summary(self):
-        if not self.rows:
-            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"]}
-        sm = [float(r[0]) for r in self.rows if r[0].replace(".", "").isdigit()]
-        mx = [float(r[1]) for r in self.rows if r[1].replace(".", "").isdigit()]
+        rows = []
+        try:
+            with open(self.path) as f:
+                for line in f:
+                    parts = [x.strip() for x in line.split(",")]
+                    if len(parts) == 7:
+                        rows.append(parts)
+        except OSError:
+            pass
+        num = lambda x: float(x) if x.replace(".", "", 1).isdigit() else None
+        sm = [num(r[0]) for r in rows if num(r[0]) is not None]
+        mx = [num(r[1]) for r in rows if num(r[1]) is not None]
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": len(rows)}
         names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
-        reasons = sorted({names[i] for r in self.rows for i in range(4) if r[3 + i].lower() == "active"})
-        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
-                "reasons": reasons, "samples": len(self.rows)}
+        reasons = sorted({names[i] for r in rows for i in range(4) if r[3 + i].lower() == "active"})
+        busy = sorted(sm)[len(sm) // 4:]          # drop the idle samples around the region
+        return {"sm_mhz": statistics.median(busy), "sm_max_mhz": max(mx) if mx else None,
+                "reasons": reasons, "samples": len(rows)}
 
 
 def peaks():
@@ -198,7 +205,7 @@ def config_of(wl, ctx):
             "vocab": sh.vocab, "d_model": sh.d_model, "layers": sh.n_layers,
             "heads": f"{sh.n_q_heads}/{sh.n_kv_heads}x{sh.head_dim}", "ffn": sh.ffn_dim,
             "temperature": wl.temperature, "logits": wl.logits_dtype, "weights": "bf16",
-            "l2": "flushed (256 MB write) before every timed step", "parallelism": "replicas"}
+            "l2": "flushed before every timed step (256 MB write, then 256 MB read)", "parallelism": "replicas"}
 
 
 def main():
@@ -257,10 +264,16 @@ def main():
         step()
     launches_per_step = ob.osprey_launch_count() - n0
     torch.cuda.synchronize()
-    flush = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    flush_w = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    flush_r = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+
+    def flush():
+        """Evict L2: write a 256 MB buffer, then read another so no dirty line is left."""
+        flush_w.zero_()
+        flush_r.sum()
 
     for _ in range(max(args.warmup, 3)):
-        flush.zero_()
+        flush()
         graph.replay()
     torch.cuda.synchronize()
     assert int(sess.status.item()) == 0 and int(vb.status.item()) == 0
@@ -271,10 +284,11 @@ def main():
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    with ClockSampler(local) as clk:
+    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
+    with ClockSampler(local, os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")) as clk:
         with torch.cuda.stream(stream):
             for i in range(args.steps):
-                flush.zero_()
+                flush()
                 starts[i].record(stream)
                 graph.replay()
                 ends[i].record(stream)
@@ -298,7 +312,7 @@ def main():
     ve = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     with torch.cuda.stream(stream):
         for i in range(args.steps):
-            flush.zero_()
+            flush()
             vs[i].record(stream)
             vgraph.replay()
             ve[i].record(stream)
@@ -315,7 +329,7 @@ def main():
         [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     with torch.cuda.stream(stream):
         for i in range(args.steps):
-            flush.zero_()
+            flush()
             es[i].record(stream)
             for k, v in h_in.items():
                 dst[k].copy_(v, non_blocking=True)

@@ -91,6 +91,7 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, dev);
     if (e == cudaSuccess) e = draft_set_attributes();
     if (e != cudaSuccess) {
+        cudaGetLastError();   // do not leave the error pending for the caller's next CUDA call
         delete ctx;
         return cuda_fail(e, "device query");
     }
@@ -164,12 +165,12 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
     size_t o_valid = take(4ull * B), o_pos0 = take(4ull * B), o_nn = take(4ull * B);
     size_t o_at = take(4ull * R_ext * D.Hkv), o_lt = take(4ull * B);
-    size_t o_xe = take(4ull * R_ext * D.d), o_se = take(2ull * R_ext * D.d);
-    size_t o_xc = take(4ull * B * D.d), o_sc = take(2ull * B * D.d);
+    size_t o_xe = take(4ull * R_ext * D.d), o_se = take(4ull * R_ext * D.d);
+    size_t o_xc = take(4ull * B * D.d), o_sc = take(4ull * B * D.d);
     size_t o_q = take(4ull * R_ext * D.Hq * D.hd);
     size_t o_ap = take(4ull * R_ext * D.Hq * ns * (D.hd + 2));
-    size_t o_ao = take(2ull * R_ext * D.Hq * D.hd);
-    size_t o_fh = take(2ull * R_ext * D.F);
+    size_t o_ao = take(4ull * R_ext * D.Hq * D.hd);
+    size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
     if (ws && base) {
         char *p = (char *)base;
@@ -179,13 +180,13 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->attn_ticket = (int *)(p + o_at);
         ws->lm_ticket = (int *)(p + o_lt);
         ws->x_ext = (float *)(p + o_xe);
-        ws->s_ext = (uint16_t *)(p + o_se);
+        ws->s_ext = (float *)(p + o_se);
         ws->x_chain = (float *)(p + o_xc);
-        ws->s_chain = (uint16_t *)(p + o_sc);
+        ws->s_chain = (float *)(p + o_sc);
         ws->q = (float *)(p + o_q);
         ws->attn_part = (float *)(p + o_ap);
-        ws->attn_out = (uint16_t *)(p + o_ao);
-        ws->ffn_h = (uint16_t *)(p + o_fh);
+        ws->attn_out = (float *)(p + o_ao);
+        ws->ffn_h = (float *)(p + o_fh);
         ws->lm_stats = (float4 *)(p + o_ls);
         ws->n_splits_max = ns;
         ws->lm_warps_max = lm_warps;
@@ -303,7 +304,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         const int R = B * rows_per_seq;
         RowMap map{ws.seq_valid, ws.seq_pos0, ws.seq_nnew, rows_per_seq, step};
         float *x = ext ? ws.x_ext : ws.x_chain;
-        uint16_t *sb = ext ? ws.s_ext : ws.s_chain;
+        float *sb = ext ? ws.s_ext : ws.s_chain;
         const int ns = attn_splits(R, D.Hkv, max_ctx, ctx->sms);
         for (int l = 0; l < D.L; ++l) {
             g.map = map;
@@ -333,17 +334,17 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.ticket = ws.attn_ticket;
             if ((e = launch_attn(at, s)) != cudaSuccess) return cuda_fail(e, "attention launch");
             g.W = (const uint16_t *)W.W_o[l];
-            g.xin_bf = ws.attn_out;
+            g.xin = ws.attn_out;
             if ((e = launch_gemv(G_OPROJ, g, gemv_rg(G_OPROJ, D, R), ctx->sms, s)) != cudaSuccess)
                 return cuda_fail(e, "o-proj launch");
             g.W = (const uint16_t *)W.W_gate[l];
             g.W2 = (const uint16_t *)W.W_up[l];
             g.gain = (const uint16_t *)W.ffn_norm[l];
-            g.out_bf = ws.ffn_h;
+            g.out = ws.ffn_h;
             if ((e = launch_gemv(G_GATEUP, g, gemv_rg(G_GATEUP, D, R), ctx->sms, s)) != cudaSuccess)
                 return cuda_fail(e, "gate/up launch");
             g.W = (const uint16_t *)W.W_down[l];
-            g.xin_bf = ws.ffn_h;
+            g.xin = ws.ffn_h;
             if ((e = launch_gemv(G_DOWN, g, gemv_rg(G_DOWN, D, R), ctx->sms, s)) != cudaSuccess)
                 return cuda_fail(e, "down launch");
         }

@@ -24,15 +24,16 @@ namespace osp {
 constexpr int GT = 256;          // threads per GEMV / LM-head block
 constexpr int GW = GT / 32;      // warps per block
 constexpr int AT = 128;          // threads per attention block
+constexpr int ATTN_MAX_SPLITS = 128;
 
 // ---------------------------------------------------------------------------
-// One warp computes TR dot products of length Kd (weights streamed from HBM,
-// 16 bytes per lane per load, NB loads per row in flight) against RG bf16
-// activation rows held in shared memory.  Every (row, activation) pair is
+// One warp computes TR dot products of length Kd (bf16 weights streamed from
+// HBM, 16 bytes per lane per load, NB loads per row in flight) against RG
+// float32 activation rows held in shared memory.  Every (row, activation) pair is
 // accumulated in the same order (ascending k, fmaf) whatever TR, NB and RG are,
 // so a recomputed logit is bitwise equal to the first one.
 template <int TR, int RG, int NB>
-__device__ __forceinline__ void warp_dot(const uint16_t *const (&w)[TR], const uint16_t *xs, int Kd,
+__device__ __forceinline__ void warp_dot(const uint16_t *const (&w)[TR], const float *xs, int Kd,
                                          float (&acc)[TR][RG]) {
     const int lane = threadIdx.x & 31;
 #pragma unroll
@@ -57,8 +58,9 @@ __device__ __forceinline__ void warp_dot(const uint16_t *const (&w)[TR], const u
                 for (int t = 0; t < TR; ++t) unpack8(wv[t][i], wf[t]);
 #pragma unroll
                 for (int r = 0; r < RG; ++r) {
-                    float xf[8];
-                    unpack8(*(const uint4 *)(xs + (size_t)r * Kd + k), xf);
+                    const float4 x0 = *(const float4 *)(xs + (size_t)r * Kd + k);
+                    const float4 x1 = *(const float4 *)(xs + (size_t)r * Kd + k + 4);
+                    const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
 #pragma unroll
                     for (int t = 0; t < TR; ++t)
 #pragma unroll
@@ -74,14 +76,24 @@ __device__ __forceinline__ void warp_dot(const uint16_t *const (&w)[TR], const u
 }
 
 // ---- prologue helpers -------------------------------------------------------------
-// dst[k] = bf16(src[k]) for a bf16 row (or zeros when src is null).
-__device__ __forceinline__ void stage_copy(uint16_t *dst, const uint16_t *src, int n) {
-    for (int c = threadIdx.x; c < n / 8; c += blockDim.x)
-        ((uint4 *)dst)[c] = src ? *((const uint4 *)src + c) : make_uint4(0, 0, 0, 0);
+// dst[k] = src[k] for a float32 row (zeros when src is null).
+__device__ __forceinline__ void stage_copy(float *dst, const float *src, int n) {
+    for (int c = threadIdx.x; c < n / 4; c += blockDim.x)
+        ((float4 *)dst)[c] = src ? *((const float4 *)src + c) : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
-// dst[k] = bf16(x[k] / sqrt(mean(x^2) + eps) * gain[k]) (zeros when x is null).
-__device__ __forceinline__ void stage_rmsnorm(uint16_t *dst, const float *x, const uint16_t *gain,
+// dst[k] = widen(src[k]) for a bf16 row (zeros when src is null).
+__device__ __forceinline__ void stage_widen(float *dst, const uint16_t *src, int n) {
+    for (int c = threadIdx.x; c < n / 8; c += blockDim.x) {
+        float f[8] = {0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f, 0.f};
+        if (src) unpack8(*((const uint4 *)src + c), f);
+        ((float4 *)dst)[2 * c] = make_float4(f[0], f[1], f[2], f[3]);
+        ((float4 *)dst)[2 * c + 1] = make_float4(f[4], f[5], f[6], f[7]);
+    }
+}
+
+// dst[k] = x[k] / sqrt(mean(x^2) + eps) * gain[k] (zeros when x is null).
+__device__ __forceinline__ void stage_rmsnorm(float *dst, const float *x, const uint16_t *gain,
                                               int d, float eps, float *red) {
     float ss = 0.f;
     if (x)
@@ -100,7 +112,7 @@ __device__ __forceinline__ void stage_rmsnorm(uint16_t *dst, const float *x, con
     __syncthreads();
     const float inv = red[32];
     for (int k = threadIdx.x; k < d; k += blockDim.x)
-        dst[k] = x ? f_to_bf(x[k] * inv * bf_to_f(gain[k])) : (uint16_t)0;
+        dst[k] = x ? x[k] * inv * bf_to_f(gain[k]) : 0.f;
     __syncthreads();
 }
 
@@ -114,7 +126,7 @@ __device__ __forceinline__ void rope_cs(double inv_freq, int pos, float &c, floa
 // ---------------------------------------------------------------------------
 template <int MODE, int RG>
 __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
-    extern __shared__ __align__(16) uint16_t xs[];
+    extern __shared__ __align__(16) float xs[];
     __shared__ float red[33];
     __shared__ int s_b[RG], s_pos[RG], s_act[RG];
     const Dims &D = a.dim;
@@ -136,13 +148,13 @@ __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
     else if (MODE == G_GATEUP) { Kd = D.d; n_tasks = D.F; }
     else { Kd = D.F; n_tasks = D.d; }
 
-    // ---- prologue: stage the activation rows (bf16) in shared memory
+    // ---- prologue: stage the activation rows (float32) in shared memory
     for (int rr = 0; rr < RG; ++rr) {
         const int r = r0 + rr;
         const bool act = s_act[rr];
-        uint16_t *row = xs + (size_t)rr * Kd;
+        float *row = xs + (size_t)rr * Kd;
         if (MODE == G_FEAT) {
-            stage_copy(row, act ? a.feats + (size_t)r * D.feat : nullptr, Kd);
+            stage_widen(row, act ? a.feats + (size_t)r * D.feat : nullptr, Kd);
             if (blockIdx.x == 0 && act) {     // residual stream of layer 0 starts at E[x]
                 const uint16_t *e = a.embed + (size_t)a.tokens[r] * D.d;
                 for (int k = threadIdx.x; k < D.d; k += blockDim.x) a.x[(size_t)r * D.d + k] = bf_to_f(e[k]);
@@ -151,11 +163,11 @@ __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
             stage_copy(row, act ? a.s + (size_t)r * D.d : nullptr, D.d);
             stage_rmsnorm(row + D.d, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
         } else if (MODE == G_OPROJ) {
-            stage_copy(row, act ? a.xin_bf + (size_t)r * Kd : nullptr, Kd);
+            stage_copy(row, act ? a.xin + (size_t)r * Kd : nullptr, Kd);
         } else if (MODE == G_GATEUP) {
             stage_rmsnorm(row, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
         } else {
-            stage_copy(row, act ? a.xin_bf + (size_t)r * Kd : nullptr, Kd);
+            stage_copy(row, act ? a.xin + (size_t)r * Kd : nullptr, Kd);
         }
     }
     __syncthreads();
@@ -182,7 +194,7 @@ __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
                 const int r = r0 + rr;
                 if (MODE == G_GATEUP) {
                     const float g = acc[0][rr], u = acc[1][rr];
-                    a.out_bf[(size_t)r * D.F + task] = f_to_bf(g / (1.f + expf(-g)) * u);
+                    a.out[(size_t)r * D.F + task] = g / (1.f + expf(-g)) * u;
                 } else {
                     const int b = s_b[rr], pos = s_pos[rr];
                     float x1 = acc[0][rr], x2 = acc[1][rr];
@@ -216,7 +228,7 @@ __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
             for (int rr = 0; rr < RG; ++rr) {
                 if (lane != rr || !s_act[rr]) continue;
                 const int r = r0 + rr;
-                if (MODE == G_FEAT) a.s[(size_t)r * D.d + task] = f_to_bf(acc[0][rr]);
+                if (MODE == G_FEAT) a.s[(size_t)r * D.d + task] = acc[0][rr];
                 else a.x[(size_t)r * D.d + task] += acc[0][rr];   // residual add (oproj, down)
             }
         }
@@ -334,20 +346,42 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
         if (dim == 0) { pp[0] = M; pp[1] = den; }
     }
     if (!arrive_last(a.ticket + (size_t)r * D.Hkv + kvh, a.n_splits)) return;
+    // last split block of this (row, KV head): merge the split partials.  The
+    // split maxima and sums are gathered in parallel first, so the merge is a
+    // few independent loads per thread rather than a chain of dependent ones.
+    __shared__ float s_w[G][ATTN_MAX_SPLITS];
+    __shared__ float s_den[G];
+    const int ns = a.n_splits;
+    const float *base = a.part + ((size_t)r * Hq + kvh * G) * ns * (HD + 2);
+    for (int idx = threadIdx.x; idx < G * ns; idx += AT) {
+        const int g = idx / ns, sp = idx % ns;
+        s_w[g][sp] = __ldcg(base + ((size_t)g * ns + sp) * (HD + 2));
+    }
+    __syncthreads();
+    if (warp < G) {
+        for (int g = warp; g < G; g += AT / 32) {
+            float M = -INFINITY;
+            for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, s_w[g][sp]);
+            M = warp_max(M);
+            float den = 0.f;
+            for (int sp = lane; sp < ns; sp += 32) {
+                const float ms = s_w[g][sp];
+                const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
+                den = fmaf(f, __ldcg(base + ((size_t)g * ns + sp) * (HD + 2) + 1), den);
+                s_w[g][sp] = f;
+            }
+            den = warp_sum(den);
+            if (lane == 0) s_den[g] = den;
+        }
+    }
+    __syncthreads();
     for (int idx = threadIdx.x; idx < G * HD; idx += AT) {
         const int g = idx / HD, dim = idx % HD;
-        const float *pp = a.part + ((size_t)r * Hq + kvh * G + g) * a.n_splits * (HD + 2);
-        float M = -INFINITY;
-        for (int s = 0; s < a.n_splits; ++s) M = fmaxf(M, __ldcg(pp + (size_t)s * (HD + 2)));
-        float num = 0.f, den = 0.f;
-        for (int s = 0; s < a.n_splits; ++s) {
-            const float ms = __ldcg(pp + (size_t)s * (HD + 2));
-            if (ms == -INFINITY) continue;
-            const float f = __expf(ms - M);
-            num = fmaf(f, __ldcg(pp + (size_t)s * (HD + 2) + 2 + dim), num);
-            den = fmaf(f, __ldcg(pp + (size_t)s * (HD + 2) + 1), den);
-        }
-        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = f_to_bf(num / den);
+        const float *pp = base + (size_t)g * ns * (HD + 2) + 2 + dim;
+        float num = 0.f;
+#pragma unroll 4
+        for (int sp = 0; sp < ns; ++sp) num = fmaf(s_w[g][sp], __ldcg(pp + (size_t)sp * (HD + 2)), num);
+        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num / s_den[g];
     }
 }
 
@@ -359,7 +393,7 @@ __device__ __forceinline__ void warp_range(int V, int warps_total, int gw, int &
 }
 
 template <int RG>
-__device__ void lm_sample(const LmArgs &a, int b, int rr, int src_row, const uint16_t *xs,
+__device__ void lm_sample(const LmArgs &a, int b, int rr, int src_row, const float *xs,
                           float *ybuf) {
     __shared__ MS shm[GW];
     __shared__ AM sha[GW];
@@ -476,7 +510,7 @@ __device__ void lm_sample(const LmArgs &a, int b, int rr, int src_row, const uin
         // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[token]
         const float *xl = a.x_in + (size_t)src_row * D.d;
         for (int k = threadIdx.x; k < D.d; k += blockDim.x)
-            a.s_chain[(size_t)b * D.d + k] = f_to_bf(xl[k]);
+            a.s_chain[(size_t)b * D.d + k] = xl[k];
         __syncthreads();
         const uint16_t *e = a.embed + (size_t)token * D.d;
         for (int k = threadIdx.x; k < D.d; k += blockDim.x)
@@ -487,7 +521,7 @@ __device__ void lm_sample(const LmArgs &a, int b, int rr, int src_row, const uin
 
 template <int RG>
 __global__ void __launch_bounds__(GT) lm_head_kernel(const LmArgs a) {
-    extern __shared__ __align__(16) uint16_t xs[];   // [RG][d] bf16, then the range's logits
+    extern __shared__ __align__(16) float xs[];   // [RG][d] float32, then the range's logits
     __shared__ float red[33];
     __shared__ int s_src[RG], s_act[RG];
     const Dims &D = a.dim;
@@ -502,7 +536,7 @@ __global__ void __launch_bounds__(GT) lm_head_kernel(const LmArgs a) {
     for (int rr = 0; rr < RG; ++rr)
         stage_rmsnorm(xs + (size_t)rr * D.d, s_act[rr] ? a.x_in + (size_t)s_src[rr] * D.d : nullptr,
                       a.gain, D.d, D.eps, red);
-    float *ybuf = (float *)(xs + (size_t)RG * D.d);
+    float *ybuf = xs + (size_t)RG * D.d;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int gw = blockIdx.x * GW + warp;
@@ -589,13 +623,16 @@ __global__ void __launch_bounds__(128) prepare_kernel(const PrepArgs a) {
 // ---------------------------------------------------------------------------
 // host side
 
+// Splits per (row, KV head): about four blocks per SM over the whole grid, at
+// most 1024 keys per block, at least 64 keys (one page per warp) per block.
 int attn_splits(int R, int Hkv, int max_ctx, int sms) {
     auto cdiv = [](long long x, long long y) { return (int)((x + y - 1) / y); };
     int want = cdiv(4LL * sms, (long long)R * Hkv);
     int by_len = cdiv(max_ctx, 1024);
     int s = want > by_len ? want : by_len;
-    int cap = cdiv(max_ctx, 32);
+    int cap = cdiv(max_ctx, 64);
     if (s > cap) s = cap;
+    if (s > ATTN_MAX_SPLITS) s = ATTN_MAX_SPLITS;
     return s < 1 ? 1 : s;
 }
 
@@ -624,11 +661,11 @@ int gemv_rg(GemvMode mode, const Dims &d, int R) {
     int rg = 1;
     while (rg < R && rg < 8) rg <<= 1;
     const size_t limit = 200 * 1024;
-    while (rg > 1 && (size_t)rg * gemv_kd(mode, d) * 2 > limit) rg >>= 1;
+    while (rg > 1 && (size_t)rg * gemv_kd(mode, d) * 4 > limit) rg >>= 1;
     return rg;
 }
 
-size_t gemv_smem(GemvMode mode, const Dims &d, int rg) { return (size_t)rg * gemv_kd(mode, d) * 2; }
+size_t gemv_smem(GemvMode mode, const Dims &d, int rg) { return (size_t)rg * gemv_kd(mode, d) * 4; }
 
 template <int MODE>
 static cudaError_t launch_gemv_m(const GemvArgs &a, int rg, int sms, cudaStream_t s) {
@@ -687,7 +724,7 @@ cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s) {
 cudaError_t launch_lm(const LmArgs &a, int rg, int blocks, cudaStream_t s) {
     const int groups = (a.B + rg - 1) / rg;
     const int range_max = (a.dim.V + a.warps_total - 1) / a.warps_total + 1;
-    const size_t smem = (size_t)rg * a.dim.d * 2 + (size_t)range_max * 4;
+    const size_t smem = (size_t)rg * a.dim.d * 4 + (size_t)range_max * 4;
     dim3 grid(blocks, groups);
     switch (rg) {
     case 1: lm_head_kernel<1><<<grid, GT, smem, s>>>(a); break;
@@ -705,14 +742,27 @@ cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+// Let a kernel use all the opt-in shared memory left after its static part.
+template <typename F>
+static cudaError_t allow_smem(F *kernel) {
+    int dev = 0, optin = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    cudaFuncAttributes fa{};
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, kernel);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 optin - (int)fa.sharedSizeBytes);
+    return e;
+}
+
 template <int MODE>
 static cudaError_t set_gemv_attr() {
-    const int mx = 227 * 1024;
     cudaError_t e;
-    if ((e = cudaFuncSetAttribute(gemv_kernel<MODE, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
-    if ((e = cudaFuncSetAttribute(gemv_kernel<MODE, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
-    if ((e = cudaFuncSetAttribute(gemv_kernel<MODE, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
-    return cudaFuncSetAttribute(gemv_kernel<MODE, 8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if ((e = allow_smem(gemv_kernel<MODE, 1>))) return e;
+    if ((e = allow_smem(gemv_kernel<MODE, 2>))) return e;
+    if ((e = allow_smem(gemv_kernel<MODE, 4>))) return e;
+    return allow_smem(gemv_kernel<MODE, 8>);
 }
 
 cudaError_t draft_set_attributes() {
@@ -722,11 +772,10 @@ cudaError_t draft_set_attributes() {
     if ((e = set_gemv_attr<G_OPROJ>())) return e;
     if ((e = set_gemv_attr<G_GATEUP>())) return e;
     if ((e = set_gemv_attr<G_DOWN>())) return e;
-    const int mx = 227 * 1024;
-    if ((e = cudaFuncSetAttribute(lm_head_kernel<1>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
-    if ((e = cudaFuncSetAttribute(lm_head_kernel<2>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
-    if ((e = cudaFuncSetAttribute(lm_head_kernel<4>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx))) return e;
-    return cudaFuncSetAttribute(lm_head_kernel<8>, cudaFuncAttributeMaxDynamicSharedMemorySize, mx);
+    if ((e = allow_smem(lm_head_kernel<1>))) return e;
+    if ((e = allow_smem(lm_head_kernel<2>))) return e;
+    if ((e = allow_smem(lm_head_kernel<4>))) return e;
+    return allow_smem(lm_head_kernel<8>);
 }
 
 }  // namespace osp

@@ -1,4 +1,5 @@
 // Draft-step kernel interface (CUDA-core GEMV path for up to 8 rows per group).
+// Activations between kernels are float32; weights and the KV cache are bf16.
 #pragma once
 
 #include <cuda_runtime.h>
@@ -19,13 +20,13 @@ struct DraftWs {
     int *attn_ticket;                      // [R_ext * Hkv]
     int *lm_ticket;                        // [groups]
     float *x_ext;                          // [B*max_new][d]  residual stream, extend rows
-    uint16_t *s_ext;                       // [B*max_new][d]  context slot (c), bf16
+    float *s_ext;                          // [B*max_new][d]  context slot (c)
     float *x_chain;                        // [B][d]          residual stream, chain rows
-    uint16_t *s_chain;                     // [B][d]          context slot (fed-back x_L), bf16
+    float *s_chain;                        // [B][d]          context slot (fed-back x_L)
     float *q;                              // [R_ext][Hq*hd]  rotated queries
     float *attn_part;                      // [R_ext][Hq][n_splits][hd+2]
-    uint16_t *attn_out;                    // [R_ext][Hq*hd]
-    uint16_t *ffn_h;                       // [R_ext][F]
+    float *attn_out;                       // [R_ext][Hq*hd]
+    float *ffn_h;                          // [R_ext][F]
     float4 *lm_stats;                      // [B][lm_warps]
     int n_splits_max, lm_warps_max;
 };
@@ -62,9 +63,9 @@ struct GemvArgs {
     const uint16_t *feats;        // [B][max_new][feat]
     int max_new;
     float *x;                     // residual stream of this step
-    uint16_t *s;                  // context slot of this step
-    const uint16_t *xin_bf;       // bf16 activation input (attn_out / ffn_h)
-    uint16_t *out_bf;             // bf16 output (s_ext / ffn_h / attn partial input)
+    float *s;                     // context slot of this step
+    const float *xin;             // activation input (attn_out / ffn_h)
+    float *out;                   // gate/up output (ffn_h)
     float *q;                     // rotated queries
     uint16_t *k_pages, *v_pages;  // this layer's pages
     const int32_t *page_table;
@@ -81,7 +82,7 @@ struct AttnArgs {
     const int32_t *page_table;
     int max_pages;
     float *part;
-    uint16_t *out;
+    float *out;
     int *ticket;
 };
 
@@ -93,7 +94,7 @@ struct LmArgs {
     const float *x_in;            // residual of the step's rows (x_ext or x_chain)
     int src_is_ext;               // extend step: read row b*max_new + n_new[b] - 1
     float *x_chain;
-    uint16_t *s_chain;
+    float *s_chain;
     float temperature;
     const float *u_draft;
     int32_t *tokens;

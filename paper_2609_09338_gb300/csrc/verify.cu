@@ -139,48 +139,53 @@ __device__ void decide(const VerifyArgs &a, int b) {
         }
     }
     __syncthreads();
-    if (threadIdx.x != 0) return;
+    if (w != 0) return;
+    // warp 0: lane i evaluates position i; the chain is a ballot.  All loads
+    // below are independent, so the decision costs one round of latency.
     const int32_t *x = a.tokens + (size_t)b * K;
     int32_t *out = a.out_tokens + (size_t)b * (K + 1);
     uint8_t *fl = a.flags + (size_t)b * (K + 1);
     Decision *dec = (Decision *)a.dec + b;
-    bool ok = true;
-    for (int i = 0; i < K; ++i) ok &= (x[i] >= 0 && x[i] < V);
-    for (int i = 0; i <= K; ++i) fl[i] = 0;
+    const int xi = lane < K ? x[lane] : 0;
+    const bool ok = __all_sync(0xffffffffu, lane >= K || (xi >= 0 && xi < V));
+    if (lane <= K) fl[lane] = 0;
     if (!ok) {
-        set_status(a.status, OSPREY_ERR_INVALID_ARG);
-        for (int i = 0; i <= K; ++i) out[i] = -1;
-        a.n_accepted[b] = 0;
-        dec->r = -1;
+        if (lane == 0) {
+            set_status(a.status, OSPREY_ERR_INVALID_ARG);
+            a.n_accepted[b] = 0;
+            dec->r = -1;
+        }
+        if (lane <= K) out[lane] = -1;
         return;
     }
-    int r = K;
+    bool accept = false;
     if (GREEDY) {
-        for (int i = 0; i < K; ++i)
-            if (sAm[i] != x[i]) { r = i; break; }
-        for (int i = 0; i < r; ++i) out[i] = x[i];
-        out[r] = sAm[r];
-    } else {
+        accept = lane < K && sAm[lane] == xi;
+    } else if (lane < K) {
         const float invT = 1.f / a.temperature;
-        for (int i = 0; i < K; ++i) {
-            size_t rowp = ((size_t)b * (K + 1) + i) * V, rowq = ((size_t)b * K + i) * V;
-            float px = expf(ld_logit(a.target, a.dtype, rowp + x[i]) * invT - sMp[i]) / sSp[i];
-            float qx = expf(ld_logit(a.draft, a.dtype, rowq + x[i]) * invT - sMq[i]) / sSq[i];
-            if (a.probs) {
-                a.probs[((size_t)b * K + i) * 2 + 0] = px;
-                a.probs[((size_t)b * K + i) * 2 + 1] = qx;
-            }
-            if (r == K && !(a.u_accept[(size_t)b * K + i] < px / qx)) r = i;
+        const size_t rowp = ((size_t)b * (K + 1) + lane) * V, rowq = ((size_t)b * K + lane) * V;
+        const float px = expf(ld_logit(a.target, a.dtype, rowp + xi) * invT - sMp[lane]) / sSp[lane];
+        const float qx = expf(ld_logit(a.draft, a.dtype, rowq + xi) * invT - sMq[lane]) / sSq[lane];
+        if (a.probs) {
+            a.probs[((size_t)b * K + lane) * 2 + 0] = px;
+            a.probs[((size_t)b * K + lane) * 2 + 1] = qx;
         }
-        for (int i = 0; i < r; ++i) out[i] = x[i];
-        out[r] = -1;  // written by verify_sample
-        dec->r = r;
-        dec->Mp = sMp[r]; dec->Sp = sSp[r];
-        dec->Mq = r < K ? sMq[r] : 0.f;
-        dec->Sq = r < K ? sSq[r] : 1.f;
+        accept = a.u_accept[(size_t)b * K + lane] < px / qx;
     }
-    for (int i = r + 1; i <= K; ++i) out[i] = -1;
-    a.n_accepted[b] = r;
+    const unsigned rej = ~__ballot_sync(0xffffffffu, accept) & ((1u << K) - 1u);
+    const int r = rej ? __ffs(rej) - 1 : K;
+    if (lane < r) out[lane] = xi;
+    else if (lane == r) out[lane] = GREEDY ? sAm[r] : -1;   // sampled: written by verify_sample
+    else if (lane <= K) out[lane] = -1;
+    if (lane == 0) {
+        a.n_accepted[b] = r;
+        if (!GREEDY) {
+            dec->r = r;
+            dec->Mp = sMp[r]; dec->Sp = sSp[r];
+            dec->Mq = r < K ? sMq[r] : 0.f;
+            dec->Sq = r < K ? sSq[r] : 1.f;
+        }
+    }
 }
 
 template <typename T, bool VEC, bool GREEDY>

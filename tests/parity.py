@@ -34,7 +34,8 @@ def gather_positions(pages, page_table_row, positions):
     """pages [L, n_pages, Hkv, P, hd] (numpy float32) -> [L, len(positions), Hkv, hd]."""
     P = pages.shape[3]
     pos = np.asarray(positions)
-    return pages[:, page_table_row[pos // P], :, pos % P, :]
+    # advanced indices split by a slice put the position axis first: move it back
+    return np.moveaxis(pages[:, page_table_row[pos // P], :, pos % P, :], 0, 1)
 
 
 def bf16_to_f32(t):

@@ -111,8 +111,9 @@ def test_dyadic_grid_bit_exact():
     equals the oracle's (all boundaries are 1/128 away from the grid points)."""
     gd = GOLD["dyadic_verify"]
     rng = np.random.default_rng(3)
-    q0 = np.asarray(gd["q_counts"], float)[rng.permutation(16)] / 64
-    p0 = np.asarray(gd["p_counts"], float)[rng.permutation(16)] / 64
+    perm = rng.permutation(16)       # p0 and q0 share one permutation (the dyadic structure)
+    q0 = np.asarray(gd["q_counts"], float)[perm] / 64
+    p0 = np.asarray(gd["p_counts"], float)[perm] / 64
     p1 = np.asarray(gd["p_counts"], float)[rng.permutation(16)] / 64
     N = 64
     grid = (np.arange(N) + 0.5) / N
