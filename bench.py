@@ -49,6 +49,7 @@ def parse():
     p.add_argument("--impl", default="osprey", choices=["osprey", "reference"])
     p.add_argument("--workload", default=BENCH_WORKLOAD, choices=sorted(WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--temperature", type=float, default=None, help="override the workload's temperature")
     return p.parse_args()
 
 
@@ -226,6 +227,8 @@ def main():
     from paper_2609_09338_gb300.session import DraftSession, VerifyBuffers
 
     wl = WORKLOADS[args.workload]
+    if args.temperature is not None:
+        wl = wl.with_(temperature=args.temperature)
     sh, B, K, T = wl.shape, wl.batch, wl.K, wl.temperature
     ctx, w, kv, di, vi = make_inputs(wl, rank)
     dev = "cuda"

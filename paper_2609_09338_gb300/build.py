@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libosprey.so")
-SOURCES = ["api.cu", "verify.cu", "kv.cu", "draft.cu"]
+SOURCES = ["api.cu", "verify.cu", "kv.cu", "draft.cu", "stream.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 
@@ -31,8 +31,10 @@ def nvcc() -> str:
 
 
 def _flags(extra=()):
+    # OSPREY_NVCC_DEFINES: extra -D tuning knobs, e.g. "-DOSP_SG_NST=24"
+    defines = os.environ.get("OSPREY_NVCC_DEFINES", "").split()
     return ARCH + ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
-                   "--expt-relaxed-constexpr", *extra]
+                   "--expt-relaxed-constexpr", *defines, *extra]
 
 
 def _stamp() -> str:

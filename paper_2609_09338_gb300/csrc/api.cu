@@ -78,6 +78,12 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
     const void *ptrs[] = {w->W_c, w->embed, w->final_norm, w->lm_head};
     for (const void *p : ptrs)
         if ((uintptr_t)p % 16) return fail(OSPREY_ERR_INVALID_ARG, "weights must be 16-byte aligned");
+    for (int l = 0; l < c.n_layers; ++l) {
+        const void *lp[] = {w->attn_norm[l], w->W_qkv[l], w->W_o[l], w->ffn_norm[l], w->W_gate[l], w->W_up[l],
+                            w->W_down[l]};
+        for (const void *p : lp)
+            if ((uintptr_t)p % 16) return fail(OSPREY_ERR_INVALID_ARG, "weights must be 16-byte aligned");
+    }
     osprey_ctx *ctx = new (std::nothrow) osprey_ctx();
     if (!ctx) return fail(OSPREY_ERR_INVALID_ARG, "out of host memory");
     ctx->cfg = c;
@@ -90,6 +96,7 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
     cudaError_t e = cudaGetDevice(&dev);
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, dev);
     if (e == cudaSuccess) e = draft_set_attributes();
+    if (e == cudaSuccess) e = stream_set_attributes();
     if (e != cudaSuccess) {
         cudaGetLastError();   // do not leave the error pending for the caller's next CUDA call
         delete ctx;
@@ -172,6 +179,9 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_ao = take(4ull * R_ext * D.Hq * D.hd);
     size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
+    const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
+    size_t o_lts = take(16ull * B * lmp.n_stages);
+    size_t o_lc = take(16ull * B * lmp.blocks);
     if (ws && base) {
         char *p = (char *)base;
         ws->seq_valid = (int *)(p + o_valid);
@@ -188,6 +198,8 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->attn_out = (float *)(p + o_ao);
         ws->ffn_h = (float *)(p + o_fh);
         ws->lm_stats = (float4 *)(p + o_ls);
+        ws->lm_tile_stats = (float4 *)(p + o_lts);
+        ws->lm_cta_stats = (float4 *)(p + o_lc);
         ws->n_splits_max = ns;
         ws->lm_warps_max = lm_warps;
     }
@@ -306,18 +318,64 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         float *x = ext ? ws.x_ext : ws.x_chain;
         float *sb = ext ? ws.s_ext : ws.s_chain;
         const int ns = attn_splits(R, D.Hkv, max_ctx, ctx->sms);
+        // activation rows per launch: the streamed kernels serve one or two
+        const bool streamed = R <= 2;
+        StreamArgs sa{};
+        sa.dim = D;
+        sa.map = map;
+        sa.R = R;
+        sa.B = B;
+        sa.K = K;
+        sa.step = step;
+        sa.max_new = max_new;
+        sa.embed = (const uint16_t *)W.embed;
+        sa.x = x;
+        sa.s = sb;
+        sa.q = ws.q;
+        sa.page_table = kv->page_table;
+        sa.max_pages = kv->max_pages_per_seq;
+        sa.status = dev_status;
+        for (int i = 0; i < D.hd / 2; ++i) sa.inv_freq[i] = ctx->inv_freq[i];
+        auto plan_into = [&](GemvMode m) {
+            const StreamPlan p = stream_plan(m, D, ctx->sms);
+            sa.mode = m;
+            sa.items = p.items;
+            sa.n_items = p.n_items;
+            sa.n_stages = p.n_stages;
+            sa.stage_bytes = p.stage_bytes;
+            sa.blocks = p.blocks;
+        };
+        auto gemv = [&](GemvMode m, const char *what) -> int {
+            const int rg = streamed ? R : gemv_rg(m, D, R);
+            cudaError_t e2;
+            if (streamed && stream_supported(m, D, rg)) {
+                plan_into(m);
+                sa.W = g.W;
+                sa.W2 = g.W2;
+                sa.gain = g.gain;
+                sa.xin = g.xin;
+                sa.out = g.out;
+                sa.k_pages = g.k_pages;
+                sa.v_pages = g.v_pages;
+                e2 = launch_stream(m, sa, rg, s);
+            } else {
+                e2 = launch_gemv(m, g, rg, ctx->sms, s);
+            }
+            return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
+        };
         for (int l = 0; l < D.L; ++l) {
             g.map = map;
             g.R = R;
             g.x = x;
             g.s = sb;
             g.W = (const uint16_t *)W.W_qkv[l];
+            g.W2 = nullptr;
             g.gain = (const uint16_t *)W.attn_norm[l];
             g.q = ws.q;
             g.k_pages = (uint16_t *)kv->k_pages + l * layer_pages;
             g.v_pages = (uint16_t *)kv->v_pages + l * layer_pages;
-            if ((e = launch_gemv(G_QKV, g, gemv_rg(G_QKV, D, R), ctx->sms, s)) != cudaSuccess)
-                return cuda_fail(e, "qkv launch");
+            int rc;
+            if ((rc = gemv(G_QKV, "qkv launch")) != OSPREY_OK) return rc;
             AttnArgs at{};
             at.dim = D;
             at.map = map;
@@ -335,49 +393,67 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             if ((e = launch_attn(at, s)) != cudaSuccess) return cuda_fail(e, "attention launch");
             g.W = (const uint16_t *)W.W_o[l];
             g.xin = ws.attn_out;
-            if ((e = launch_gemv(G_OPROJ, g, gemv_rg(G_OPROJ, D, R), ctx->sms, s)) != cudaSuccess)
-                return cuda_fail(e, "o-proj launch");
+            if ((rc = gemv(G_OPROJ, "o-proj launch")) != OSPREY_OK) return rc;
             g.W = (const uint16_t *)W.W_gate[l];
             g.W2 = (const uint16_t *)W.W_up[l];
             g.gain = (const uint16_t *)W.ffn_norm[l];
             g.out = ws.ffn_h;
-            if ((e = launch_gemv(G_GATEUP, g, gemv_rg(G_GATEUP, D, R), ctx->sms, s)) != cudaSuccess)
-                return cuda_fail(e, "gate/up launch");
+            if ((rc = gemv(G_GATEUP, "gate/up launch")) != OSPREY_OK) return rc;
             g.W = (const uint16_t *)W.W_down[l];
+            g.W2 = nullptr;
             g.xin = ws.ffn_h;
-            if ((e = launch_gemv(G_DOWN, g, gemv_rg(G_DOWN, D, R), ctx->sms, s)) != cudaSuccess)
-                return cuda_fail(e, "down launch");
+            if ((rc = gemv(G_DOWN, "down launch")) != OSPREY_OK) return rc;
         }
-        LmArgs lm{};
-        lm.dim = D;
-        lm.map = map;
-        lm.B = B;
-        lm.K = K;
-        lm.step = step;
-        lm.max_new = max_new;
-        lm.W = (const uint16_t *)W.lm_head;
-        lm.gain = (const uint16_t *)W.final_norm;
-        lm.embed = (const uint16_t *)W.embed;
-        lm.x_in = x;
-        lm.src_is_ext = ext;
-        lm.x_chain = ws.x_chain;
-        lm.s_chain = ws.s_chain;
-        lm.temperature = temperature;
-        lm.u_draft = u_draft;
-        lm.tokens = draft_tokens;
-        lm.qx = draft_qx;
-        lm.stats = draft_stats;
-        lm.logits = draft_logits;
-        lm.warp_stats = ws.lm_stats;
-        lm.ticket = ws.lm_ticket;
-        const int blocks = lm_blocks(D.V, ctx->sms);
-        lm.warps_total = blocks * 8;
-        int rg = 1;
-        while (rg < B && rg < 8) rg <<= 1;
         const bool probe = step < ctx->n_probe;
         if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
-        if ((e = launch_lm(lm, rg, blocks, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
+        if (B <= 2 && stream_supported(G_LM, D, B)) {
+            plan_into(G_LM);
+            sa.W = (const uint16_t *)W.lm_head;
+            sa.gain = (const uint16_t *)W.final_norm;
+            sa.x_in = x;
+            sa.src_is_ext = ext;
+            sa.x_chain = ws.x_chain;
+            sa.s_chain = ws.s_chain;
+            sa.temperature = temperature;
+            sa.u_draft = u_draft;
+            sa.tokens = draft_tokens;
+            sa.qx = draft_qx;
+            sa.stats = draft_stats;
+            sa.logits = draft_logits;
+            sa.tile_stats = ws.lm_tile_stats;
+            sa.cta_stats = ws.lm_cta_stats;
+            sa.ticket = ws.lm_ticket;
+            if ((e = launch_stream(G_LM, sa, B, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
+        } else {
+            LmArgs lm{};
+            lm.dim = D;
+            lm.map = map;
+            lm.B = B;
+            lm.K = K;
+            lm.step = step;
+            lm.max_new = max_new;
+            lm.W = (const uint16_t *)W.lm_head;
+            lm.gain = (const uint16_t *)W.final_norm;
+            lm.embed = (const uint16_t *)W.embed;
+            lm.x_in = x;
+            lm.src_is_ext = ext;
+            lm.x_chain = ws.x_chain;
+            lm.s_chain = ws.s_chain;
+            lm.temperature = temperature;
+            lm.u_draft = u_draft;
+            lm.tokens = draft_tokens;
+            lm.qx = draft_qx;
+            lm.stats = draft_stats;
+            lm.logits = draft_logits;
+            lm.warp_stats = ws.lm_stats;
+            lm.ticket = ws.lm_ticket;
+            const int blocks = lm_blocks(D.V, ctx->sms);
+            lm.warps_total = blocks * 8;
+            int rg = 1;
+            while (rg < B && rg < 8) rg <<= 1;
+            if ((e = launch_lm(lm, rg, blocks, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
+        }
         if (probe && (e = probe_record(ctx->probe_end[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
     }

@@ -18,6 +18,7 @@
 #include "common.cuh"
 #include "draft.cuh"
 #include "internal.h"
+#include "tma.cuh"
 
 namespace osp {
 
@@ -247,6 +248,7 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
     __shared__ float sm_acc[AT / 32][G][HD];
     const Dims &D = a.dim;
     const int split = blockIdx.x, kvh = blockIdx.y, r = blockIdx.z;
+    pdl_trigger();   // the next projection may start streaming its weights
     int b, pos;
     if (!a.map.row(r, b, pos)) return;
     const int n_keys = pos + 1;

@@ -28,6 +28,8 @@ struct DraftWs {
     float *attn_out;                       // [R_ext][Hq*hd]
     float *ffn_h;                          // [R_ext][F]
     float4 *lm_stats;                      // [B][lm_warps]
+    float4 *lm_tile_stats;                 // [B][lm stages]   (streamed LM head)
+    float4 *lm_cta_stats;                  // [B][sms]
     int n_splits_max, lm_warps_max;
 };
 
@@ -113,7 +115,48 @@ struct PrepArgs {
     int32_t *status;
 };
 
-enum GemvMode { G_FEAT = 0, G_QKV = 1, G_OPROJ = 2, G_GATEUP = 3, G_DOWN = 4 };
+enum GemvMode { G_FEAT = 0, G_QKV = 1, G_OPROJ = 2, G_GATEUP = 3, G_DOWN = 4, G_LM = 5 };
+
+// Arguments of the TMA-streamed GEMV (stream.cu): one or two activation rows.
+struct StreamArgs {
+    Dims dim;
+    RowMap map;
+    int mode, R, B, K, step, max_new;
+    const uint16_t *W, *W2, *gain, *embed;
+    float *x;                     // residual stream (read by qkv/gateup, += by oproj/down)
+    const float *s;               // context slot (qkv)
+    const float *xin;             // attention output (oproj) / SwiGLU hidden (down)
+    float *out;                   // SwiGLU hidden (gateup)
+    float *q;
+    uint16_t *k_pages, *v_pages;
+    const int32_t *page_table;
+    int max_pages;
+    double inv_freq[64];
+    // LM head
+    const float *x_in;
+    int src_is_ext;
+    float *x_chain, *s_chain;
+    float temperature;
+    const float *u_draft;
+    int32_t *tokens;
+    float *qx, *stats, *logits;
+    float4 *tile_stats;           // [B][n_stages]
+    float4 *cta_stats;            // [B][blocks]
+    int *ticket;                  // [groups]
+    int32_t *status;
+    // plan (stream_plan)
+    int items, n_items, n_stages, stage_bytes, blocks;
+};
+
+struct StreamPlan {
+    int items, n_items, n_stages, stage_bytes, blocks;
+    size_t smem;
+};
+
+StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms);
+bool stream_supported(GemvMode mode, const Dims &D, int rg);
+cudaError_t launch_stream(GemvMode mode, const StreamArgs &a, int rg, cudaStream_t s);
+cudaError_t stream_set_attributes();
 
 cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s);
 cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaStream_t s);

@@ -1,0 +1,749 @@
+// TMA-streamed GEMV for one or two activation rows (the single-stream decode
+// regime, HBM-bound).
+//
+// Block = 8 consumer warps + 1 producer warp.  The weight rows a block owns
+// are cut into stages (8-16 KB); the producer streams them with 1-D bulk
+// copies (cp.async.bulk) into an 8-slot shared-memory ring, slot w being
+// consumed by warp w, with full/empty mbarriers (every wait bounded).  The
+// activation rows are staged once in shared memory as float32.  Launches use
+// programmatic dependent launch: the producer starts streaming weights before
+// the previous kernel has finished; the consumers wait for it
+// (griddepcontrol.wait) before they read activations.
+//
+// Modes (Sec. 3.3 Eq. 1-3 per layer; LM head per chain step):
+//   QKV     [q;k;v] = W~_qkv [s; RMSNorm(x)], rotary on q,k; k,v -> pages
+//   OPROJ   x += W_o attn              DOWN  x += W_down h
+//   GATEUP  h = silu(W_gate n) * (W_up n), n = RMSNorm(x)
+//   LM      logits = W_lm RMSNorm(x_L); per-stage (tile) and per-block
+//           (max, sum exp, argmax); the last block draws the token by inverse
+//           CDF: block -> tile -> recompute that tile's logits -> id.
+#include <math.h>
+
+#include "common.cuh"
+#include "draft.cuh"
+#include "internal.h"
+#include "tma.cuh"
+
+namespace osp {
+
+// Tuning knobs (compile-time): ring slots per block, stage bytes for the LM
+// head and for the per-layer projections, order in which a block walks its
+// stages (0: ascending; 1: ascending from a per-block rotation), blocks per SM.
+#ifndef OSP_SG_NST
+#define OSP_SG_NST 8
+#endif
+#ifndef OSP_SG_LM_STAGE
+#define OSP_SG_LM_STAGE 8192
+#endif
+#ifndef OSP_SG_STAGE
+#define OSP_SG_STAGE 4096
+#endif
+#ifndef OSP_SG_ORDER
+#define OSP_SG_ORDER 0
+#endif
+#ifndef OSP_SG_BLOCKS_PER_SM
+#define OSP_SG_BLOCKS_PER_SM 2
+#endif
+#ifndef OSP_SG_NPROD
+#define OSP_SG_NPROD 1   // producer lanes; lane p issues stages p, p + NPROD, ...
+#endif
+
+
+constexpr int SG_CW = 8;                      // consumer warps
+constexpr int SG_THREADS = (SG_CW + 1) * 32;  // + one producer warp
+constexpr int SG_NST = OSP_SG_NST;            // ring slots; warp w consumes slots w, w + 8, ... in turn
+constexpr int SG_MAXR = 8;                    // weight rows per stage at most
+static_assert(SG_NST % SG_CW == 0, "ring slots must be a multiple of the consumer warps");
+
+__device__ __forceinline__ int sg_kd(const StreamArgs &a) {
+    const Dims &D = a.dim;
+    switch (a.mode) {
+    case G_QKV: return 2 * D.d;
+    case G_OPROJ: return D.Hq * D.hd;
+    case G_GATEUP: return D.d;
+    case G_DOWN: return D.F;
+    default: return D.d;   // G_LM
+    }
+}
+
+__device__ __forceinline__ bool sg_pair(int mode) { return mode == G_QKV || mode == G_GATEUP; }
+
+// Dot of one bf16 weight row in shared memory with RG float32 rows: lane l
+// takes elements base + 8l .. base + 8l + 7 of every 256-wide chunk, in
+// ascending order, then a butterfly sum (the order warp_dot uses on global
+// memory, so a recomputed value is bitwise equal).
+template <int RG>
+__device__ __forceinline__ void smem_dot(const uint16_t *w, const float *xs, int Kd, float (&acc)[RG]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int r = 0; r < RG; ++r) acc[r] = 0.f;
+#pragma unroll 4
+    for (int base = 0; base < Kd; base += 256) {
+        const uint4 wv = *(const uint4 *)(w + base + lane * 8);
+        float wf[8];
+        unpack8(wv, wf);
+#pragma unroll
+        for (int r = 0; r < RG; ++r) {
+            const float4 x0 = *(const float4 *)(xs + (size_t)r * Kd + base + lane * 8);
+            const float4 x1 = *(const float4 *)(xs + (size_t)r * Kd + base + lane * 8 + 4);
+            const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[r] = fmaf(wf[e], xf[e], acc[r]);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < RG; ++r) acc[r] = warp_sum(acc[r]);
+}
+
+// NR rows at once (rows past `cnt` skipped): independent accumulators, the
+// activation chunk read once for all rows, butterflies interleaved.  Each
+// row's value is computed in exactly the order smem_dot / global_dot use.
+template <int NR, int RG>
+__device__ __forceinline__ void smem_dot_rows(const uint16_t *w, unsigned valid, const float *xs, int Kd,
+                                              float (&acc)[NR][RG]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int i = 0; i < NR; ++i)
+#pragma unroll
+        for (int r = 0; r < RG; ++r) acc[i][r] = 0.f;
+#pragma unroll 2
+    for (int base = 0; base < Kd; base += 256) {
+        uint4 wv[NR];
+#pragma unroll
+        for (int i = 0; i < NR; ++i)
+            wv[i] = ((valid >> i) & 1u) ? *(const uint4 *)(w + (size_t)i * Kd + base + lane * 8)
+                                        : make_uint4(0, 0, 0, 0);
+#pragma unroll
+        for (int r = 0; r < RG; ++r) {
+            const float4 x0 = *(const float4 *)(xs + (size_t)r * Kd + base + lane * 8);
+            const float4 x1 = *(const float4 *)(xs + (size_t)r * Kd + base + lane * 8 + 4);
+            const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+            for (int i = 0; i < NR; ++i) {
+                float wf[8];
+                unpack8(wv[i], wf);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[i][r] = fmaf(wf[e], xf[e], acc[i][r]);
+            }
+        }
+    }
+#pragma unroll
+    for (int o = 16; o; o >>= 1)
+#pragma unroll
+        for (int i = 0; i < NR; ++i)
+#pragma unroll
+            for (int r = 0; r < RG; ++r) acc[i][r] += __shfl_xor_sync(0xffffffffu, acc[i][r], o);
+}
+
+// Same arithmetic reading the row from global memory (LM-head recompute).
+template <int RG>
+__device__ __forceinline__ void global_dot(const uint16_t *w, const float *xs, int Kd, float (&acc)[RG]) {
+    const int lane = threadIdx.x & 31;
+#pragma unroll
+    for (int r = 0; r < RG; ++r) acc[r] = 0.f;
+#pragma unroll 4
+    for (int base = 0; base < Kd; base += 256) {
+        const uint4 wv = ld_stream(w + base + lane * 8);
+        float wf[8];
+        unpack8(wv, wf);
+#pragma unroll
+        for (int r = 0; r < RG; ++r) {
+            const float4 x0 = *(const float4 *)(xs + (size_t)r * Kd + base + lane * 8);
+            const float4 x1 = *(const float4 *)(xs + (size_t)r * Kd + base + lane * 8 + 4);
+            const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[r] = fmaf(wf[e], xf[e], acc[r]);
+        }
+    }
+#pragma unroll
+    for (int r = 0; r < RG; ++r) acc[r] = warp_sum(acc[r]);
+}
+
+// RMSNorm of a float32 row into shared memory by the consumer threads only.
+__device__ __forceinline__ void consumer_rmsnorm(float *dst, const float *x, const uint16_t *gain, int d,
+                                                 float eps, float *red) {
+    const int nt = SG_CW * 32;
+    float ss = 0.f;
+    if (x)
+        for (int k = threadIdx.x; k < d; k += nt) ss = fmaf(x[k], x[k], ss);
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    named_sync(1, nt);
+    if (threadIdx.x == 0) {
+        float t = 0.f;
+        for (int w = 0; w < SG_CW; ++w) t += red[w];
+        red[32] = rsqrtf(t / (float)d + eps);
+    }
+    named_sync(1, nt);
+    const float inv = red[32];
+    for (int k = threadIdx.x; k < d; k += nt) dst[k] = x ? x[k] * inv * bf_to_f(gain[k]) : 0.f;
+    named_sync(1, nt);
+}
+
+__device__ __forceinline__ void consumer_copy(float *dst, const float *src, int n) {
+    for (int c = threadIdx.x; c < n / 4; c += SG_CW * 32)
+        ((float4 *)dst)[c] = src ? ((const float4 *)src)[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+__device__ __forceinline__ void rope_cs2(double inv_freq, int pos, float &c, float &s) {
+    const double turns = (double)pos * inv_freq * 0.15915494309189535;
+    const double frac = turns - floor(turns);
+    sincosf((float)(frac * 6.283185307179586), &s, &c);
+}
+
+struct StageGeom {
+    int i0, cnt;                  // first item, items in this stage
+    const uint16_t *src0, *src1;  // segment sources (src1: pair modes)
+    uint32_t seg_bytes;           // bytes of one segment
+};
+
+__device__ __forceinline__ StageGeom stage_geom(const StreamArgs &a, int st, int Kd) {
+    StageGeom g;
+    g.i0 = st * a.items;
+    g.cnt = min(a.items, a.n_items - g.i0);
+    g.seg_bytes = (uint32_t)g.cnt * Kd * 2;
+    if (a.mode == G_QKV) {
+        const int half = a.dim.hd / 2;
+        const int h = g.i0 / half, i = g.i0 % half;
+        g.src0 = a.W + ((size_t)h * a.dim.hd + i) * Kd;
+        g.src1 = a.W + ((size_t)h * a.dim.hd + half + i) * Kd;
+    } else if (a.mode == G_GATEUP) {
+        g.src0 = a.W + (size_t)g.i0 * Kd;
+        g.src1 = a.W2 + (size_t)g.i0 * Kd;
+    } else {
+        g.src0 = a.W + (size_t)g.i0 * Kd;
+        g.src1 = nullptr;
+    }
+    return g;
+}
+
+// ---------------------------------------------------------------------------
+// Ordered inverse-CDF pick over n weighted entries (ids in ascending order):
+// the smallest i with target < C_i, C the inclusive cumulative weight.  Each
+// thread takes a contiguous run of entries.  Returns i (or, if rounding left
+// target past the last sum, the last entry with weight) and writes the
+// cumulative weight before it to *before.
+template <typename Weight>
+__device__ int cdf_pick(int n, Weight weight, float target, float *before, float *total) {
+    __shared__ float sh[33];
+    __shared__ int s_pick, s_last;
+    __shared__ float s_before;
+    const int per = (n + blockDim.x - 1) / blockDim.x;
+    const int e0 = threadIdx.x * per, e1 = min(n, e0 + per);
+    float mine = 0.f;
+    for (int e = e0; e < e1; ++e) mine += weight(e);
+    float tot;
+    const float ex = block_excl_scan(mine, sh, &tot);
+    if (threadIdx.x == 0) { s_pick = 0x7fffffff; s_last = -1; }
+    __syncthreads();
+    float run = ex, bfound = 0.f, blast = 0.f;
+    int found = 0x7fffffff, last = -1;
+    for (int e = e0; e < e1; ++e) {
+        const float c = weight(e);
+        if (c > 0.f) { last = e; blast = run; }
+        if (found == 0x7fffffff && c > 0.f && target < run + c) { found = e; bfound = run; }
+        run += c;
+    }
+    atomicMin(&s_pick, found);
+    atomicMax(&s_last, last);
+    __syncthreads();
+    const int chosen = s_pick != 0x7fffffff ? s_pick : (s_last >= 0 ? s_last : 0);
+    if (s_pick != 0x7fffffff && found == chosen) s_before = bfound;
+    if (s_pick == 0x7fffffff && last == chosen) s_before = blast;
+    if (s_pick == 0x7fffffff && s_last < 0 && threadIdx.x == 0) s_before = 0.f;
+    __syncthreads();
+    *before = s_before;
+    *total = tot;
+    __syncthreads();
+    return chosen;
+}
+
+template <int RG>
+__device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row, const float *xs, float *ybuf,
+                                 int nblk) {
+    __shared__ MS shm[SG_CW + 1];
+    __shared__ AM sha[SG_CW + 1];
+    __shared__ int s_tok;
+    __shared__ float s_e;
+    const Dims &D = a.dim;
+    const bool greedy = a.temperature == 0.f;
+    const float invT = greedy ? 1.f : 1.f / a.temperature;
+    const int t = threadIdx.x;
+    const float4 *cst = a.cta_stats + (size_t)b * nblk;
+
+    // (max, sum) and argmax over all blocks
+    MS ms{-INFINITY, 0.f};
+    AM am{-INFINITY, 0x7fffffff};
+    for (int e = t; e < nblk; e += blockDim.x) {
+        const float4 v = __ldcg(cst + e);
+        ms = ms_combine(ms, MS{v.x, v.y});
+        am = am_combine(am, AM{v.z, __float_as_int(v.w)});
+    }
+    const MS tot = block_ms(ms, shm);
+    const AM best = block_am(am, sha);
+    const float M = tot.m;
+    int token;
+    float qx, S;
+    if (greedy) {
+        token = best.i;
+        qx = 1.f;
+        S = tot.s;
+    } else {
+        auto w = [&](const float4 v) { return v.x == -INFINITY ? 0.f : v.y * __expf(v.x - M); };
+        // level 1: blocks (contiguous vocabulary ranges)
+        float before1, S1;
+        float target = 0.f;
+        {
+            // the target u * S needs the total first
+            float dummy_before;
+            cdf_pick(nblk, [&](int e) { return w(__ldcg(cst + e)); }, INFINITY, &dummy_before, &S1);
+        }
+        S = S1;
+        target = a.u_draft[(size_t)b * a.K + a.step] * S;
+        const int blk = cdf_pick(nblk, [&](int e) { return w(__ldcg(cst + e)); }, target, &before1, &S1);
+        // level 2: tiles (stages) of that block
+        const int st0 = (int)((long long)a.n_stages * blk / nblk);
+        const int st1 = (int)((long long)a.n_stages * (blk + 1) / nblk);
+        const float4 *tst = a.tile_stats + (size_t)b * a.n_stages + st0;
+        float before2, S2;
+        const int tl = cdf_pick(st1 - st0, [&](int e) { return w(__ldcg(tst + e)); }, target - before1, &before2, &S2);
+        const float before = before1 + before2;
+        // level 3: recompute that tile's logits (same arithmetic as the first pass)
+        const int lo = (st0 + tl) * a.items, hi = min(D.V, lo + a.items);
+        const int warp = t >> 5, lane = t & 31;
+        for (int n = lo + warp; n < hi; n += SG_CW + 1) {
+            float acc[RG];
+            global_dot<RG>(a.W + (size_t)n * D.d, xs, D.d, acc);
+            if (lane == 0) ybuf[n - lo] = acc[rr] * invT;
+        }
+        __syncthreads();
+        if (warp == 0) {
+            float run = before;
+            int tok = -1, lastp = -1;
+            float etok = 0.f, elast = 0.f;
+            for (int base = lo; base < hi && tok < 0; base += 32) {
+                const int n = base + lane;
+                const float e = n < hi ? __expf(ybuf[n - lo] - M) : 0.f;
+                const float inc = warp_incl_scan(e) + run;
+                const unsigned hit = __ballot_sync(0xffffffffu, n < hi && e > 0.f && target < inc);
+                const unsigned pos = __ballot_sync(0xffffffffu, n < hi && e > 0.f);
+                if (pos) {
+                    const int l2 = 31 - __clz(pos);
+                    lastp = base + l2;
+                    elast = __shfl_sync(0xffffffffu, e, l2);
+                }
+                if (hit) {
+                    const int l2 = __ffs(hit) - 1;
+                    tok = base + l2;
+                    etok = __shfl_sync(0xffffffffu, e, l2);
+                }
+                run = __shfl_sync(0xffffffffu, inc, 31);
+            }
+            if (lane == 0) {
+                if (tok < 0) { tok = lastp >= 0 ? lastp : lo; etok = elast; }
+                s_tok = tok;
+                s_e = etok;
+            }
+        }
+        __syncthreads();
+        token = s_tok;
+        qx = s_e / S;
+    }
+    if (t == 0) {
+        a.tokens[(size_t)b * a.K + a.step] = token;
+        if (a.qx) a.qx[(size_t)b * a.K + a.step] = qx;
+        if (a.stats) {
+            a.stats[((size_t)b * a.K + a.step) * 2 + 0] = M;
+            a.stats[((size_t)b * a.K + a.step) * 2 + 1] = logf(S);
+        }
+    }
+    if (a.step + 1 < a.K) {
+        // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[token]
+        const float *xl = a.x_in + (size_t)src_row * D.d;
+        for (int k = t; k < D.d; k += blockDim.x) a.s_chain[(size_t)b * D.d + k] = xl[k];
+        __syncthreads();
+        const uint16_t *e = a.embed + (size_t)token * D.d;
+        for (int k = t; k < D.d; k += blockDim.x) a.x_chain[(size_t)b * D.d + k] = bf_to_f(e[k]);
+    }
+    __syncthreads();
+}
+
+// ---------------------------------------------------------------------------
+// NRS = weight rows per stage (single modes: items; pair modes: 2 * items, the
+// second segment at row `items` of the slot).
+template <int MODE, int RG, int NRS>
+__global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kernel(const StreamArgs a) {
+    constexpr bool PAIR = MODE == G_QKV || MODE == G_GATEUP;
+    constexpr int NI = PAIR ? NRS / 2 : NRS;   // items per full stage
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(8) uint64_t full[SG_NST], empty[SG_NST];
+    __shared__ float red[33];
+    __shared__ int s_b[RG], s_pos[RG], s_act[RG], s_src[RG], s_abort;
+    __shared__ float4 s_wstats[SG_CW][RG];
+    const Dims &D = a.dim;
+    const int Kd = sg_kd(a);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    uint8_t *ring = smem;
+    float *xs = (float *)(smem + (size_t)SG_NST * a.stage_bytes);
+    float *ybuf = xs + (size_t)RG * Kd;
+    const int nblk = gridDim.x;
+    const int st0 = (int)((long long)a.n_stages * blockIdx.x / nblk);
+    const int st1 = (int)((long long)a.n_stages * (blockIdx.x + 1) / nblk);
+    const int nloc = st1 - st0;
+    const int r0 = blockIdx.y * RG;
+    const int rot = OSP_SG_ORDER == 1 && nloc > 0 ? (int)((blockIdx.x * 2654435761u) % (unsigned)nloc) : 0;
+    auto stage_of = [&](int j) { return st0 + (j + rot >= nloc ? j + rot - nloc : j + rot); };
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < SG_NST; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        s_abort = 0;
+        mbar_fence_init();
+    }
+    __syncthreads();
+    pdl_trigger();
+
+    if (warp == SG_CW) {
+        // ---- producer: weights do not depend on the previous kernel
+        if (lane < OSP_SG_NPROD) {
+            const uint64_t pol = MODE == G_LM ? policy_evict_first() : policy_evict_last();
+            int issued = 0;
+            for (int j = lane; j < nloc; j += OSP_SG_NPROD) {
+                const int slot = j % SG_NST;
+                if (j >= SG_NST && !mbar_wait(&empty[slot], ((j / SG_NST) - 1) & 1)) {
+                    set_status(a.status, OSPREY_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                    break;
+                }
+                if (s_abort) break;
+                const StageGeom g = stage_geom(a, stage_of(j), Kd);
+                uint8_t *dst = ring + (size_t)slot * a.stage_bytes;
+                mbar_arrive_expect_tx(&full[slot], PAIR ? 2 * g.seg_bytes : g.seg_bytes);
+                bulk_g2s_hint(dst, g.src0, g.seg_bytes, &full[slot], pol);
+                if (PAIR) bulk_g2s_hint(dst + (size_t)NI * Kd * 2, g.src1, g.seg_bytes, &full[slot], pol);
+                issued = j + 1;
+            }
+            if (s_abort) {
+                // let every copy this lane issued land before the block can exit
+                for (int j = lane; j < issued; j += OSP_SG_NPROD)
+                    if (j + SG_NST >= issued) mbar_wait(&full[j % SG_NST], (j / SG_NST) & 1, 200000000LL);
+            }
+        }
+    } else {
+        // ---- consumers
+        pdl_wait();
+        if (threadIdx.x < RG) {
+            int b = 0, pos = 0, src = 0;
+            bool act;
+            if (MODE == G_LM) {
+                b = r0 + threadIdx.x;
+                act = b < a.B && a.map.valid[b];
+                src = act ? (a.src_is_ext ? b * a.max_new + a.map.nnew[b] - 1 : b) : 0;
+            } else {
+                const int r = r0 + threadIdx.x;
+                act = r < a.R && a.map.row(r, b, pos);
+                src = r;
+            }
+            s_b[threadIdx.x] = b;
+            s_pos[threadIdx.x] = pos;
+            s_act[threadIdx.x] = act;
+            s_src[threadIdx.x] = src;
+        }
+        named_sync(1, SG_CW * 32);
+        for (int rr = 0; rr < RG; ++rr) {
+            const bool act = s_act[rr];
+            const int r = s_src[rr];
+            float *row = xs + (size_t)rr * Kd;
+            if (MODE == G_QKV) {
+                consumer_copy(row, act ? a.s + (size_t)r * D.d : nullptr, D.d);
+                consumer_rmsnorm(row + D.d, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
+            } else if (MODE == G_GATEUP) {
+                consumer_rmsnorm(row, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
+            } else if (MODE == G_LM) {
+                consumer_rmsnorm(row, act ? a.x_in + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
+            } else {
+                consumer_copy(row, act ? a.xin + (size_t)r * Kd : nullptr, Kd);
+            }
+        }
+        named_sync(1, SG_CW * 32);
+
+        const float invT = (MODE == G_LM && a.temperature > 0.f) ? 1.f / a.temperature : 1.f;
+        float wm[RG], ws[RG], wbv[RG];
+        int wbi[RG];
+#pragma unroll
+        for (int rr = 0; rr < RG; ++rr) { wm[rr] = -INFINITY; ws[rr] = 0.f; wbv[rr] = -INFINITY; wbi[rr] = 0x7fffffff; }
+
+        for (int j = warp; j < nloc; j += SG_CW) {
+            const int slot = j % SG_NST;
+            if (!mbar_wait(&full[slot], (j / SG_NST) & 1)) {
+                set_status(a.status, OSPREY_ERR_TIMEOUT);
+                atomicExch(&s_abort, 1);
+                mbar_wait(&full[slot], (j / SG_NST) & 1, 200000000LL);   // bounded drain
+                break;
+            }
+            const int st = stage_of(j);
+            const StageGeom g = stage_geom(a, st, Kd);
+            const uint16_t *rows = (const uint16_t *)(ring + (size_t)slot * a.stage_bytes);
+            unsigned valid = (1u << g.cnt) - 1u;
+            if (PAIR) valid |= valid << NI;
+            float acc[NRS][RG];
+            smem_dot_rows<NRS, RG>(rows, valid, xs, Kd, acc);
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[slot]);   // the slot can be refilled
+
+            if (PAIR) {
+#pragma unroll
+                for (int i = 0; i < NI; ++i) {
+                    if (i >= g.cnt) break;
+                    const int item = g.i0 + i;
+#pragma unroll
+                    for (int rr = 0; rr < RG; ++rr) {
+                        if (lane != rr || !s_act[rr]) continue;
+                        const int r = r0 + rr;
+                        if (MODE == G_GATEUP) {
+                            const float gv = acc[i][rr], uv = acc[i + NI][rr];
+                            a.out[(size_t)r * D.F + item] = gv / (1.f + expf(-gv)) * uv;
+                        } else {
+                            const int half = D.hd / 2;
+                            const int h = item / half, ii = item % half;
+                            const int b = s_b[rr], pos = s_pos[rr];
+                            float x1 = acc[i][rr], x2 = acc[i + NI][rr];
+                            if (h < D.Hq + D.Hkv) {
+                                float c, sn;
+                                rope_cs2(a.inv_freq[ii], pos, c, sn);
+                                const float y1 = x1 * c - x2 * sn, y2 = x2 * c + x1 * sn;
+                                x1 = y1;
+                                x2 = y2;
+                            }
+                            if (h < D.Hq) {
+                                float *q = a.q + (size_t)r * D.Hq * D.hd + (size_t)h * D.hd;
+                                q[ii] = x1;
+                                q[ii + half] = x2;
+                            } else {
+                                const bool is_k = h < D.Hq + D.Hkv;
+                                const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
+                                const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
+                                uint16_t *dst = (is_k ? a.k_pages : a.v_pages) +
+                                                (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * D.hd;
+                                dst[ii] = f_to_bf(x1);
+                                dst[ii + half] = f_to_bf(x2);
+                            }
+                        }
+                    }
+                }
+            } else if (MODE == G_LM) {
+                float tm[RG], ts[RG], tbv[RG];
+                int tbi[RG];
+#pragma unroll
+                for (int rr = 0; rr < RG; ++rr) { tm[rr] = -INFINITY; ts[rr] = 0.f; tbv[rr] = -INFINITY; tbi[rr] = 0x7fffffff; }
+#pragma unroll
+                for (int i = 0; i < NI; ++i) {
+                    if (i >= g.cnt) break;
+                    const int item = g.i0 + i;
+#pragma unroll
+                    for (int rr = 0; rr < RG; ++rr) {
+                        const float z = acc[i][rr];
+                        if (a.logits && lane == 0 && s_act[rr])
+                            a.logits[((size_t)(r0 + rr) * a.K + a.step) * D.V + item] = z;
+                        const float y = z * invT;
+                        if (y > tm[rr]) { ts[rr] = ts[rr] * __expf(tm[rr] - y) + 1.f; tm[rr] = y; }
+                        else ts[rr] += __expf(y - tm[rr]);
+                        if (z > tbv[rr]) { tbv[rr] = z; tbi[rr] = item; }
+                    }
+                }
+#pragma unroll
+                for (int rr = 0; rr < RG; ++rr) {
+                    if (lane == 0 && r0 + rr < a.B)
+                        a.tile_stats[(size_t)(r0 + rr) * a.n_stages + st] =
+                            make_float4(tm[rr], ts[rr], tbv[rr], __int_as_float(tbi[rr]));
+                    const MS c = ms_combine(MS{wm[rr], ws[rr]}, MS{tm[rr], ts[rr]});
+                    wm[rr] = c.m;
+                    ws[rr] = c.s;
+                    const AM m2 = am_combine(AM{wbv[rr], wbi[rr]}, AM{tbv[rr], tbi[rr]});
+                    wbv[rr] = m2.v;
+                    wbi[rr] = m2.i;
+                }
+            } else {
+#pragma unroll
+                for (int i = 0; i < NI; ++i) {
+                    if (i >= g.cnt) break;
+#pragma unroll
+                    for (int rr = 0; rr < RG; ++rr)
+                        if (lane == rr && s_act[rr]) a.x[(size_t)s_src[rr] * D.d + g.i0 + i] += acc[i][rr];
+                }
+            }
+        }
+        if (MODE == G_LM && lane == 0)
+#pragma unroll
+            for (int rr = 0; rr < RG; ++rr) s_wstats[warp][rr] = make_float4(wm[rr], ws[rr], wbv[rr], __int_as_float(wbi[rr]));
+    }
+    if (MODE != G_LM) return;
+    __syncthreads();
+    if (warp == 0) {
+#pragma unroll
+        for (int rr = 0; rr < RG; ++rr) {
+            float4 v = lane < SG_CW ? s_wstats[lane][rr] : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+            if (lane >= SG_CW) v.w = __int_as_float(0x7fffffff);
+            const MS m = warp_ms(MS{v.x, v.y});
+            const AM am = warp_am(AM{v.z, __float_as_int(v.w)});
+            if (lane == 0 && r0 + rr < a.B)
+                a.cta_stats[(size_t)(r0 + rr) * nblk + blockIdx.x] = make_float4(m.m, m.s, am.v, __int_as_float(am.i));
+        }
+    }
+    if (!arrive_last(a.ticket + blockIdx.y, nblk)) return;
+    for (int rr = 0; rr < RG; ++rr)
+        if (s_act[rr]) lm_sample_stream<RG>(a, r0 + rr, rr, s_src[rr], xs, ybuf, nblk);
+}
+
+// ---------------------------------------------------------------------------
+// host side
+
+static int pow2_floor(int x) {
+    int p = 1;
+    while (p * 2 <= x) p *= 2;
+    return p;
+}
+
+static int host_kd(GemvMode mode, const Dims &D) {
+    switch (mode) {
+    case G_QKV: return 2 * D.d;
+    case G_OPROJ: return D.Hq * D.hd;
+    case G_GATEUP: return D.d;
+    case G_DOWN: return D.F;
+    default: return D.d;
+    }
+}
+
+StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms) {
+    StreamPlan p{};
+    const int Kd = host_kd(mode, D);
+    const int row_bytes = Kd * 2;
+    const int target = mode == G_LM ? OSP_SG_LM_STAGE : OSP_SG_STAGE;   // bytes per stage
+    int rows = target / row_bytes;
+    const bool pair = mode == G_QKV || mode == G_GATEUP;
+    rows = rows < (pair ? 2 : 1) ? (pair ? 2 : 1) : rows;
+    rows = rows > SG_MAXR ? SG_MAXR : (!pair && rows >= 6 ? 6 : pow2_floor(rows));
+    if (pair) {
+        int sp = rows / 2;
+        if (mode == G_QKV && sp > D.hd / 2) sp = D.hd / 2;
+        p.items = sp;
+        p.n_items = mode == G_QKV ? (D.Hq + 2 * D.Hkv) * D.hd / 2 : D.F;
+        p.stage_bytes = 2 * sp * row_bytes;
+    } else {
+        p.items = rows;
+        p.n_items = mode == G_LM ? D.V : D.d;
+        p.stage_bytes = rows * row_bytes;
+    }
+    p.n_stages = (p.n_items + p.items - 1) / p.items;
+    p.blocks = p.n_stages < sms * OSP_SG_BLOCKS_PER_SM ? p.n_stages : sms * OSP_SG_BLOCKS_PER_SM;
+    p.smem = (size_t)SG_NST * p.stage_bytes;
+    return p;
+}
+
+static size_t stream_smem(GemvMode mode, const Dims &D, int rg, const StreamPlan &p) {
+    const int range = mode == G_LM ? p.items : 0;
+    return (size_t)SG_NST * p.stage_bytes + (size_t)rg * host_kd(mode, D) * 4 + (size_t)(range + 4) * 4;
+}
+
+bool stream_supported(GemvMode mode, const Dims &D, int rg) {
+    if (rg < 1 || rg > 2 || mode == G_FEAT) return false;
+    const StreamPlan p = stream_plan(mode, D, 1);
+    return stream_smem(mode, D, rg, p) <= 200 * 1024;
+}
+
+template <int MODE, int RG, int NRS>
+static cudaError_t launch_stream_t(const StreamArgs &a, int groups, int blocks, size_t smem, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(blocks, groups);
+    cfg.blockDim = dim3(SG_THREADS);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e = cudaLaunchKernelEx(&cfg, stream_kernel<MODE, RG, NRS>, a);
+    count_launch();
+    return e;
+}
+
+template <int MODE, int RG>
+static cudaError_t launch_stream_nrs(const StreamArgs &a, int nrs, int groups, int blocks, size_t smem,
+                                     cudaStream_t s) {
+    switch (nrs) {
+    case 1: return (MODE == G_QKV || MODE == G_GATEUP) ? cudaErrorInvalidValue
+                                                       : launch_stream_t<MODE, RG, 1>(a, groups, blocks, smem, s);
+    case 2: return launch_stream_t<MODE, RG, 2>(a, groups, blocks, smem, s);
+    case 4: return launch_stream_t<MODE, RG, 4>(a, groups, blocks, smem, s);
+    case 6: return (MODE == G_QKV || MODE == G_GATEUP) ? cudaErrorInvalidValue
+                                                       : launch_stream_t<MODE, RG, 6>(a, groups, blocks, smem, s);
+    case 8: return launch_stream_t<MODE, RG, 8>(a, groups, blocks, smem, s);
+    default: return cudaErrorInvalidValue;
+    }
+}
+
+cudaError_t launch_stream(GemvMode mode, const StreamArgs &a, int rg, cudaStream_t s) {
+    const int rows = mode == G_LM ? a.B : a.R;
+    const int groups = (rows + rg - 1) / rg;
+    StreamPlan p{a.items, a.n_items, a.n_stages, a.stage_bytes, a.blocks, 0};
+    const size_t smem = stream_smem(mode, a.dim, rg, p);
+    const int blocks = a.n_stages < a.blocks ? a.n_stages : a.blocks;
+    const bool pair = mode == G_QKV || mode == G_GATEUP;
+    const int nrs = pair ? 2 * a.items : a.items;
+#define OSP_STREAM_CASE(M)                                                                          \
+    case M:                                                                                         \
+        return rg == 1 ? launch_stream_nrs<M, 1>(a, nrs, groups, blocks, smem, s)                   \
+                       : launch_stream_nrs<M, 2>(a, nrs, groups, blocks, smem, s);
+    switch (mode) {
+        OSP_STREAM_CASE(G_QKV)
+        OSP_STREAM_CASE(G_OPROJ)
+        OSP_STREAM_CASE(G_GATEUP)
+        OSP_STREAM_CASE(G_DOWN)
+        OSP_STREAM_CASE(G_LM)
+    default: return cudaErrorInvalidValue;
+    }
+#undef OSP_STREAM_CASE
+}
+
+template <typename F>
+static cudaError_t allow_smem_s(F *kernel) {
+    int dev = 0, optin = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    cudaFuncAttributes fa{};
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, kernel);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
+    return e;
+}
+
+template <int MODE, int RG>
+static cudaError_t attr_all() {
+    cudaError_t e;
+    if (!(MODE == G_QKV || MODE == G_GATEUP)) {
+        if ((e = allow_smem_s(stream_kernel<MODE, RG, 1>)) != cudaSuccess) return e;
+        if ((e = allow_smem_s(stream_kernel<MODE, RG, 6>)) != cudaSuccess) return e;
+    }
+    if ((e = allow_smem_s(stream_kernel<MODE, RG, 2>)) != cudaSuccess) return e;
+    if ((e = allow_smem_s(stream_kernel<MODE, RG, 4>)) != cudaSuccess) return e;
+    return allow_smem_s(stream_kernel<MODE, RG, 8>);
+}
+
+cudaError_t stream_set_attributes() {
+    cudaError_t e;
+#define OSP_ATTR(M)                                                   \
+    if ((e = attr_all<M, 1>()) != cudaSuccess) return e;             \
+    if ((e = attr_all<M, 2>()) != cudaSuccess) return e;
+    OSP_ATTR(G_QKV)
+    OSP_ATTR(G_OPROJ)
+    OSP_ATTR(G_GATEUP)
+    OSP_ATTR(G_DOWN)
+    OSP_ATTR(G_LM)
+#undef OSP_ATTR
+    return cudaSuccess;
+}
+
+}  // namespace osp
