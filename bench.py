@@ -20,6 +20,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import threading
 import time
 
@@ -31,9 +32,12 @@ sys.path.insert(0, ROOT)
 from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
 from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: E402
 
-# dram__bytes_read.sum + dram__bytes_write.sum of one LM-head launch, from an
-# ncu capture of this workload; valid only for the draft.cu it was taken on.
-LM_TRAFFIC = {"draft_cu_sha256": None, "bytes_per_launch": None}
+# dram__bytes_read.sum + dram__bytes_write.sum of one LM-head launch (mean of
+# two captured launches of this workload under ncu --set full); valid
+# only for the stream.cu it was taken on.
+LM_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/stream.cu",
+              "sha256": "0ab17c7a28a51773fee611c3edd7e72ad1a37cda19fd9f132d0eae5d07c8223e",
+              "bytes_per_launch": 314_541_312}
 
 
 def _sha(path):
@@ -287,8 +291,9 @@ def main():
     if world > 1:
         dist.barrier()
     torch.cuda.synchronize()
-    os.makedirs(os.path.join(ROOT, "gpurun_out"), exist_ok=True)
-    with ClockSampler(local, os.path.join(ROOT, "gpurun_out", f"clocks_rank{rank}.csv")) as clk:
+    clk_file = tempfile.NamedTemporaryFile(prefix=f"osprey_clocks_{rank}_", suffix=".csv", delete=False)
+    clk_file.close()
+    with ClockSampler(local, clk_file.name) as clk:
         with torch.cuda.stream(stream):
             for i in range(args.steps):
                 flush()
@@ -298,6 +303,11 @@ def main():
                 ends[i].synchronize()
                 lm_ms.extend(ob.osprey_probe_read(sess.ctx, K))
         torch.cuda.synchronize()
+    clocks = clk.summary()
+    try:
+        os.unlink(clk_file.name)
+    except OSError:
+        pass
     if world > 1:
         dist.barrier()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
@@ -350,8 +360,8 @@ def main():
     peak, peak_kind = peaks()
     lm_mean_ms = sum(lm_ms) / len(lm_ms)
     lm_gbs = nb["lm_head_launch"] / (lm_mean_ms * 1e-3) / 1e9
-    sha = _sha(os.path.join(ROOT, "paper_2609_09338_gb300", "csrc", "draft.cu"))
-    traffic = LM_TRAFFIC["bytes_per_launch"] if LM_TRAFFIC["draft_cu_sha256"] == sha else None
+    sha = _sha(os.path.join(ROOT, LM_TRAFFIC["source"]))
+    traffic = LM_TRAFFIC["bytes_per_launch"] if LM_TRAFFIC["sha256"] == sha else None
     acc_len = float(vb.n_accepted.float().mean().item()) + 1.0
 
     if rank == 0:
@@ -366,7 +376,7 @@ def main():
             "draft_step_bytes": nb["draft"],
             "step_hbm_frac": (nb["draft"] + nb["verify"]) / (ms * 1e-3) / 1e9 / peak,
             "synthetic_al": acc_len,
-            "roofline": {"kernel": "lm_head_kernel (fused final RMSNorm + LM-head GEMV + online softmax)",
+            "roofline": {"kernel": "stream_kernel<LM> (final RMSNorm + TMA-streamed LM-head GEMV + on-chip sampling)",
                          "bound": "hbm", "achieved": lm_gbs, "peak": peak, "unit": "GB/s",
                          "frac": lm_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
                          "bytes_per_launch": nb["lm_head_launch"], "mean_launch_us": lm_mean_ms * 1e3,
@@ -374,7 +384,7 @@ def main():
             "e2e": {"value": world * 1e3 / e2e_ms, "unit": "steps/s", "h2d_bytes_per_step": h2d,
                     "d2h_bytes_per_step": d2h},
             "gpu_launches": launches_per_step * args.steps,
-            "clocks": clk.summary(),
+            "clocks": clocks,
         }
         if not args.no_cpu_baseline:
             res["cpu_baseline"] = cpu_baseline(wl, ctx, w, kv, di, vi)
