@@ -186,6 +186,32 @@ int osprey_verify(int B, int K, int V, int logits_dtype, const void *target_logi
                   int32_t *n_accepted, uint8_t *flags, float *probs, void *workspace,
                   size_t workspace_bytes, int32_t *dev_status, void *stream);
 
+/* Allocation-free variant of osprey_verify (the paper has no counterpart; this is
+ * for callers that cannot allocate device memory).  Some callers must not call
+ * cudaMalloc: an engine that has already reserved nearly all HBM for weights and
+ * its KV cache (an extra allocation fails or fragments its pool), or code on a
+ * latency-critical path where cudaMalloc/cudaFree may block or synchronise the
+ * device.  This entry point takes the same arguments as osprey_verify minus the
+ * workspace and uses instead a scratch array of OSPREY_VERIFY_STATIC_SCRATCH_BYTES
+ * that the library keeps in device global memory (every GPU that loads the
+ * library holds it until the process exits).
+ *   - It allocates nothing: no cudaMalloc/cudaFree, no allocating library call.
+ *   - The first call on a device looks up the array's device address (a one-time
+ *     set-up per device, done with that device current); make that first call
+ *     before any stream capture.
+ *   - Requests whose scratch would exceed the array (see
+ *     osprey_verify_workspace_bytes) return OSPREY_ERR_CAPACITY with a message.
+ *   - All calls share the one array: calls whose work can overlap on the GPU
+ *     (different streams, or different host threads) race and must be
+ *     serialised by the caller.  The counters that must start at zero are
+ *     cleared on the call's stream before its kernels run. */
+#define OSPREY_VERIFY_STATIC_SCRATCH_BYTES (4u << 20)
+int osprey_verify_static(int B, int K, int V, int logits_dtype, const void *target_logits,
+                         const void *draft_logits, const int32_t *draft_tokens, float temperature,
+                         const float *u_accept, const float *u_sample, int32_t *out_tokens,
+                         int32_t *n_accepted, uint8_t *flags, float *probs, int32_t *dev_status,
+                         void *stream);
+
 /* ---- measurement hooks (not part of the method) ------------------------------
  * osprey_probe_enable: make n_slots pairs of timing events in the context (n = 0
  * releases them).  While enabled, osprey_draft_step records pair k around its

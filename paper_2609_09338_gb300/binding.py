@@ -74,12 +74,16 @@ _c_verify_ws = _sig("osprey_verify_workspace_bytes", _sz, [ctypes.c_int, ctypes.
 _c_verify = _sig("osprey_verify", ctypes.c_int,
                  [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32, _vp, _vp, _vp, _vp,
                   _vp, _vp, _vp, _sz, _vp, _vp])
+_c_verify_static = _sig("osprey_verify_static", ctypes.c_int,
+                        [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
+                         _vp, _vp, _vp, _vp, _vp])
 _c_probe_enable = _sig("osprey_probe_enable", ctypes.c_int, [_vp, ctypes.c_int])
 _c_probe_read = _sig("osprey_probe_read", ctypes.c_int, [_vp, ctypes.POINTER(_f32), ctypes.c_int])
 _c_launch_count = _sig("osprey_launch_count", _i64, [])
 
 EXPORTED = ["osprey_last_error", "osprey_create", "osprey_destroy", "osprey_draft_workspace_bytes",
             "osprey_kv_append", "osprey_draft_step", "osprey_verify_workspace_bytes", "osprey_verify",
+            "osprey_verify_static",
             "osprey_probe_enable", "osprey_probe_read", "osprey_launch_count"]
 
 
@@ -287,6 +291,35 @@ def osprey_verify(target_logits: torch.Tensor, draft_logits, draft_tokens: torch
     _check(_c_verify(B, K, V, dt, _ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens), float(temperature),
                      _ptr(u_accept), _ptr(u_sample), _ptr(out_tokens), _ptr(n_accepted), _ptr(flags), _ptr(probs),
                      _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+
+
+VERIFY_STATIC_SCRATCH_BYTES = 4 << 20
+
+
+def osprey_verify_static(target_logits: torch.Tensor, draft_logits, draft_tokens: torch.Tensor, temperature: float,
+                         u_accept, u_sample, out_tokens: torch.Tensor, n_accepted: torch.Tensor, flags: torch.Tensor,
+                         probs=None, status: torch.Tensor = None, stream=None):
+    """osprey_verify without a workspace argument, for callers that cannot
+    allocate device memory: the library's own static scratch array is used
+    (calls that can overlap on the GPU must be serialised by the caller)."""
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    dt = {torch.float32: OSPREY_F32, torch.bfloat16: OSPREY_BF16}.get(target_logits.dtype)
+    if dt is None:
+        raise TypeError("logits must be float32 or bfloat16")
+    _need(target_logits, target_logits.dtype, (B, K + 1, V), "target_logits")
+    if draft_logits is not None:
+        _need(draft_logits, target_logits.dtype, (B, K, V), "draft_logits")
+    _need(draft_tokens, torch.int32, (B, K), "draft_tokens")
+    _need(out_tokens, torch.int32, (B, K + 1), "out_tokens")
+    _need(n_accepted, torch.int32, (B,), "n_accepted")
+    _need(flags, torch.uint8, (B, K + 1), "flags")
+    if probs is not None:
+        _need(probs, torch.float32, (B, K, 2), "probs")
+    _need(status, torch.int32, (1,), "status")
+    _check(_c_verify_static(B, K, V, dt, _ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens),
+                            float(temperature), _ptr(u_accept), _ptr(u_sample), _ptr(out_tokens), _ptr(n_accepted),
+                            _ptr(flags), _ptr(probs), _ptr(status), _stream(stream)))
 
 
 def osprey_probe_enable(ctx: Ctx, n_slots: int):

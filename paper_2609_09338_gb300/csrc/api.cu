@@ -25,6 +25,8 @@ static int fail(int code, const char *fmt, ...) {
     return code;
 }
 
+void set_last_error(const char *msg) { snprintf(g_err, sizeof g_err, "%s", msg); }
+
 static int cuda_fail(cudaError_t e, const char *what) {
     return fail(OSPREY_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
 }

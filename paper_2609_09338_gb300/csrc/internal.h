@@ -12,6 +12,9 @@ namespace osp {
 // Counts every kernel the library launches (or captures), for measurement.
 void count_launch(int n = 1);
 
+// Sets the message osprey_last_error() returns on this thread.
+void set_last_error(const char *msg);
+
 // ---------------------------------------------------------------- verify
 struct VerifyArgs {
     int B, K, V, dtype;

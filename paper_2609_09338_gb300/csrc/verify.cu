@@ -14,6 +14,9 @@
 #include <float.h>
 #include <math.h>
 
+#include <cstdio>
+#include <mutex>
+
 #include "common.cuh"
 #include "internal.h"
 
@@ -416,3 +419,75 @@ cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s) {
 }
 
 }  // namespace osp
+
+// ---------------------------------------------------------------------------
+// Allocation-free verify: the scratch lives in this file-scope device array
+// instead of a caller workspace.  Host code may not use the array's name as a
+// device address (on the host it names a stand-in), so its device address is
+// looked up once per device with cudaGetSymbolAddress, with that device current.
+namespace osp {
+
+static __device__ __align__(256) unsigned char g_verify_scratch[OSPREY_VERIFY_STATIC_SCRATCH_BYTES];
+
+namespace {
+std::mutex g_scratch_mu;
+constexpr int kMaxDevices = 256;
+void *g_scratch_addr[kMaxDevices] = {};
+}  // namespace
+
+}  // namespace osp
+
+extern "C" int osprey_verify_static(int B, int K, int V, int logits_dtype, const void *target_logits,
+                                    const void *draft_logits, const int32_t *draft_tokens, float temperature,
+                                    const float *u_accept, const float *u_sample, int32_t *out_tokens,
+                                    int32_t *n_accepted, uint8_t *flags, float *probs, int32_t *dev_status,
+                                    void *stream) {
+    using namespace osp;
+    if (B == 0) return OSPREY_OK;
+    const size_t need = osprey_verify_workspace_bytes(B, K, V);
+    if (need == 0)   // bad B, K or V: let the regular entry point report it
+        return osprey_verify(B, K, V, logits_dtype, target_logits, draft_logits, draft_tokens, temperature,
+                             u_accept, u_sample, out_tokens, n_accepted, flags, probs, nullptr, 0, dev_status,
+                             stream);
+    if (need > OSPREY_VERIFY_STATIC_SCRATCH_BYTES) {
+        char msg[256];
+        snprintf(msg, sizeof msg,
+                 "osprey_verify_static: B=%d, K=%d, V=%d needs %zu bytes of scratch; the static scratch holds %u",
+                 B, K, V, need, (unsigned)OSPREY_VERIFY_STATIC_SCRATCH_BYTES);
+        set_last_error(msg);
+        return OSPREY_ERR_CAPACITY;
+    }
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
+        set_last_error("osprey_verify_static: no usable current device");
+        return OSPREY_ERR_CUDA;
+    }
+    void *base = nullptr;
+    {
+        std::lock_guard<std::mutex> lock(g_scratch_mu);
+        if (!g_scratch_addr[dev]) {
+            void *p = nullptr;
+            e = cudaGetSymbolAddress(&p, g_verify_scratch);
+            if (e != cudaSuccess || !p) {
+                cudaGetLastError();
+                set_last_error("osprey_verify_static: cudaGetSymbolAddress of the scratch array failed");
+                return OSPREY_ERR_CUDA;
+            }
+            g_scratch_addr[dev] = p;
+        }
+        base = g_scratch_addr[dev];
+    }
+    // the arrival counters must start at zero; everything else is written before it is read
+    VerifyArgs view{};
+    verify_workspace_layout(B, K, V, &view, base);
+    cudaStream_t s = (cudaStream_t)stream;
+    if ((e = cudaMemsetAsync(view.ticket1, 0, sizeof(int) * (size_t)B, s)) != cudaSuccess ||
+        (e = cudaMemsetAsync(view.ticket2, 0, sizeof(int) * (size_t)B, s)) != cudaSuccess) {
+        set_last_error("osprey_verify_static: clearing the scratch counters failed");
+        return OSPREY_ERR_CUDA;
+    }
+    return osprey_verify(B, K, V, logits_dtype, target_logits, draft_logits, draft_tokens, temperature, u_accept,
+                         u_sample, out_tokens, n_accepted, flags, probs, base, OSPREY_VERIFY_STATIC_SCRATCH_BYTES,
+                         dev_status, stream);
+}
