@@ -54,6 +54,8 @@ def parse():
     p.add_argument("--workload", default=BENCH_WORKLOAD, choices=sorted(WORKLOADS))
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--temperature", type=float, default=None, help="override the workload's temperature")
+    p.add_argument("--verify-sweep", action="store_true",
+                   help="time verify alone over batch x K at V=200064 (fp32 and bf16 logits)")
     return p.parse_args()
 
 
@@ -213,10 +215,57 @@ def config_of(wl, ctx):
             "l2": "flushed before every timed step (256 MB write, then 256 MB read)", "parallelism": "replicas"}
 
 
+def verify_sweep(args):
+    """Verify alone: GB/s against the HBM roofline over batch x K (V = 200064)."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_09338_gb300.session import VerifyBuffers
+    torch.cuda.set_device(0)
+    V, T = 200064, 1.0
+    peak, peak_kind = peaks()
+    flush_w = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    flush_r = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
+    gen = torch.Generator(device="cuda").manual_seed(1234)
+    points = []
+    for dtype in (torch.float32, torch.bfloat16):
+        for B in (1, 8, 64, 256):
+            for K in (1, 4, 8):
+                zp = torch.randn((B, K + 1, V), generator=gen, device="cuda").to(dtype)
+                zq = torch.randn((B, K, V), generator=gen, device="cuda").to(dtype)
+                x = torch.randint(0, V, (B, K), generator=gen, device="cuda", dtype=torch.int32)
+                ua = torch.rand((B, K), generator=gen, device="cuda")
+                us = torch.rand((B, K + 1), generator=gen, device="cuda")
+                vb = VerifyBuffers(B, K, V)
+                for _ in range(3):
+                    vb.run(zp, zq, x, T, ua, us)
+                ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                      for _ in range(args.steps)]
+                for s_, e_ in ev:
+                    flush_w.zero_()
+                    flush_r.sum()
+                    s_.record()
+                    vb.run(zp, zq, x, T, ua, us)
+                    e_.record()
+                torch.cuda.synchronize()
+                us_ = 1e3 * sum(s_.elapsed_time(e_) for s_, e_ in ev) / len(ev)
+                nbytes = (B * (K + 1) * V + B * K * V) * zp.element_size()
+                gbs = nbytes / (us_ * 1e-6) / 1e9
+                points.append({"dtype": "f32" if dtype == torch.float32 else "bf16", "B": B, "K": K,
+                               "bytes": nbytes, "us": round(us_, 2), "GBps": round(gbs, 1),
+                               "frac": round(gbs / peak, 3), "roofline_us": round(nbytes / peak / 1e3, 2)})
+                del zp, zq
+    print(json.dumps({"metric": "verify GB/s sweep", "peak": peak, "peak_kind": peak_kind, "V": V,
+                      "temperature": T, "steps": args.steps, "l2": "flushed before every call",
+                      "verify_sweep": points}))
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
+    if args.verify_sweep:
+        return verify_sweep(args)
     import torch
     import torch.distributed as dist
     world = int(os.environ.get("WORLD_SIZE", "1"))

@@ -350,7 +350,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         auto gemv = [&](GemvMode m, const char *what) -> int {
             const int rg = streamed ? R : gemv_rg(m, D, R);
             cudaError_t e2;
-            if (streamed && stream_supported(m, D, rg)) {
+            if (streamed && stream_supported(m, D, rg, ctx->sms)) {
                 plan_into(m);
                 sa.W = g.W;
                 sa.W2 = g.W2;
@@ -409,7 +409,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         const bool probe = step < ctx->n_probe;
         if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
-        if (B <= 2 && stream_supported(G_LM, D, B)) {
+        if (B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
             plan_into(G_LM);
             sa.W = (const uint16_t *)W.lm_head;
             sa.gain = (const uint16_t *)W.final_norm;

@@ -154,7 +154,7 @@ struct StreamPlan {
 };
 
 StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms);
-bool stream_supported(GemvMode mode, const Dims &D, int rg);
+bool stream_supported(GemvMode mode, const Dims &D, int rg, int sms);
 cudaError_t launch_stream(GemvMode mode, const StreamArgs &a, int rg, cudaStream_t s);
 cudaError_t stream_set_attributes();
 

@@ -220,32 +220,37 @@ __device__ __forceinline__ StageGeom stage_geom(const StreamArgs &a, int st, int
 // ---------------------------------------------------------------------------
 // Ordered inverse-CDF pick over n weighted entries (ids in ascending order):
 // the smallest i with target < C_i, C the inclusive cumulative weight.  Each
-// thread takes a contiguous run of entries.  Returns i (or, if rounding left
-// target past the last sum, the last entry with weight) and writes the
-// cumulative weight before it to *before.
-template <typename Weight>
-__device__ int cdf_pick(int n, Weight weight, float target, float *before, float *total) {
-    __shared__ float sh[33];
+// thread holds at most PER consecutive weights (w[]), loaded once.  Returns i
+// (or, if rounding left target past the last sum, the last entry with weight)
+// and the cumulative weight before it.  *total receives the sum of all weights
+// (as the scan computed it).
+// target_or_u: the target itself, or (scale_by_total) a uniform u whose target
+// is u times the total this scan computes.
+template <int PER>
+__device__ int cdf_pick_regs(const float (&w)[PER], int e0, int n, float target_or_u, bool scale_by_total,
+                             float *before, float *total, float *sh) {
     __shared__ int s_pick, s_last;
     __shared__ float s_before;
-    const int per = (n + blockDim.x - 1) / blockDim.x;
-    const int e0 = threadIdx.x * per, e1 = min(n, e0 + per);
     float mine = 0.f;
-    for (int e = e0; e < e1; ++e) mine += weight(e);
+#pragma unroll
+    for (int k = 0; k < PER; ++k) mine += w[k];
     float tot;
     const float ex = block_excl_scan(mine, sh, &tot);
+    const float target = scale_by_total ? target_or_u * tot : target_or_u;
     if (threadIdx.x == 0) { s_pick = 0x7fffffff; s_last = -1; }
     __syncthreads();
     float run = ex, bfound = 0.f, blast = 0.f;
     int found = 0x7fffffff, last = -1;
-    for (int e = e0; e < e1; ++e) {
-        const float c = weight(e);
-        if (c > 0.f) { last = e; blast = run; }
-        if (found == 0x7fffffff && c > 0.f && target < run + c) { found = e; bfound = run; }
+#pragma unroll
+    for (int k = 0; k < PER; ++k) {
+        const int e = e0 + k;
+        const float c = w[k];
+        if (e < n && c > 0.f) { last = e; blast = run; }
+        if (e < n && found == 0x7fffffff && c > 0.f && target < run + c) { found = e; bfound = run; }
         run += c;
     }
-    atomicMin(&s_pick, found);
-    atomicMax(&s_last, last);
+    if (found != 0x7fffffff) atomicMin(&s_pick, found);
+    if (last >= 0) atomicMax(&s_last, last);
     __syncthreads();
     const int chosen = s_pick != 0x7fffffff ? s_pick : (s_last >= 0 ? s_last : 0);
     if (s_pick != 0x7fffffff && found == chosen) s_before = bfound;
@@ -258,11 +263,14 @@ __device__ int cdf_pick(int n, Weight weight, float target, float *before, float
     return chosen;
 }
 
+constexpr int SG_PICK_PER = 2;   // entries per thread in a pick (blocks and tiles per block <= 2 x 288)
+
 template <int RG>
 __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row, const float *xs, float *ybuf,
                                  int nblk) {
     __shared__ MS shm[SG_CW + 1];
     __shared__ AM sha[SG_CW + 1];
+    __shared__ float sh_scan[33];
     __shared__ int s_tok;
     __shared__ float s_e;
     const Dims &D = a.dim;
@@ -271,42 +279,52 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
     const int t = threadIdx.x;
     const float4 *cst = a.cta_stats + (size_t)b * nblk;
 
-    // (max, sum) and argmax over all blocks
+    // level 1: one load per block entry; (max, sum) and argmax over all blocks
+    const int e0 = t * SG_PICK_PER;
+    float4 v[SG_PICK_PER];
     MS ms{-INFINITY, 0.f};
     AM am{-INFINITY, 0x7fffffff};
-    for (int e = t; e < nblk; e += blockDim.x) {
-        const float4 v = __ldcg(cst + e);
-        ms = ms_combine(ms, MS{v.x, v.y});
-        am = am_combine(am, AM{v.z, __float_as_int(v.w)});
+#pragma unroll
+    for (int k = 0; k < SG_PICK_PER; ++k) {
+        v[k] = e0 + k < nblk ? __ldcg(cst + e0 + k) : make_float4(-INFINITY, 0.f, -INFINITY, __int_as_float(0x7fffffff));
+        ms = ms_combine(ms, MS{v[k].x, v[k].y});
+        am = am_combine(am, AM{v[k].z, __float_as_int(v[k].w)});
     }
-    const MS tot = block_ms(ms, shm);
-    const AM best = block_am(am, sha);
-    const float M = tot.m;
+    const float M = block_ms(ms, shm).m;
     int token;
     float qx, S;
     if (greedy) {
-        token = best.i;
+        token = block_am(am, sha).i;
         qx = 1.f;
-        S = tot.s;
+        // S relative to M of the raw logits, for the stats output
+        float c[SG_PICK_PER];
+#pragma unroll
+        for (int k = 0; k < SG_PICK_PER; ++k) c[k] = v[k].x == -INFINITY ? 0.f : v[k].y * __expf(v[k].x - M);
+        float mine = 0.f;
+#pragma unroll
+        for (int k = 0; k < SG_PICK_PER; ++k) mine += c[k];
+        block_excl_scan(mine, sh_scan, &S);
     } else {
-        auto w = [&](const float4 v) { return v.x == -INFINITY ? 0.f : v.y * __expf(v.x - M); };
-        // level 1: blocks (contiguous vocabulary ranges)
-        float before1, S1;
-        float target = 0.f;
-        {
-            // the target u * S needs the total first
-            float dummy_before;
-            cdf_pick(nblk, [&](int e) { return w(__ldcg(cst + e)); }, INFINITY, &dummy_before, &S1);
-        }
-        S = S1;
-        target = a.u_draft[(size_t)b * a.K + a.step] * S;
-        const int blk = cdf_pick(nblk, [&](int e) { return w(__ldcg(cst + e)); }, target, &before1, &S1);
+        float c1[SG_PICK_PER];
+#pragma unroll
+        for (int k = 0; k < SG_PICK_PER; ++k) c1[k] = v[k].x == -INFINITY ? 0.f : v[k].y * __expf(v[k].x - M);
+        // the target u * S needs the total: the pick's own scan provides it
+        const float u = a.u_draft[(size_t)b * a.K + a.step];
+        float before1;
+        const int blk = cdf_pick_regs<SG_PICK_PER>(c1, e0, nblk, u, true, &before1, &S, sh_scan);
+        const float target = u * S;
         // level 2: tiles (stages) of that block
         const int st0 = (int)((long long)a.n_stages * blk / nblk);
         const int st1 = (int)((long long)a.n_stages * (blk + 1) / nblk);
         const float4 *tst = a.tile_stats + (size_t)b * a.n_stages + st0;
+        float c2[SG_PICK_PER];
+#pragma unroll
+        for (int k = 0; k < SG_PICK_PER; ++k) {
+            const float4 w2 = e0 + k < st1 - st0 ? __ldcg(tst + e0 + k) : make_float4(-INFINITY, 0.f, 0.f, 0.f);
+            c2[k] = w2.x == -INFINITY ? 0.f : w2.y * __expf(w2.x - M);
+        }
         float before2, S2;
-        const int tl = cdf_pick(st1 - st0, [&](int e) { return w(__ldcg(tst + e)); }, target - before1, &before2, &S2);
+        const int tl = cdf_pick_regs<SG_PICK_PER>(c2, e0, st1 - st0, target - before1, false, &before2, &S2, sh_scan);
         const float before = before1 + before2;
         // level 3: recompute that tile's logits (same arithmetic as the first pass)
         const int lo = (st0 + tl) * a.items, hi = min(D.V, lo + a.items);
@@ -647,10 +665,14 @@ static size_t stream_smem(GemvMode mode, const Dims &D, int rg, const StreamPlan
     return (size_t)SG_NST * p.stage_bytes + (size_t)rg * host_kd(mode, D) * 4 + (size_t)(range + 4) * 4;
 }
 
-bool stream_supported(GemvMode mode, const Dims &D, int rg) {
+bool stream_supported(GemvMode mode, const Dims &D, int rg, int sms) {
     if (rg < 1 || rg > 2 || mode == G_FEAT) return false;
-    const StreamPlan p = stream_plan(mode, D, 1);
-    return stream_smem(mode, D, rg, p) <= 200 * 1024;
+    const StreamPlan p = stream_plan(mode, D, sms);
+    if (stream_smem(mode, D, rg, p) > 200 * 1024) return false;
+    // the LM head's sampler holds at most SG_PICK_PER entries per thread at each level
+    const int cap = SG_PICK_PER * SG_THREADS;
+    if (mode == G_LM && (p.blocks > cap || (p.n_stages + p.blocks - 1) / p.blocks > cap)) return false;
+    return true;
 }
 
 template <int MODE, int RG, int NRS>
