@@ -16,6 +16,13 @@ void count_launch(int n = 1);
 void set_last_error(const char *msg);
 
 // ---------------------------------------------------------------- verify
+struct Decision {
+    int r;          // first rejected position (K = all accepted), -1 = invalid sequence
+    float Mp, Sp;   // normalisers of target row r (logits / T)
+    float Mq, Sq;   // of draft row r (r < K)
+    int pad[3];
+};
+
 struct VerifyArgs {
     int B, K, V, dtype;
     float temperature;
@@ -33,7 +40,16 @@ struct VerifyArgs {
     int *ticket1;   // [B]
     int *ticket2;   // [B]
     int nch;
+    // streamed path (vstream.cu): per-tile partials, 4 KB row chunks
+    void *tpart;    // [B][K+1][nch3] float4
+    void *tsum;     // [B][nch3] float2
+    int *trow;      // [B][K+1] per-row arrival counters
+    void *rowstat;  // [B][K+1] float4 row summaries
+    int nch3;
+    size_t counter_bytes;   // ticket1, ticket2 and trow are one block from ticket1 on
 };
+cudaError_t launch_verify_stream(const VerifyArgs &a, int sms, cudaStream_t s);
+bool verify_stream_ok(const VerifyArgs &a);
 size_t verify_workspace_layout(int B, int K, int V, VerifyArgs *a, void *base);
 cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s);
 

@@ -26,13 +26,6 @@ constexpr int VT = 256;                 // threads per block
 constexpr int VCHUNK = 8192;            // logits of one row per block
 constexpr int VPER = VCHUNK / VT;       // logits per thread
 
-struct Decision {
-    int r;          // first rejected position (K = all accepted), -1 = invalid sequence
-    float Mp, Sp;   // normalisers of target row r (logits / T)
-    float Mq, Sq;   // of draft row r (r < K)
-    int pad[3];
-};
-
 template <typename T> struct Vec;
 template <> struct Vec<float> { static constexpr int W = 4; };
 template <> struct Vec<uint16_t> { static constexpr int W = 8; };
@@ -244,7 +237,10 @@ __global__ void __launch_bounds__(VT) verify_sample(VerifyArgs a) {
     const int c = (int)(blockIdx.x % nch), b = (int)(blockIdx.x / nch);
     const Decision d = ((const Decision *)a.dec)[b];   // written by verify_stats
     const float invT = 1.f / a.temperature;
-    const bool valid = d.r >= 0;
+    // a decision outside [-1, K] means the workspace was not produced by
+    // verify_stats (e.g. counters not zeroed): read nothing through it
+    const bool valid = d.r >= 0 && d.r <= K;
+    if (!valid && d.r != -1 && threadIdx.x == 0) set_status(a.status, OSPREY_ERR_INVALID_ARG);
     const int r = valid ? d.r : 0;
     const bool residual = r < K;
     const T *zp = (const T *)a.target + ((size_t)b * (K + 1) + r) * V;
@@ -373,13 +369,19 @@ __global__ void __launch_bounds__(VT) verify_sample(VerifyArgs a) {
 
 size_t verify_workspace_layout(int B, int K, int V, VerifyArgs *a, void *base) {
     const int nch = (V + VCHUNK - 1) / VCHUNK;
+    const int nch3 = (V + 1023) / 1024;   // 4 KB chunks of float32 rows (bf16 rows use half)
     auto al = [](size_t x) { return (x + 255) & ~(size_t)255; };
     size_t off = 0;
-    size_t o_t1 = off; off = al(off + sizeof(int) * B);
-    size_t o_t2 = off; off = al(off + sizeof(int) * B);
+    // arrival counters first, in one block (they must start at zero)
+    const size_t o_t1 = 0, o_t2 = sizeof(int) * (size_t)B, o_tr = 2 * sizeof(int) * (size_t)B;
+    const size_t ctr = o_tr + sizeof(int) * (size_t)B * (K + 1);
+    off = al(ctr);
+    size_t o_rs = off; off = al(off + (size_t)16 * B * (K + 1));
     size_t o_part = off; off = al(off + (size_t)16 * B * (K + 1) * nch);
     size_t o_dec = off; off = al(off + sizeof(Decision) * B);
     size_t o_cs = off; off = al(off + (size_t)8 * B * nch);
+    size_t o_tp = off; off = al(off + (size_t)16 * B * (K + 1) * nch3);
+    size_t o_ts = off; off = al(off + (size_t)8 * B * nch3);
     if (a && base) {
         char *p = (char *)base;
         a->ticket1 = (int *)(p + o_t1);
@@ -388,6 +390,12 @@ size_t verify_workspace_layout(int B, int K, int V, VerifyArgs *a, void *base) {
         a->dec = p + o_dec;
         a->csum = p + o_cs;
         a->nch = nch;
+        a->tpart = p + o_tp;
+        a->tsum = p + o_ts;
+        a->trow = (int *)(p + o_tr);
+        a->rowstat = p + o_rs;
+        a->nch3 = nch3;
+        a->counter_bytes = ctr;
     }
     return off;
 }
@@ -410,6 +418,13 @@ static cudaError_t launch_t(const VerifyArgs &a, cudaStream_t s) {
 }
 
 cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s) {
+    if (verify_stream_ok(a)) {
+        int dev = 0, sms = 0;
+        cudaError_t e = cudaGetDevice(&dev);
+        if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+        if (e != cudaSuccess) return e;
+        return launch_verify_stream(a, sms, s);
+    }
     const bool f32 = a.dtype == OSPREY_F32;
     const int W = f32 ? 4 : 8;
     bool vec = (a.V % W) == 0 && ((uintptr_t)a.target % 16) == 0 &&
@@ -482,8 +497,7 @@ extern "C" int osprey_verify_static(int B, int K, int V, int logits_dtype, const
     VerifyArgs view{};
     verify_workspace_layout(B, K, V, &view, base);
     cudaStream_t s = (cudaStream_t)stream;
-    if ((e = cudaMemsetAsync(view.ticket1, 0, sizeof(int) * (size_t)B, s)) != cudaSuccess ||
-        (e = cudaMemsetAsync(view.ticket2, 0, sizeof(int) * (size_t)B, s)) != cudaSuccess) {
+    if ((e = cudaMemsetAsync(view.ticket1, 0, view.counter_bytes, s)) != cudaSuccess) {
         set_last_error("osprey_verify_static: clearing the scratch counters failed");
         return OSPREY_ERR_CUDA;
     }
