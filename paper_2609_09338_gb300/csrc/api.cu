@@ -182,7 +182,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
     const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
-    size_t o_lts = take(16ull * B * lmp.n_stages);
+    size_t o_lz = take(4ull * B * D.V);
     size_t o_lc = take(16ull * B * lmp.blocks);
     if (ws && base) {
         char *p = (char *)base;
@@ -200,7 +200,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->attn_out = (float *)(p + o_ao);
         ws->ffn_h = (float *)(p + o_fh);
         ws->lm_stats = (float4 *)(p + o_ls);
-        ws->lm_tile_stats = (float4 *)(p + o_lts);
+        ws->lm_z = (float *)(p + o_lz);
         ws->lm_cta_stats = (float4 *)(p + o_lc);
         ws->n_splits_max = ns;
         ws->lm_warps_max = lm_warps;
@@ -423,7 +423,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             sa.qx = draft_qx;
             sa.stats = draft_stats;
             sa.logits = draft_logits;
-            sa.tile_stats = ws.lm_tile_stats;
+            sa.z = ws.lm_z;
             sa.cta_stats = ws.lm_cta_stats;
             sa.ticket = ws.lm_ticket;
             if ((e = launch_stream(G_LM, sa, B, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");

@@ -249,6 +249,7 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
     const Dims &D = a.dim;
     const int split = blockIdx.x, kvh = blockIdx.y, r = blockIdx.z;
     pdl_trigger();   // the next projection may start streaming its weights
+    pdl_wait();      // q and this step's K/V row come from the QKV kernel
     int b, pos;
     if (!a.map.row(r, b, pos)) return;
     const int n_keys = pos + 1;
@@ -348,42 +349,72 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
         if (dim == 0) { pp[0] = M; pp[1] = den; }
     }
     if (!arrive_last(a.ticket + (size_t)r * D.Hkv + kvh, a.n_splits)) return;
-    // last split block of this (row, KV head): merge the split partials.  The
-    // split maxima and sums are gathered in parallel first, so the merge is a
-    // few independent loads per thread rather than a chain of dependent ones.
-    __shared__ float s_w[G][ATTN_MAX_SPLITS];
+    // last split block of this (row, KV head): merge the split partials.  A
+    // thread issues every load it needs at once (split maxima and sums, and its
+    // accumulator values for up to SPR splits), so up to SPR splits cost one
+    // round trip to L2.
+    constexpr int IPT = (G * HD + AT - 1) / AT;            // (head, dim) items per thread
+    constexpr int SPR = IPT >= 8 ? 8 : (IPT >= 4 ? 16 : 32);  // splits per pass, <= 64 values held
+    __shared__ float s_w[G][ATTN_MAX_SPLITS], s_l[G][ATTN_MAX_SPLITS];
     __shared__ float s_den[G];
     const int ns = a.n_splits;
     const float *base = a.part + ((size_t)r * Hq + kvh * G) * ns * (HD + 2);
     for (int idx = threadIdx.x; idx < G * ns; idx += AT) {
         const int g = idx / ns, sp = idx % ns;
-        s_w[g][sp] = __ldcg(base + ((size_t)g * ns + sp) * (HD + 2));
+        const float *pp = base + ((size_t)g * ns + sp) * (HD + 2);
+        s_w[g][sp] = __ldcg(pp);
+        s_l[g][sp] = __ldcg(pp + 1);
+    }
+    float v[IPT][SPR];
+    auto load_pass = [&](int s0) {
+#pragma unroll
+        for (int it = 0; it < IPT; ++it) {
+            const int idx = threadIdx.x + it * AT;
+            const int g = idx / HD, dim = idx % HD;
+#pragma unroll
+            for (int k = 0; k < SPR; ++k)
+                v[it][k] = idx < G * HD && s0 + k < ns
+                               ? __ldcg(base + ((size_t)g * ns + s0 + k) * (HD + 2) + 2 + dim)
+                               : 0.f;
+        }
+    };
+    load_pass(0);
+    __syncthreads();
+    for (int g = warp; g < G; g += AT / 32) {
+        float M = -INFINITY;
+        for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, s_w[g][sp]);
+        M = warp_max(M);
+        float den = 0.f;
+        for (int sp = lane; sp < ns; sp += 32) {
+            const float ms = s_w[g][sp];
+            const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
+            den = fmaf(f, s_l[g][sp], den);
+            s_w[g][sp] = f;
+        }
+        den = warp_sum(den);
+        if (lane == 0) s_den[g] = den;
     }
     __syncthreads();
-    if (warp < G) {
-        for (int g = warp; g < G; g += AT / 32) {
-            float M = -INFINITY;
-            for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, s_w[g][sp]);
-            M = warp_max(M);
-            float den = 0.f;
-            for (int sp = lane; sp < ns; sp += 32) {
-                const float ms = s_w[g][sp];
-                const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
-                den = fmaf(f, __ldcg(base + ((size_t)g * ns + sp) * (HD + 2) + 1), den);
-                s_w[g][sp] = f;
-            }
-            den = warp_sum(den);
-            if (lane == 0) s_den[g] = den;
+    float num[IPT];
+#pragma unroll
+    for (int it = 0; it < IPT; ++it) num[it] = 0.f;
+    for (int s0 = 0; s0 < ns; s0 += SPR) {
+        if (s0 > 0) load_pass(s0);
+#pragma unroll
+        for (int it = 0; it < IPT; ++it) {
+            const int g = (threadIdx.x + it * AT) / HD;
+            if (g >= G) continue;
+#pragma unroll
+            for (int k = 0; k < SPR; ++k)
+                if (s0 + k < ns) num[it] = fmaf(s_w[g][s0 + k], v[it][k], num[it]);
         }
     }
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < G * HD; idx += AT) {
+#pragma unroll
+    for (int it = 0; it < IPT; ++it) {
+        const int idx = threadIdx.x + it * AT;
+        if (idx >= G * HD) continue;
         const int g = idx / HD, dim = idx % HD;
-        const float *pp = base + (size_t)g * ns * (HD + 2) + 2 + dim;
-        float num = 0.f;
-#pragma unroll 4
-        for (int sp = 0; sp < ns; ++sp) num = fmaf(s_w[g][sp], __ldcg(pp + (size_t)sp * (HD + 2)), num);
-        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num / s_den[g];
+        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num[it] / s_den[g];
     }
 }
 
@@ -701,26 +732,40 @@ cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaS
     }
 }
 
+template <int HD, int G>
+static cudaError_t launch_attn_t(const AttnArgs &a, cudaStream_t s) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(a.n_splits, a.dim.Hkv, a.R);
+    cfg.blockDim = dim3(AT);
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, attn_kernel<HD, G>, a);
+}
+
 cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s) {
-    dim3 grid(a.n_splits, a.dim.Hkv, a.R);
     const int G = a.dim.Hq / a.dim.Hkv;
+    cudaError_t e;
     if (a.dim.hd == 128) {
         switch (G) {
-        case 1: attn_kernel<128, 1><<<grid, AT, 0, s>>>(a); break;
-        case 2: attn_kernel<128, 2><<<grid, AT, 0, s>>>(a); break;
-        case 4: attn_kernel<128, 4><<<grid, AT, 0, s>>>(a); break;
-        default: attn_kernel<128, 8><<<grid, AT, 0, s>>>(a); break;
+        case 1: e = launch_attn_t<128, 1>(a, s); break;
+        case 2: e = launch_attn_t<128, 2>(a, s); break;
+        case 4: e = launch_attn_t<128, 4>(a, s); break;
+        default: e = launch_attn_t<128, 8>(a, s); break;
         }
     } else {
         switch (G) {
-        case 1: attn_kernel<64, 1><<<grid, AT, 0, s>>>(a); break;
-        case 2: attn_kernel<64, 2><<<grid, AT, 0, s>>>(a); break;
-        case 4: attn_kernel<64, 4><<<grid, AT, 0, s>>>(a); break;
-        default: attn_kernel<64, 8><<<grid, AT, 0, s>>>(a); break;
+        case 1: e = launch_attn_t<64, 1>(a, s); break;
+        case 2: e = launch_attn_t<64, 2>(a, s); break;
+        case 4: e = launch_attn_t<64, 4>(a, s); break;
+        default: e = launch_attn_t<64, 8>(a, s); break;
         }
     }
     count_launch();
-    return cudaGetLastError();
+    return e;
 }
 
 cudaError_t launch_lm(const LmArgs &a, int rg, int blocks, cudaStream_t s) {

@@ -28,7 +28,7 @@ struct DraftWs {
     float *attn_out;                       // [R_ext][Hq*hd]
     float *ffn_h;                          // [R_ext][F]
     float4 *lm_stats;                      // [B][lm_warps]
-    float4 *lm_tile_stats;                 // [B][lm stages]   (streamed LM head)
+    float *lm_z;                           // [B][V] logits of the chain step (streamed LM head)
     float4 *lm_cta_stats;                  // [B][sms]
     int n_splits_max, lm_warps_max;
 };
@@ -140,7 +140,7 @@ struct StreamArgs {
     const float *u_draft;
     int32_t *tokens;
     float *qx, *stats, *logits;
-    float4 *tile_stats;           // [B][n_stages]
+    float *z;                     // [B][V] logits of the chain step (when logits is null)
     float4 *cta_stats;            // [B][blocks]
     int *ticket;                  // [groups]
     int32_t *status;

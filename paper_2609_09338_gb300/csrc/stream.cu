@@ -180,6 +180,54 @@ __device__ __forceinline__ void consumer_rmsnorm(float *dst, const float *x, con
     named_sync(1, nt);
 }
 
+// Register-held variant for d <= SG_PV * 4 * 256: the caller issues the loads
+// of x (and of the gain, before griddepcontrol.wait) together, so the
+// normalisation costs a single round trip.
+constexpr int SG_PV = 4;   // float4 of a d-vector per consumer thread
+__device__ __forceinline__ void load_vec4(float4 (&v)[SG_PV], const float *src, int n4) {
+#pragma unroll
+    for (int k = 0; k < SG_PV; ++k) {
+        const int c = threadIdx.x + k * SG_CW * 32;
+        v[k] = src && c < n4 ? ((const float4 *)src)[c] : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+}
+__device__ __forceinline__ void load_gain4(uint2 (&g)[SG_PV], const uint16_t *gain, int n4) {
+#pragma unroll
+    for (int k = 0; k < SG_PV; ++k) {
+        const int c = threadIdx.x + k * SG_CW * 32;
+        g[k] = c < n4 ? ((const uint2 *)gain)[c] : make_uint2(0u, 0u);
+    }
+}
+__device__ __forceinline__ void store_vec4(float *dst, const float4 (&v)[SG_PV], int n4) {
+#pragma unroll
+    for (int k = 0; k < SG_PV; ++k) {
+        const int c = threadIdx.x + k * SG_CW * 32;
+        if (c < n4) ((float4 *)dst)[c] = v[k];
+    }
+}
+__device__ __forceinline__ void consumer_rmsnorm_regs(float *dst, const float4 (&x)[SG_PV], const uint2 (&g)[SG_PV],
+                                                      int d, float eps, float *red) {
+    const int nt = SG_CW * 32;
+    float ss = 0.f;
+#pragma unroll
+    for (int k = 0; k < SG_PV; ++k) ss += x[k].x * x[k].x + x[k].y * x[k].y + x[k].z * x[k].z + x[k].w * x[k].w;
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    named_sync(1, nt);
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < SG_CW; ++w) t += red[w];
+    const float inv = rsqrtf(t / (float)d + eps);
+#pragma unroll
+    for (int k = 0; k < SG_PV; ++k) {
+        const int c = threadIdx.x + k * nt;
+        if (c < d / 4)
+            ((float4 *)dst)[c] = make_float4(x[k].x * inv * bf_lo(g[k].x), x[k].y * inv * bf_hi(g[k].x),
+                                             x[k].z * inv * bf_lo(g[k].y), x[k].w * inv * bf_hi(g[k].y));
+    }
+    named_sync(1, nt);
+}
+
 __device__ __forceinline__ void consumer_copy(float *dst, const float *src, int n) {
     for (int c = threadIdx.x; c < n / 4; c += SG_CW * 32)
         ((float4 *)dst)[c] = src ? ((const float4 *)src)[c] : make_float4(0.f, 0.f, 0.f, 0.f);
@@ -263,7 +311,14 @@ __device__ int cdf_pick_regs(const float (&w)[PER], int e0, int n, float target_
     return chosen;
 }
 
-constexpr int SG_PICK_PER = 2;   // entries per thread in a pick (blocks and tiles per block <= 2 x 288)
+constexpr int SG_PICK_PER = 2;    // block entries per thread in the first pick (blocks <= 2 x 288)
+constexpr int SG_PICK2_PER = 4;   // ids per thread in the second pick (ids per block <= 4 x 288)
+
+// Logits of row b at the current chain step: the caller's draft_logits when
+// given, else the workspace row.
+__device__ __forceinline__ float *lm_zrow(const StreamArgs &a, int b) {
+    return a.logits ? a.logits + ((size_t)b * a.K + a.step) * a.dim.V : a.z + (size_t)b * a.dim.V;
+}
 
 template <int RG>
 __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row, const float *xs, float *ybuf,
@@ -271,13 +326,13 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
     __shared__ MS shm[SG_CW + 1];
     __shared__ AM sha[SG_CW + 1];
     __shared__ float sh_scan[33];
-    __shared__ int s_tok;
     __shared__ float s_e;
     const Dims &D = a.dim;
     const bool greedy = a.temperature == 0.f;
     const float invT = greedy ? 1.f : 1.f / a.temperature;
     const int t = threadIdx.x;
     const float4 *cst = a.cta_stats + (size_t)b * nblk;
+    const float u = greedy ? 0.f : a.u_draft[(size_t)b * a.K + a.step];
 
     // level 1: one load per block entry; (max, sum) and argmax over all blocks
     const int e0 = t * SG_PICK_PER;
@@ -309,62 +364,31 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
 #pragma unroll
         for (int k = 0; k < SG_PICK_PER; ++k) c1[k] = v[k].x == -INFINITY ? 0.f : v[k].y * __expf(v[k].x - M);
         // the target u * S needs the total: the pick's own scan provides it
-        const float u = a.u_draft[(size_t)b * a.K + a.step];
         float before1;
         const int blk = cdf_pick_regs<SG_PICK_PER>(c1, e0, nblk, u, true, &before1, &S, sh_scan);
         const float target = u * S;
-        // level 2: tiles (stages) of that block
+        // level 2: every logit of that block's id range, written by the main
+        // pass (one load each, all in flight together)
         const int st0 = (int)((long long)a.n_stages * blk / nblk);
         const int st1 = (int)((long long)a.n_stages * (blk + 1) / nblk);
-        const float4 *tst = a.tile_stats + (size_t)b * a.n_stages + st0;
-        float c2[SG_PICK_PER];
+        const int lo = st0 * a.items, hi = min(D.V, st1 * a.items);
+        const float *zr = lm_zrow(a, b);
+        const int f0 = t * SG_PICK2_PER;
+        float c2[SG_PICK2_PER];
 #pragma unroll
-        for (int k = 0; k < SG_PICK_PER; ++k) {
-            const float4 w2 = e0 + k < st1 - st0 ? __ldcg(tst + e0 + k) : make_float4(-INFINITY, 0.f, 0.f, 0.f);
-            c2[k] = w2.x == -INFINITY ? 0.f : w2.y * __expf(w2.x - M);
+        for (int k = 0; k < SG_PICK2_PER; ++k) {
+            const int n = lo + f0 + k;
+            c2[k] = n < hi ? __ldcg(zr + n) : -INFINITY;
         }
+#pragma unroll
+        for (int k = 0; k < SG_PICK2_PER; ++k) c2[k] = c2[k] == -INFINITY ? 0.f : __expf(c2[k] * invT - M);
         float before2, S2;
-        const int tl = cdf_pick_regs<SG_PICK_PER>(c2, e0, st1 - st0, target - before1, false, &before2, &S2, sh_scan);
-        const float before = before1 + before2;
-        // level 3: recompute that tile's logits (same arithmetic as the first pass)
-        const int lo = (st0 + tl) * a.items, hi = min(D.V, lo + a.items);
-        const int warp = t >> 5, lane = t & 31;
-        for (int n = lo + warp; n < hi; n += SG_CW + 1) {
-            float acc[RG];
-            global_dot<RG>(a.W + (size_t)n * D.d, xs, D.d, acc);
-            if (lane == 0) ybuf[n - lo] = acc[rr] * invT;
-        }
+        const int idx = cdf_pick_regs<SG_PICK2_PER>(c2, f0, hi - lo, target - before1, false, &before2, &S2, sh_scan);
+#pragma unroll
+        for (int k = 0; k < SG_PICK2_PER; ++k)
+            if (f0 + k == idx) s_e = c2[k];
         __syncthreads();
-        if (warp == 0) {
-            float run = before;
-            int tok = -1, lastp = -1;
-            float etok = 0.f, elast = 0.f;
-            for (int base = lo; base < hi && tok < 0; base += 32) {
-                const int n = base + lane;
-                const float e = n < hi ? __expf(ybuf[n - lo] - M) : 0.f;
-                const float inc = warp_incl_scan(e) + run;
-                const unsigned hit = __ballot_sync(0xffffffffu, n < hi && e > 0.f && target < inc);
-                const unsigned pos = __ballot_sync(0xffffffffu, n < hi && e > 0.f);
-                if (pos) {
-                    const int l2 = 31 - __clz(pos);
-                    lastp = base + l2;
-                    elast = __shfl_sync(0xffffffffu, e, l2);
-                }
-                if (hit) {
-                    const int l2 = __ffs(hit) - 1;
-                    tok = base + l2;
-                    etok = __shfl_sync(0xffffffffu, e, l2);
-                }
-                run = __shfl_sync(0xffffffffu, inc, 31);
-            }
-            if (lane == 0) {
-                if (tok < 0) { tok = lastp >= 0 ? lastp : lo; etok = elast; }
-                s_tok = tok;
-                s_e = etok;
-            }
-        }
-        __syncthreads();
-        token = s_tok;
+        token = lo + idx;
         qx = s_e / S;
     }
     if (t == 0) {
@@ -378,10 +402,14 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
     if (a.step + 1 < a.K) {
         // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[token]
         const float *xl = a.x_in + (size_t)src_row * D.d;
-        for (int k = t; k < D.d; k += blockDim.x) a.s_chain[(size_t)b * D.d + k] = xl[k];
-        __syncthreads();
         const uint16_t *e = a.embed + (size_t)token * D.d;
-        for (int k = t; k < D.d; k += blockDim.x) a.x_chain[(size_t)b * D.d + k] = bf_to_f(e[k]);
+        for (int k = 4 * t; k < D.d; k += 4 * blockDim.x) {   // d is a multiple of 256
+            const float4 xv = __ldcg((const float4 *)(xl + k));
+            const uint2 ev = *(const uint2 *)(e + k);
+            *(float4 *)(a.s_chain + (size_t)b * D.d + k) = xv;
+            *(float4 *)(a.x_chain + (size_t)b * D.d + k) =
+                make_float4(bf_lo(ev.x), bf_hi(ev.x), bf_lo(ev.y), bf_hi(ev.y));
+        }
     }
     __syncthreads();
 }
@@ -451,7 +479,8 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kerne
         }
     } else {
         // ---- consumers
-        pdl_wait();
+        // the row map and the norm gain were written before the chain started:
+        // read them while the previous kernel finishes
         if (threadIdx.x < RG) {
             int b = 0, pos = 0, src = 0;
             bool act;
@@ -469,12 +498,25 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kerne
             s_act[threadIdx.x] = act;
             s_src[threadIdx.x] = src;
         }
+        constexpr bool NORM = MODE == G_QKV || MODE == G_GATEUP || MODE == G_LM;
+        const bool regs = D.d <= SG_PV * 4 * SG_CW * 32;
+        uint2 gv[SG_PV];
+        if (NORM && regs) load_gain4(gv, a.gain, D.d / 4);
         named_sync(1, SG_CW * 32);
+        pdl_wait();
         for (int rr = 0; rr < RG; ++rr) {
             const bool act = s_act[rr];
             const int r = s_src[rr];
             float *row = xs + (size_t)rr * Kd;
-            if (MODE == G_QKV) {
+            if (NORM && regs) {
+                // every load of the row issued at once: x (and the context slot for qkv)
+                const float *xsrc = MODE == G_LM ? a.x_in : a.x;
+                float4 xv[SG_PV], sv[SG_PV];
+                load_vec4(xv, act ? xsrc + (size_t)r * D.d : nullptr, D.d / 4);
+                if (MODE == G_QKV) load_vec4(sv, act ? a.s + (size_t)r * D.d : nullptr, D.d / 4);
+                consumer_rmsnorm_regs(MODE == G_QKV ? row + D.d : row, xv, gv, D.d, D.eps, red);
+                if (MODE == G_QKV) store_vec4(row, sv, D.d / 4);
+            } else if (MODE == G_QKV) {
                 consumer_copy(row, act ? a.s + (size_t)r * D.d : nullptr, D.d);
                 consumer_rmsnorm(row + D.d, act ? a.x + (size_t)r * D.d : nullptr, a.gain, D.d, D.eps, red);
             } else if (MODE == G_GATEUP) {
@@ -563,8 +605,7 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kerne
 #pragma unroll
                     for (int rr = 0; rr < RG; ++rr) {
                         const float z = acc[i][rr];
-                        if (a.logits && lane == 0 && s_act[rr])
-                            a.logits[((size_t)(r0 + rr) * a.K + a.step) * D.V + item] = z;
+                        if (lane == 0 && s_act[rr]) lm_zrow(a, r0 + rr)[item] = z;
                         const float y = z * invT;
                         if (y > tm[rr]) { ts[rr] = ts[rr] * __expf(tm[rr] - y) + 1.f; tm[rr] = y; }
                         else ts[rr] += __expf(y - tm[rr]);
@@ -573,9 +614,6 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kerne
                 }
 #pragma unroll
                 for (int rr = 0; rr < RG; ++rr) {
-                    if (lane == 0 && r0 + rr < a.B)
-                        a.tile_stats[(size_t)(r0 + rr) * a.n_stages + st] =
-                            make_float4(tm[rr], ts[rr], tbv[rr], __int_as_float(tbi[rr]));
                     const MS c = ms_combine(MS{wm[rr], ws[rr]}, MS{tm[rr], ts[rr]});
                     wm[rr] = c.m;
                     ws[rr] = c.s;
@@ -670,8 +708,9 @@ bool stream_supported(GemvMode mode, const Dims &D, int rg, int sms) {
     const StreamPlan p = stream_plan(mode, D, sms);
     if (stream_smem(mode, D, rg, p) > 200 * 1024) return false;
     // the LM head's sampler holds at most SG_PICK_PER entries per thread at each level
-    const int cap = SG_PICK_PER * SG_THREADS;
-    if (mode == G_LM && (p.blocks > cap || (p.n_stages + p.blocks - 1) / p.blocks > cap)) return false;
+    if (mode == G_LM && (p.blocks > SG_PICK_PER * SG_THREADS ||
+                         (long long)((p.n_stages + p.blocks - 1) / p.blocks) * p.items > SG_PICK2_PER * SG_THREADS))
+        return false;
     return true;
 }
 
