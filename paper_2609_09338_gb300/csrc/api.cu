@@ -1,6 +1,7 @@
 // C ABI: argument validation, workspace layout and launch sequencing.
 #include <atomic>
 #include <cmath>
+#include <cstdlib>
 #include <cstdarg>
 #include <cstdio>
 #include <cstring>
@@ -42,6 +43,7 @@ struct osprey_ctx {
     osprey_weights w;
     Dims dim;
     int sms;
+    int attn_cs;    // cluster size of the attention kernel (0: split partials in global memory)
     double inv_freq[64];
     int n_probe;
     cudaEvent_t *probe_begin, *probe_end;
@@ -99,6 +101,12 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
     if (e == cudaSuccess) e = cudaDeviceGetAttribute(&ctx->sms, cudaDevAttrMultiProcessorCount, dev);
     if (e == cudaSuccess) e = draft_set_attributes();
     if (e == cudaSuccess) e = stream_set_attributes();
+    if (e == cudaSuccess) {
+        // OSPREY_ATTN_CLUSTER=0 selects the attention kernel that merges split
+        // partials through global memory (also used where clusters cannot run)
+        const char *env = std::getenv("OSPREY_ATTN_CLUSTER");
+        ctx->attn_cs = env && env[0] == '0' ? 0 : attn_cluster_size(ctx->dim);
+    }
     if (e != cudaSuccess) {
         cudaGetLastError();   // do not leave the error pending for the caller's next CUDA call
         delete ctx;
@@ -382,8 +390,8 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.dim = D;
             at.map = map;
             at.R = R;
-            at.n_splits = ns;
-            at.split_len = attn_split_len(max_ctx, ns);
+            at.n_splits = ctx->attn_cs ? ctx->attn_cs : ns;
+            at.split_len = attn_split_len(max_ctx, at.n_splits);
             at.q = ws.q;
             at.k_pages = g.k_pages;
             at.v_pages = g.v_pages;
@@ -392,7 +400,8 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.part = ws.attn_part;
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
-            if ((e = launch_attn(at, s)) != cudaSuccess) return cuda_fail(e, "attention launch");
+            e = ctx->attn_cs ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
+            if (e != cudaSuccess) return cuda_fail(e, "attention launch");
             g.W = (const uint16_t *)W.W_o[l];
             g.xin = ws.attn_out;
             if ((rc = gemv(G_OPROJ, "o-proj launch")) != OSPREY_OK) return rc;

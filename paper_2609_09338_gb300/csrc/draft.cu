@@ -20,6 +20,8 @@
 #include "internal.h"
 #include "tma.cuh"
 
+#include <cooperative_groups.h>
+
 namespace osp {
 
 constexpr int GT = 256;          // threads per GEMV / LM-head block
@@ -419,6 +421,200 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
 }
 
 // ---------------------------------------------------------------------------
+// Split-KV GQA decode attention with the split merge kept on chip.  A cluster
+// of CS blocks takes one (row, KV head); block k of the cluster takes the k-th
+// key range, its 8 warps the range's pages round-robin.  Each block reduces its
+// warps in shared memory; after a cluster barrier every block merges one slice
+// of the G x HD outputs from all CS block partials through distributed shared
+// memory, and a second barrier keeps the partials alive until all slices are
+// done.  Every block of a cluster shares the row, so a block either reaches both
+// barriers or its whole cluster returns before the first.
+// Before griddepcontrol.wait (for G <= 2) a warp already loads its first page
+// id and the K/V rows of that page below pos0, the context committed before
+// this draft call, which no kernel of the call writes.
+#ifndef OSP_ATTN_CS
+#define OSP_ATTN_CS 8       // blocks per cluster (16 needs the non-portable cluster size)
+#endif
+#ifndef OSP_ATTN_WARPS
+#define OSP_ATTN_WARPS 8    // warps per block
+#endif
+constexpr int ACT = OSP_ATTN_WARPS * 32;
+
+template <int HD, int G, int CS>
+__global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
+    namespace cg = cooperative_groups;
+    constexpr int LPK = HD / 8;
+    constexpr int KPL = 32 / LPK;
+    constexpr int NIT = 16 / KPL;     // loads per page (16 positions)
+    constexpr int NW = ACT / 32;
+    constexpr bool PREFETCH = G <= 2;
+    constexpr int SLICE = G * HD / CS;   // outputs merged by each block of the cluster
+    static_assert(SLICE <= ACT && SLICE * CS == G * HD, "slice");
+    __shared__ float sm_m[NW][G], sm_l[NW][G];
+    __shared__ float sm_acc[NW][G][HD];
+    __shared__ float bm[G], bl[G];
+    __shared__ float bacc[G][HD];
+    cg::cluster_group cluster = cg::this_cluster();
+    const Dims &D = a.dim;
+    const int split = (int)cluster.block_rank(), kvh = blockIdx.y, r = blockIdx.z;
+    pdl_trigger();   // the next projection may start streaming its weights
+    int b, pos;
+    if (!a.map.row(r, b, pos)) return;   // the whole cluster (same row) leaves here
+    const int n_keys = pos + 1, pos0 = a.map.pos0[b];
+    const int k_begin = split * a.split_len;
+    const int k_end = min(n_keys, k_begin + a.split_len);
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int kg = lane / LPK, dl = (lane % LPK) * 8;
+    const float scale = rsqrtf((float)HD);
+    const size_t head_stride = (size_t)D.P * HD;
+
+    int pg = k_begin / D.P + warp;
+    uint4 kr[NIT], vr[NIT];
+    const uint16_t *kb0 = nullptr, *vb0 = nullptr;
+    bool first = PREFETCH && pg * D.P < k_end;
+    if (first) {
+        const int page = __ldg(a.page_table + (size_t)b * a.max_pages + pg);
+        kb0 = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
+        vb0 = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
+#pragma unroll
+        for (int it = 0; it < NIT; ++it) {
+            const int slot = it * KPL + kg;
+            if (pg * D.P + slot < pos0) {
+                kr[it] = ld_stream(kb0 + slot * HD + dl);
+                vr[it] = ld_stream(vb0 + slot * HD + dl);
+            }
+        }
+    }
+    pdl_wait();   // q and this call's K/V rows come from the QKV kernels
+
+    float q[G][8], acc[G][8], m_run[G], l[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+        const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dl;
+#pragma unroll
+        for (int e = 0; e < 8; ++e) { q[g][e] = qp[e] * scale; acc[g][e] = 0.f; }
+        m_run[g] = -INFINITY;
+        l[g] = 0.f;
+    }
+    for (; pg * D.P < k_end; pg += NW) {
+        if (first) {
+            // the prefetched page: rows of this call now
+#pragma unroll
+            for (int it = 0; it < NIT; ++it) {
+                const int slot = it * KPL + kg;
+                if (pg * D.P + slot >= pos0) {
+                    kr[it] = ld_stream(kb0 + slot * HD + dl);
+                    vr[it] = ld_stream(vb0 + slot * HD + dl);
+                }
+            }
+            first = false;
+        } else {
+            const int page = a.page_table[(size_t)b * a.max_pages + pg];
+            const uint16_t *kb = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
+            const uint16_t *vb = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
+#pragma unroll
+            for (int it = 0; it < NIT; ++it) {
+                const int slot = it * KPL + kg;
+                kr[it] = ld_stream(kb + slot * HD + dl);
+                vr[it] = ld_stream(vb + slot * HD + dl);
+            }
+        }
+#pragma unroll
+        for (int g = 0; g < G; ++g) {
+            float sc[NIT];
+            float mx = -INFINITY;
+#pragma unroll
+            for (int it = 0; it < NIT; ++it) {
+                float kf[8];
+                unpack8(kr[it], kf);
+                float p = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) p = fmaf(q[g][e], kf[e], p);
+#pragma unroll
+                for (int o = LPK / 2; o; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
+                const int key = pg * D.P + it * KPL + kg;
+                sc[it] = key < k_end ? p : -INFINITY;
+                mx = fmaxf(mx, sc[it]);
+            }
+#pragma unroll
+            for (int o = LPK; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+            const float m_new = fmaxf(m_run[g], mx);
+            if (m_new == -INFINITY) continue;   // no key of this page for the warp yet
+            const float corr = __expf(m_run[g] - m_new);
+            l[g] *= corr;
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[g][e] *= corr;
+#pragma unroll
+            for (int it = 0; it < NIT; ++it) {
+                const float p = __expf(sc[it] - m_new);
+                float vf[8];
+                unpack8(vr[it], vf);
+                l[g] += p;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p, vf[e], acc[g][e]);
+            }
+            m_run[g] = m_new;
+        }
+    }
+    // merge the key groups of the warp, then the warps of the block
+#pragma unroll
+    for (int g = 0; g < G; ++g) {
+#pragma unroll
+        for (int o = LPK; o < 32; o <<= 1) {
+            l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) acc[g][e] += __shfl_xor_sync(0xffffffffu, acc[g][e], o);
+        }
+        if (lane < LPK) {
+#pragma unroll
+            for (int e = 0; e < 8; ++e) sm_acc[warp][g][dl + e] = acc[g][e];
+        }
+        if (lane == 0) { sm_m[warp][g] = m_run[g]; sm_l[warp][g] = l[g]; }
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < G * HD; idx += ACT) {
+        const int g = idx / HD, dim = idx % HD;
+        float M = -INFINITY;
+#pragma unroll
+        for (int w = 0; w < NW; ++w) M = fmaxf(M, sm_m[w][g]);
+        float num = 0.f, den = 0.f;
+        if (M != -INFINITY)
+#pragma unroll
+            for (int w = 0; w < NW; ++w) {
+                const float f = sm_m[w][g] == -INFINITY ? 0.f : __expf(sm_m[w][g] - M);
+                num = fmaf(f, sm_acc[w][g][dim], num);
+                den = fmaf(f, sm_l[w][g], den);
+            }
+        bacc[g][dim] = num;
+        if (dim == 0) { bm[g] = M; bl[g] = den; }
+    }
+    cluster.sync();   // every block's partial is visible to its cluster
+    if (threadIdx.x < SLICE) {
+        const int idx = split * SLICE + threadIdx.x;
+        const int g = idx / HD, dim = idx % HD;
+        float pm[CS], pl[CS], pa[CS];
+#pragma unroll
+        for (int k = 0; k < CS; ++k) {
+            pm[k] = *cluster.map_shared_rank(&bm[g], k);
+            pl[k] = *cluster.map_shared_rank(&bl[g], k);
+            pa[k] = *cluster.map_shared_rank(&bacc[g][dim], k);
+        }
+        float M = -INFINITY;
+#pragma unroll
+        for (int k = 0; k < CS; ++k) M = fmaxf(M, pm[k]);
+        float num = 0.f, den = 0.f;
+#pragma unroll
+        for (int k = 0; k < CS; ++k) {
+            const float f = pm[k] == -INFINITY ? 0.f : __expf(pm[k] - M);
+            num = fmaf(f, pa[k], num);
+            den = fmaf(f, pl[k], den);
+        }
+        a.out[(size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num / den;
+    }
+    cluster.sync();   // the partials stay readable until every slice is merged
+}
+
+// ---------------------------------------------------------------------------
 // LM head + on-chip sampling.
 __device__ __forceinline__ void warp_range(int V, int warps_total, int gw, int &lo, int &hi) {
     lo = (int)(((long long)V * gw) / warps_total);
@@ -762,6 +958,104 @@ cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s) {
         case 2: e = launch_attn_t<64, 2>(a, s); break;
         case 4: e = launch_attn_t<64, 4>(a, s); break;
         default: e = launch_attn_t<64, 8>(a, s); break;
+        }
+    }
+    count_launch();
+    return e;
+}
+
+template <int HD, int G, int CS>
+static cudaLaunchConfig_t attn_cluster_cfg(const AttnArgs &a, cudaStream_t s, cudaLaunchAttribute (&attr)[2]) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(CS, a.dim.Hkv, a.R);
+    cfg.blockDim = dim3(ACT);
+    cfg.stream = s;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cfg;
+}
+
+// Whether clusters of CS blocks of this kernel can be resident on the device
+// (sets the non-portable size attribute when CS > 8).
+template <int HD, int G, int CS>
+static bool attn_cluster_ok(const Dims &D) {
+    auto k = attn_cluster_kernel<HD, G, CS>;
+    if (CS > 8 && cudaFuncSetAttribute(k, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    AttnArgs a{};
+    a.dim = D;
+    a.R = 1;
+    cudaLaunchAttribute attr[2];
+    cudaLaunchConfig_t cfg = attn_cluster_cfg<HD, G, CS>(a, nullptr, attr);
+    cfg.numAttrs = 1;   // the occupancy query takes the cluster shape only
+    int n = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, k, &cfg) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return n >= 1;
+}
+
+template <int HD, int G>
+static int attn_cluster_size_t(const Dims &D) {
+    if (OSP_ATTN_CS == 16 && attn_cluster_ok<HD, G, 16>(D)) return 16;
+    if (attn_cluster_ok<HD, G, 8>(D)) return 8;
+    return 0;
+}
+
+int attn_cluster_size(const Dims &D) {
+    const int G = D.Hq / D.Hkv;
+    if (D.hd == 128) {
+        switch (G) {
+        case 1: return attn_cluster_size_t<128, 1>(D);
+        case 2: return attn_cluster_size_t<128, 2>(D);
+        case 4: return attn_cluster_size_t<128, 4>(D);
+        default: return attn_cluster_size_t<128, 8>(D);
+        }
+    }
+    switch (G) {
+    case 1: return attn_cluster_size_t<64, 1>(D);
+    case 2: return attn_cluster_size_t<64, 2>(D);
+    case 4: return attn_cluster_size_t<64, 4>(D);
+    default: return attn_cluster_size_t<64, 8>(D);
+    }
+}
+
+template <int HD, int G>
+static cudaError_t launch_attn_cluster_t(const AttnArgs &a, int cs, cudaStream_t s) {
+    cudaLaunchAttribute attr[2];
+    if (cs == 16) {
+        cudaLaunchConfig_t cfg = attn_cluster_cfg<HD, G, 16>(a, s, attr);
+        return cudaLaunchKernelEx(&cfg, attn_cluster_kernel<HD, G, 16>, a);
+    }
+    cudaLaunchConfig_t cfg = attn_cluster_cfg<HD, G, 8>(a, s, attr);
+    return cudaLaunchKernelEx(&cfg, attn_cluster_kernel<HD, G, 8>, a);
+}
+
+cudaError_t launch_attn_cluster(const AttnArgs &a, int cs, cudaStream_t s) {
+    const int G = a.dim.Hq / a.dim.Hkv;
+    cudaError_t e;
+    if (a.dim.hd == 128) {
+        switch (G) {
+        case 1: e = launch_attn_cluster_t<128, 1>(a, cs, s); break;
+        case 2: e = launch_attn_cluster_t<128, 2>(a, cs, s); break;
+        case 4: e = launch_attn_cluster_t<128, 4>(a, cs, s); break;
+        default: e = launch_attn_cluster_t<128, 8>(a, cs, s); break;
+        }
+    } else {
+        switch (G) {
+        case 1: e = launch_attn_cluster_t<64, 1>(a, cs, s); break;
+        case 2: e = launch_attn_cluster_t<64, 2>(a, cs, s); break;
+        case 4: e = launch_attn_cluster_t<64, 4>(a, cs, s); break;
+        default: e = launch_attn_cluster_t<64, 8>(a, cs, s); break;
         }
     }
     count_launch();

@@ -161,6 +161,10 @@ cudaError_t stream_set_attributes();
 cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s);
 cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaStream_t s);
 cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s);
+// Cluster size (16 or 8) the on-chip-merge attention can run with on the
+// current device for this shape, 0 if clusters are not available.
+int attn_cluster_size(const Dims &D);
+cudaError_t launch_attn_cluster(const AttnArgs &a, int cs, cudaStream_t s);
 cudaError_t launch_lm(const LmArgs &a, int rg, int blocks, cudaStream_t s);
 int attn_splits(int R, int Hkv, int max_ctx, int sms);
 int attn_split_len(int max_ctx, int n_splits);

@@ -47,6 +47,12 @@ namespace osp {
 #ifndef OSP_SG_NPROD
 #define OSP_SG_NPROD 1   // producer lanes; lane p issues stages p, p + NPROD, ...
 #endif
+// L2 priority of the weight streams: the LM head is loaded evict-first (it is
+// read once per chain step and does not fit in L2); layer weights at normal
+// priority.  Evict-last would keep layer weights in L2 across the chain steps
+// of a call, but such lines also survive later traffic (a flush of twice the
+// L2 size left about a third of them resident), and the layer weights are
+// fetched while the previous kernel finishes, off the critical path, anyway.
 
 
 constexpr int SG_CW = 8;                      // consumer warps
@@ -454,7 +460,7 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kerne
     if (warp == SG_CW) {
         // ---- producer: weights do not depend on the previous kernel
         if (lane < OSP_SG_NPROD) {
-            const uint64_t pol = MODE == G_LM ? policy_evict_first() : policy_evict_last();
+            const uint64_t pol = policy_evict_first();
             int issued = 0;
             for (int j = lane; j < nloc; j += OSP_SG_NPROD) {
                 const int slot = j % SG_NST;
@@ -467,8 +473,12 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kerne
                 const StageGeom g = stage_geom(a, stage_of(j), Kd);
                 uint8_t *dst = ring + (size_t)slot * a.stage_bytes;
                 mbar_arrive_expect_tx(&full[slot], PAIR ? 2 * g.seg_bytes : g.seg_bytes);
-                bulk_g2s_hint(dst, g.src0, g.seg_bytes, &full[slot], pol);
-                if (PAIR) bulk_g2s_hint(dst + (size_t)NI * Kd * 2, g.src1, g.seg_bytes, &full[slot], pol);
+                if (MODE == G_LM) {
+                    bulk_g2s_hint(dst, g.src0, g.seg_bytes, &full[slot], pol);
+                } else {
+                    bulk_g2s(dst, g.src0, g.seg_bytes, &full[slot]);
+                    if (PAIR) bulk_g2s(dst + (size_t)NI * Kd * 2, g.src1, g.seg_bytes, &full[slot]);
+                }
                 issued = j + 1;
             }
             if (s_abort) {

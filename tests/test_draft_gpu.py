@@ -114,8 +114,13 @@ def check_case(case, o=None, min_checked_frac=0.5):
         pos = np.arange(case["ctx"][b], case["ctx"][b] + nn + K - 1)
         for name, pages in (("new_k", g["k_pages"]), ("new_v", g["v_pages"])):
             got = gather_positions(pages, case["kv"]["page_table"][b], pos)
-            # both sides hold bf16 values: equal up to one rounding step
-            np.testing.assert_allclose(got, o[name][i], rtol=2.0 ** -7, atol=1e-4)
+            want = o[name][i]
+            # both sides hold bf16 values: equal up to one rounding step at the
+            # value's own scale; near zero a value two layers deep also carries the
+            # float32 accumulation error of its row, bounded here by a quarter bf16
+            # step at the row's largest magnitude
+            row = np.abs(want).max(-1, keepdims=True)
+            np.testing.assert_array_less(np.abs(got - want), 2.0 ** -7 * np.abs(want) + 2.0 ** -9 * row + 1e-6)
     return checked, len(idx) * K
 
 
@@ -216,4 +221,19 @@ def test_workload_full_size(name, T, sample):
     wl = WORKLOADS[name]
     ctx = syn.make_contexts(wl)
     case = run_case(wl.shape, ctx, wl.K, T, wl.seed, sample_seqs=sample)
+    check_case(case)
+
+
+@pytest.mark.parametrize("which", ["ragged", "hd128_g4"])
+def test_attention_split_partials_in_global_memory(which, monkeypatch):
+    """The attention kernel that merges its split partials through global memory
+    (selected with OSPREY_ATTN_CLUSTER=0, and used where thread-block clusters
+    cannot run) against the oracle."""
+    monkeypatch.setenv("OSPREY_ATTN_CLUSTER", "0")
+    if which == "ragged":
+        shape = replace(TINY, n_layers=2, n_q_heads=8, n_kv_heads=2)
+        case = run_case(shape, [5, 0, 31, 64], 3, 0.0, 31, n_new=[3, 1, 2, 3], max_new=3)
+    else:
+        shape = replace(TINY, head_dim=128, n_q_heads=8, n_kv_heads=2, d_model=512, vocab=5000)
+        case = run_case(shape, [100, 1000, 17], 5, 0.7, 41, peaked=True)
     check_case(case)
