@@ -36,8 +36,8 @@ from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: 
 # two captured launches of this workload under ncu --set full); valid
 # only for the stream.cu it was taken on.
 LM_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/stream.cu",
-              "sha256": "0ab17c7a28a51773fee611c3edd7e72ad1a37cda19fd9f132d0eae5d07c8223e",
-              "bytes_per_launch": 314_541_312}
+              "sha256": "6d2d8e13865a495755e07e57e7d0dc969b35d6497914adcb89b08b88e1e83221",
+              "bytes_per_launch": 314_518_784}
 
 
 def _sha(path):
