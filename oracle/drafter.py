@@ -127,8 +127,13 @@ class _SeqCache:
 
 
 def forward_row(W: dict, shape, cache: _SeqCache, token: int, s: np.ndarray, pos: int,
-                new_k: list, new_v: list) -> np.ndarray:
-    """One drafter position through every layer; returns x_L (pre final norm)."""
+                new_k: list, new_v: list, forced=None) -> np.ndarray:
+    """One drafter position through every layer; returns x_L (pre final norm).
+
+    new_k/new_v receive the rows this computation produces.  With ``forced`` =
+    (k [L, Hkv, hd], v [L, Hkv, hd]) the cache holds those rows instead (another
+    run's cached values at this position), so attention reads the same cache
+    state as that run."""
     Hq, Hkv, hd = shape.n_q_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
     x = W["embed"][token].copy()
@@ -141,8 +146,8 @@ def forward_row(W: dict, shape, cache: _SeqCache, token: int, s: np.ndarray, pos
         q, k = rope(q, pos, theta), round_to_bf16(rope(k, pos, theta))
         v = round_to_bf16(v)
         assert cache.length(l) == pos, "positions must be contiguous"
-        cache.k[l].append(k)
-        cache.v[l].append(v)
+        cache.k[l].append(k if forced is None else np.asarray(forced[0][l], dtype=np.float64))
+        cache.v[l].append(v if forced is None else np.asarray(forced[1][l], dtype=np.float64))
         new_k[l].append(k)
         new_v[l].append(v)
         attn = gqa_attention(q, np.asarray(cache.k[l]), np.asarray(cache.v[l]))
@@ -189,7 +194,8 @@ def sample(z: np.ndarray, temperature: float, u: float) -> dict:
 def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
                ctx_lens: np.ndarray, tokens: np.ndarray, feats: np.ndarray,
                n_new: np.ndarray, K: int, temperature: float, u_draft: np.ndarray,
-               forced_tokens: np.ndarray | None = None, widened: dict | None = None) -> dict:
+               forced_tokens: np.ndarray | None = None, widened: dict | None = None,
+               forced_kv: list | None = None) -> dict:
     """One draft call for a batch of sequences.
 
     prefix_k/prefix_v: [L, sum(ctx), Hkv, hd] bf16 bits, sequence b owning rows
@@ -199,6 +205,14 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
     row's output gives draft token 1; chain steps 2..K feed the sampled token
     (or ``forced_tokens[b, k-1]`` when given, to follow another run's chain) and
     the previous row's x_L in the context slot (Sec. 3.4).
+
+    forced_kv (optional): per sequence b a pair (k, v) of [L, n_new + K - 1, Hkv,
+    hd] arrays, another run's cached rows at the positions this call writes.  The
+    cache then holds those rows, as the chain follows forced_tokens: each step
+    is computed from the same cache state as that run, while new_k/new_v still
+    report the rows this computation produces.  (Cached rows are bf16, so a
+    difference of one rounding step in a row would otherwise propagate along the
+    chain.)
 
     Returns logits [B, K, V], tokens/qx [B, K], stats [B, K, 2], margins [B, K],
     new_k/new_v: per sequence [L, n_new + K - 1, Hkv, hd], and g [B, d] (the
@@ -219,9 +233,14 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
         new_k = [[] for _ in range(L)]
         new_v = [[] for _ in range(L)]
         nb = int(n_new[b])
+        fk = None if forced_kv is None else forced_kv[b]
+
+        def fr(i):
+            return None if fk is None else (fk[0][:, i], fk[1][:, i])
+
         for j in range(nb):
             c = feature_projection(W["W_c"], widen(feats[b, j]))
-            g = forward_row(W, shape, cache, int(tokens[b, j]), c, L0 + j, new_k, new_v)
+            g = forward_row(W, shape, cache, int(tokens[b, j]), c, L0 + j, new_k, new_v, fr(j))
         for k in range(K):
             h = rmsnorm(g, W["final_norm"], shape.rms_eps)
             z = W["lm_head"] @ h
@@ -234,7 +253,7 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
             if k == K - 1:
                 break
             nxt = int(forced_tokens[b, k]) if forced_tokens is not None else smp["token"]
-            g = forward_row(W, shape, cache, nxt, g, L0 + nb + k, new_k, new_v)
+            g = forward_row(W, shape, cache, nxt, g, L0 + nb + k, new_k, new_v, fr(nb + k))
         out["g"][b] = g
         out["new_k"].append(np.asarray(new_k))
         out["new_v"].append(np.asarray(new_v))

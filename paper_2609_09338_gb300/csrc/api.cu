@@ -8,6 +8,7 @@
 #include <new>
 
 #include "draft.cuh"
+#include "tc.cuh"
 #include "internal.h"
 #include "osprey.h"
 
@@ -44,6 +45,9 @@ struct osprey_ctx {
     Dims dim;
     int sms;
     int attn_cs;    // cluster size of the attention kernel (0: split partials in global memory)
+    bool tc;        // batched rows (3..80) run their projections on tcgen05
+    CUtensorMap tm_c, tm_lm, tm_qkv[OSPREY_MAX_LAYERS], tm_o[OSPREY_MAX_LAYERS], tm_gate[OSPREY_MAX_LAYERS],
+        tm_up[OSPREY_MAX_LAYERS], tm_down[OSPREY_MAX_LAYERS];
     double inv_freq[64];
     int n_probe;
     cudaEvent_t *probe_begin, *probe_end;
@@ -106,6 +110,20 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
         // partials through global memory (also used where clusters cannot run)
         const char *env = std::getenv("OSPREY_ATTN_CLUSTER");
         ctx->attn_cs = env && env[0] == '0' ? 0 : attn_cluster_size(ctx->dim);
+        // OSPREY_TC=0 keeps batched rows on the CUDA-core GEMV
+        const char *tenv = std::getenv("OSPREY_TC");
+        const Dims &D = ctx->dim;
+        const osprey_weights &W = ctx->w;
+        bool tc = !(tenv && tenv[0] == '0') && tc_available() && tc_set_attributes() == cudaSuccess;
+        tc = tc && tc_encode_weight(&ctx->tm_c, W.W_c, D.d, D.feat) && tc_encode_weight(&ctx->tm_lm, W.lm_head, D.V, D.d);
+        for (int l = 0; tc && l < D.L; ++l)
+            tc = tc_encode_weight(&ctx->tm_qkv[l], W.W_qkv[l], (D.Hq + 2 * D.Hkv) * D.hd, 2 * D.d) &&
+                 tc_encode_weight(&ctx->tm_o[l], W.W_o[l], D.d, D.Hq * D.hd) &&
+                 tc_encode_weight(&ctx->tm_gate[l], W.W_gate[l], D.F, D.d) &&
+                 tc_encode_weight(&ctx->tm_up[l], W.W_up[l], D.F, D.d) &&
+                 tc_encode_weight(&ctx->tm_down[l], W.W_down[l], D.d, D.F);
+        ctx->tc = tc;
+        cudaGetLastError();
     }
     if (e != cudaSuccess) {
         cudaGetLastError();   // do not leave the error pending for the caller's next CUDA call
@@ -192,6 +210,15 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
     size_t o_lz = take(4ull * B * D.V);
     size_t o_lc = take(16ull * B * lmp.blocks);
+    // tensor-core path: bf16 operand planes, QKV output, row-sampler partials
+    const long long tc_rows = std::min<long long>(std::max<long long>(R_ext, B), TC_MAX_ROWS);
+    const long long np = (tc_rows + 15) / 16 * 16;
+    const long long nqkv = (long long)(D.Hq + 2 * D.Hkv) * D.hd;
+    const bool tcw = ctx->tc;
+    size_t o_xq = take(tcw ? 2ull * TC_PLANES * np * 2 * D.d : 0), o_yq = take(tcw ? 4ull * np * nqkv : 0);
+    size_t o_xo = take(tcw ? 2ull * TC_PLANES * np * D.Hq * D.hd : 0), o_xg = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
+    size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
+    size_t o_rp = take(tcw ? 16ull * B * row_sample_chunks(D.V) : 0), o_rt = take(tcw ? 4ull * B : 0);
     if (ws && base) {
         char *p = (char *)base;
         ws->seq_valid = (int *)(p + o_valid);
@@ -210,6 +237,14 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->lm_stats = (float4 *)(p + o_ls);
         ws->lm_z = (float *)(p + o_lz);
         ws->lm_cta_stats = (float4 *)(p + o_lc);
+        ws->tc_xq = (uint16_t *)(p + o_xq);
+        ws->tc_yq = (float *)(p + o_yq);
+        ws->tc_xo = (uint16_t *)(p + o_xo);
+        ws->tc_xg = (uint16_t *)(p + o_xg);
+        ws->tc_xh = (uint16_t *)(p + o_xh);
+        ws->tc_xl = (uint16_t *)(p + o_xl);
+        ws->rs_part = (float4 *)(p + o_rp);
+        ws->rs_ticket = (int *)(p + o_rt);
         ws->n_splits_max = ns;
         ws->lm_warps_max = lm_warps;
     }
@@ -317,8 +352,60 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
     g.max_pages = kv->max_pages_per_seq;
     g.n_pages = kv->n_pages;
     for (int i = 0; i < D.hd / 2; ++i) g.inv_freq[i] = ctx->inv_freq[i];
-    if ((e = launch_gemv(G_FEAT, g, gemv_rg(G_FEAT, D, g.R), ctx->sms, s)) != cudaSuccess)
+    // tensor-core path for 3..TC_MAX_ROWS activation rows
+    auto tc_rows = [&](int rows) { return ctx->tc && rows >= 3 && rows <= TC_MAX_ROWS; };
+    auto npad_of = [](int rows) { return (rows + 15) / 16 * 16; };
+    auto tc_gemm = [&](int epi, int rows, int K_, int nout, int planes, const CUtensorMap &wa, const CUtensorMap *wb,
+                       const void *xbuf, bool in_place_rows, float *y, int ldy, uint16_t *h,
+                       const char *what) -> int {
+        const int np = npad_of(rows);
+        CUtensorMap xm;
+        const bool ok = in_place_rows ? tc_encode_rows(&xm, xbuf, rows, np, K_) : tc_encode_operand(&xm, xbuf, planes, np, K_);
+        if (!ok) return fail(OSPREY_ERR_INVALID_ARG, "%s: tensor map encoding failed", what);
+        TcArgs ta{};
+        ta.epi = epi;
+        ta.R = rows;
+        ta.npad = np;
+        ta.K = K_;
+        ta.nout = nout;
+        ta.planes = planes;
+        ta.y = y;
+        ta.x = y;
+        ta.ldy = ldy;
+        ta.h = h;
+        ta.status = dev_status;
+        const cudaError_t e2 = launch_tc(ta, wa, wb, xm, ctx->sms, s);
+        return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
+    };
+    auto planes = [&](const float *src, const uint16_t *gain, int d_, int rows, int ld, int col0, uint16_t *dst,
+                      int rows_per_seq, bool last_of_seq, const char *what) -> int {
+        PlaneArgs pl{};
+        pl.src = src;
+        pl.gain = gain;
+        pl.eps = D.eps;
+        pl.d = d_;
+        pl.R = rows;
+        pl.npad = npad_of(rows);
+        pl.ld = ld;
+        pl.col0 = col0;
+        pl.dst = dst;
+        pl.nnew = ws.seq_nnew;
+        pl.max_new = max_new;
+        pl.last_of_seq = last_of_seq;
+        pl.valid = ws.seq_valid;
+        pl.rows_per_seq = rows_per_seq;
+        const cudaError_t e2 = launch_planes(pl, s);
+        return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
+    };
+    if (tc_rows(B * max_new)) {
+        EmbedArgs ea{D.d, B * max_new, max_new, ws.seq_valid, ws.seq_nnew, tokens, (const uint16_t *)W.embed, ws.x_ext};
+        if ((e = launch_embed_rows(ea, s)) != cudaSuccess) return cuda_fail(e, "embedding launch");
+        const int rc = tc_gemm(TC_STORE, B * max_new, D.feat, D.d, 1, ctx->tm_c, nullptr, feats, true, ws.s_ext, D.d,
+                               nullptr, "feature projection launch");
+        if (rc != OSPREY_OK) return rc;
+    } else if ((e = launch_gemv(G_FEAT, g, gemv_rg(G_FEAT, D, g.R), ctx->sms, s)) != cudaSuccess) {
         return cuda_fail(e, "feature projection launch");
+    }
 
     for (int step = 0; step < K; ++step) {
         const bool ext = step == 0;
@@ -373,7 +460,62 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             }
             return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
         };
-        for (int l = 0; l < D.L; ++l) {
+        const bool tcp = !streamed && tc_rows(R);
+        for (int l = 0; l < D.L && tcp; ++l) {
+            uint16_t *kp = (uint16_t *)kv->k_pages + l * layer_pages;
+            uint16_t *vp = (uint16_t *)kv->v_pages + l * layer_pages;
+            const int nqkv = (D.Hq + 2 * D.Hkv) * D.hd;
+            int rc;
+            // [s; RMSNorm(x)] -> QKV (Eq. 2-3) -> RoPE and the paged K/V rows
+            if ((rc = planes(sb, nullptr, D.d, R, 2 * D.d, 0, ws.tc_xq, rows_per_seq, false, "qkv operand")) != OSPREY_OK ||
+                (rc = planes(x, (const uint16_t *)W.attn_norm[l], D.d, R, 2 * D.d, D.d, ws.tc_xq, rows_per_seq, false,
+                             "qkv operand")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_STORE, R, 2 * D.d, nqkv, TC_PLANES, ctx->tm_qkv[l], nullptr, ws.tc_xq, false, ws.tc_yq, nqkv,
+                              nullptr, "qkv launch")) != OSPREY_OK)
+                return rc;
+            QkvPostArgs qp{};
+            qp.dim = D;
+            qp.map = map;
+            qp.R = R;
+            qp.y = ws.tc_yq;
+            qp.q = ws.q;
+            qp.k_pages = kp;
+            qp.v_pages = vp;
+            qp.page_table = kv->page_table;
+            qp.max_pages = kv->max_pages_per_seq;
+            for (int i = 0; i < D.hd / 2; ++i) qp.inv_freq[i] = ctx->inv_freq[i];
+            if ((e = launch_qkv_post(qp, s)) != cudaSuccess) return cuda_fail(e, "rope launch");
+            AttnArgs at{};
+            at.dim = D;
+            at.map = map;
+            at.R = R;
+            at.n_splits = ctx->attn_cs ? ctx->attn_cs : ns;
+            at.split_len = attn_split_len(max_ctx, at.n_splits);
+            at.q = ws.q;
+            at.k_pages = kp;
+            at.v_pages = vp;
+            at.page_table = kv->page_table;
+            at.max_pages = kv->max_pages_per_seq;
+            at.part = ws.attn_part;
+            at.out = ws.attn_out;
+            at.ticket = ws.attn_ticket;
+            e = ctx->attn_cs ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
+            if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+            // x += W_o attn;  x += W_down (silu(W_g n) * W_u n),  n = RMSNorm(x)
+            const int ha = D.Hq * D.hd;
+            if ((rc = planes(ws.attn_out, nullptr, ha, R, ha, 0, ws.tc_xo, rows_per_seq, false, "o-proj operand")) !=
+                    OSPREY_OK ||
+                (rc = tc_gemm(TC_RESID, R, ha, D.d, TC_PLANES, ctx->tm_o[l], nullptr, ws.tc_xo, false, x, D.d, nullptr,
+                              "o-proj launch")) != OSPREY_OK ||
+                (rc = planes(x, (const uint16_t *)W.ffn_norm[l], D.d, R, D.d, 0, ws.tc_xg, rows_per_seq, false,
+                             "gate/up operand")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_SWIGLU, R, D.d, D.F, TC_PLANES, ctx->tm_gate[l], &ctx->tm_up[l], ws.tc_xg, false, nullptr, 0,
+                              ws.tc_xh, "gate/up launch")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_RESID, R, D.F, D.d, TC_PLANES, ctx->tm_down[l], nullptr, ws.tc_xh, false, x, D.d, nullptr,
+                              "down launch")) != OSPREY_OK)
+                return rc;
+        }
+        for (int l = 0; l < D.L && !tcp; ++l) {
             g.map = map;
             g.R = R;
             g.x = x;
@@ -436,6 +578,40 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             sa.cta_stats = ws.lm_cta_stats;
             sa.ticket = ws.lm_ticket;
             if ((e = launch_stream(G_LM, sa, B, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
+        } else if (tc_rows(B)) {
+            // final RMSNorm rows -> logits (draft_logits when requested) -> on-chip sampling
+            int rc;
+            float *zb = draft_logits ? draft_logits + (size_t)step * D.V : ws.lm_z;
+            const long long ldz = draft_logits ? (long long)K * D.V : D.V;
+            if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand")) !=
+                    OSPREY_OK ||
+                (rc = tc_gemm(TC_STORE, B, D.d, D.V, TC_PLANES, ctx->tm_lm, nullptr, ws.tc_xl, false, zb, (int)ldz, nullptr,
+                              "lm head launch")) != OSPREY_OK)
+                return rc;
+            RowSampleArgs rs{};
+            rs.dim = D;
+            rs.B = B;
+            rs.K = K;
+            rs.step = step;
+            rs.max_new = max_new;
+            rs.src_is_ext = ext;
+            rs.valid = ws.seq_valid;
+            rs.nnew = ws.seq_nnew;
+            rs.z = zb;
+            rs.ldz = ldz;
+            rs.temperature = temperature;
+            rs.u_draft = u_draft;
+            rs.tokens = draft_tokens;
+            rs.qx = draft_qx;
+            rs.stats = draft_stats;
+            rs.x_in = x;
+            rs.x_chain = ws.x_chain;
+            rs.s_chain = ws.s_chain;
+            rs.embed = (const uint16_t *)W.embed;
+            rs.part = ws.rs_part;
+            rs.ticket = ws.rs_ticket;
+            rs.nch = row_sample_chunks(D.V);
+            if ((e = launch_row_sample(rs, s)) != cudaSuccess) return cuda_fail(e, "sampler launch");
         } else {
             LmArgs lm{};
             lm.dim = D;

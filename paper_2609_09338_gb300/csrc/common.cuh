@@ -176,6 +176,14 @@ __device__ __forceinline__ bool arrive_last(int *counter, int total) {
     return s_last;
 }
 
+// cos and sin of the rotary angle pos * inv_freq: the angle is reduced to
+// [0, 2 pi) in double (whole turns removed) before the float sincos.
+__device__ __forceinline__ void rope_cs2(double inv_freq, int pos, float &c, float &s) {
+    const double turns = (double)pos * inv_freq * 0.15915494309189535;
+    const double frac = turns - floor(turns);
+    sincosf((float)(frac * 6.283185307179586), &s, &c);
+}
+
 __device__ __forceinline__ void set_status(int32_t *status, int code) {
     if (status) atomicCAS((int *)status, 0, code);
 }

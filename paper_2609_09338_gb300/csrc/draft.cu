@@ -469,11 +469,19 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
     const size_t head_stride = (size_t)D.P * HD;
 
     int pg = k_begin / D.P + warp;
+    // page ids of the warp's first pages (the page table is fixed for the call)
+    constexpr int NPID = 4;
+    int pid[NPID];
+#pragma unroll
+    for (int k = 0; k < NPID; ++k) {
+        const int pk = pg + k * NW;
+        pid[k] = pk * D.P < k_end ? __ldg(a.page_table + (size_t)b * a.max_pages + pk) : 0;
+    }
     uint4 kr[NIT], vr[NIT];
     const uint16_t *kb0 = nullptr, *vb0 = nullptr;
     bool first = PREFETCH && pg * D.P < k_end;
     if (first) {
-        const int page = __ldg(a.page_table + (size_t)b * a.max_pages + pg);
+        const int page = pid[0];
         kb0 = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
         vb0 = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
 #pragma unroll
@@ -496,7 +504,7 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
         m_run[g] = -INFINITY;
         l[g] = 0.f;
     }
-    for (; pg * D.P < k_end; pg += NW) {
+    for (int it_pg = 0; pg * D.P < k_end; pg += NW, ++it_pg) {
         if (first) {
             // the prefetched page: rows of this call now
 #pragma unroll
@@ -509,7 +517,11 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
             }
             first = false;
         } else {
-            const int page = a.page_table[(size_t)b * a.max_pages + pg];
+            int page = 0;
+#pragma unroll
+            for (int k = 0; k < NPID; ++k)
+                if (k == it_pg) page = pid[k];
+            if (it_pg >= NPID) page = a.page_table[(size_t)b * a.max_pages + pg];
             const uint16_t *kb = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
             const uint16_t *vb = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
 #pragma unroll

@@ -30,6 +30,15 @@ struct DraftWs {
     float4 *lm_stats;                      // [B][lm_warps]
     float *lm_z;                           // [B][V] logits of the chain step (streamed LM head)
     float4 *lm_cta_stats;                  // [B][sms]
+    // tensor-core path (rows padded to np <= 80): bf16 operand planes [TC_PLANES][np][...]
+    uint16_t *tc_xq;                       // [P][np][2d]    [s; RMSNorm(x)] for QKV
+    float *tc_yq;                          // [np][(Hq+2Hkv)hd] QKV output before RoPE
+    uint16_t *tc_xo;                       // [P][np][Hq*hd] attention output
+    uint16_t *tc_xg;                       // [P][np][d]     RMSNorm(x) for gate/up
+    uint16_t *tc_xh;                       // [P][np][F]     SwiGLU hidden (down operand)
+    uint16_t *tc_xl;                       // [P][np][d]     final RMSNorm rows for the LM head
+    float4 *rs_part;                       // [B][V/4096]    row-sampler chunk partials
+    int *rs_ticket;                        // [B]
     int n_splits_max, lm_warps_max;
 };
 

@@ -239,11 +239,6 @@ __device__ __forceinline__ void consumer_copy(float *dst, const float *src, int 
         ((float4 *)dst)[c] = src ? ((const float4 *)src)[c] : make_float4(0.f, 0.f, 0.f, 0.f);
 }
 
-__device__ __forceinline__ void rope_cs2(double inv_freq, int pos, float &c, float &s) {
-    const double turns = (double)pos * inv_freq * 0.15915494309189535;
-    const double frac = turns - floor(turns);
-    sincosf((float)(frac * 6.283185307179586), &s, &c);
-}
 
 struct StageGeom {
     int i0, cnt;                  // first item, items in this stage

@@ -1,0 +1,639 @@
+// Batched-row draft step on tcgen05 tensor cores: streamed swap-AB GEMMs for
+// the projections of Sec. 3.3 (Eq. 1-3, MLP, LM head), operand preparation,
+// RoPE + paged K/V write, and per-row sampling of the draft token (Sec. 3.1).
+//
+// tc_kernel: persistent, one CTA per SM, 6 warps.
+//   warp 0     issues 2-D TMA copies of one 128-row weight tile (two for the
+//              gate/up pair) and the activation planes per 64-wide k-block into
+//              an nst-slot shared-memory ring (128-byte swizzle);
+//   warp 1     issues tcgen05.mma (M 128, N npad, K 16, bf16 in, float32
+//              accumulate in TMEM) per k-block and plane, then commits the
+//              k-block to the slot's "empty" barrier and the tile to the
+//              accumulator's "full" barrier;
+//   warps 2-5  read the accumulator (tcgen05.ld, TMEM lane group = warp % 4)
+//              and run the epilogue while the next tile accumulates into the
+//              other TMEM buffer.
+// Every wait is bounded; on expiry the CTA records OSPREY_ERR_TIMEOUT, stops
+// issuing, lets its copies and MMAs land and frees its TMEM.
+#include <cudaTypedefs.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "internal.h"
+#include "tc.cuh"
+#include "tma.cuh"
+
+namespace osp {
+
+constexpr int TC_THREADS = 192;
+constexpr int TC_ABYTES = 128 * 128;    // weight tile: 128 rows x 64 bf16
+constexpr int TC_MAXST = 8;
+constexpr size_t TC_SMEM_CAP = 200 * 1024;
+#ifndef OSP_TC_SEGKB
+#define OSP_TC_SEGKB 8   // k-blocks (64 wide) per accumulation segment
+#endif
+
+// ---------------------------------------------------------------- tcgen05 PTX
+__device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *m, int x, int y, uint64_t *bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(
+            smem_u32(dst)),
+        "l"(m), "r"(x), "r"(y), "r"(smem_u32(bar))
+        : "memory");
+}
+// Shared-memory matrix descriptor: K-major tile, rows 128 bytes apart inside
+// 8-row (1024-byte) swizzle atoms.
+__device__ __forceinline__ uint64_t tc_desc(uint32_t saddr) {
+    uint64_t d = (uint64_t)((saddr & 0x3FFFFu) >> 4);
+    d |= (uint64_t)1 << 16;              // leading byte offset (unused for swizzled K-major)
+    d |= (uint64_t)(1024 >> 4) << 32;    // stride byte offset: one 8-row atom
+    d |= (uint64_t)1 << 46;              // descriptor version
+    d |= (uint64_t)2 << 61;              // 128-byte swizzle
+    return d;
+}
+// Instruction descriptor, kind::f16: bf16 A and B (K-major), float32 D.
+__host__ __device__ constexpr uint32_t tc_idesc(int M, int N) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(N >> 3) << 17) | ((uint32_t)(M >> 4) << 24);
+}
+__device__ __forceinline__ void tc_mma(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+    asm volatile("{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\ntcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(d),
+                 "l"(a), "l"(b), "r"(idesc), "r"(acc)
+                 : "memory");
+}
+__device__ __forceinline__ void tc_commit(uint64_t *bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(smem_u32(bar))
+                 : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() { asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_fence_after() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
+__device__ __forceinline__ void tc_ld16(uint32_t taddr, float (&v)[16]) {
+    uint32_t r[16];
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]), "=r"(r[8]),
+          "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+#pragma unroll
+    for (int j = 0; j < 16; ++j) v[j] = __uint_as_float(r[j]);
+}
+__device__ __forceinline__ void tc_ld_wait() { asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory"); }
+__device__ __forceinline__ void tc_st16(uint32_t taddr, const float (&v)[16]) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};" ::"r"(
+            taddr),
+        "r"(__float_as_uint(v[0])), "r"(__float_as_uint(v[1])), "r"(__float_as_uint(v[2])), "r"(__float_as_uint(v[3])),
+        "r"(__float_as_uint(v[4])), "r"(__float_as_uint(v[5])), "r"(__float_as_uint(v[6])), "r"(__float_as_uint(v[7])),
+        "r"(__float_as_uint(v[8])), "r"(__float_as_uint(v[9])), "r"(__float_as_uint(v[10])), "r"(__float_as_uint(v[11])),
+        "r"(__float_as_uint(v[12])), "r"(__float_as_uint(v[13])), "r"(__float_as_uint(v[14])), "r"(__float_as_uint(v[15]))
+        : "memory");
+}
+__device__ __forceinline__ void tc_st_wait() { asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory"); }
+
+// x ~= q0 + q1 + q2 with q_i = bf16(x - q0 - ... - q_{i-1}): 8 significant bits
+// per plane, so three planes carry a float32 value's 24 (up to the last rounding).
+__device__ __forceinline__ void tc_split(float x, uint16_t (&q)[TC_PLANES]) {
+    float r = x;
+#pragma unroll
+    for (int i = 0; i < TC_PLANES; ++i) {
+        q[i] = f_to_bf(r);
+        r -= bf_to_f(q[i]);
+    }
+}
+
+// ---------------------------------------------------------------- GEMM kernel
+template <int EPI>
+__global__ void __launch_bounds__(TC_THREADS, 1)
+    tc_kernel(const __grid_constant__ CUtensorMap wa, const __grid_constant__ CUtensorMap wb,
+              const __grid_constant__ CUtensorMap xm, const TcArgs a, int nst) {
+    constexpr bool PAIR = EPI == TC_SWIGLU;
+    constexpr int NA = PAIR ? 2 : 1;
+    extern __shared__ uint8_t raw[];
+    uint8_t *sm = (uint8_t *)(((uintptr_t)raw + 1023) & ~(uintptr_t)1023);
+    __shared__ __align__(8) uint64_t full[TC_MAXST], empty[TC_MAXST], accf[2], acce[2], fin;
+    __shared__ uint32_t s_tmem;
+    __shared__ int s_abort;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int n_items = (a.nout + 127) / 128;
+    const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
+    const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
+    const int nloc = i1 - i0, nkb = a.K / 64, npad = a.npad;
+    const uint32_t bbytes = (uint32_t)a.planes * npad * 128;
+    const uint32_t stage = NA * TC_ABYTES + bbytes;
+    // TMEM: two segment buffers and (when a tile has several segments) the
+    // running float32 total of the tile
+    const uint32_t acc_cols = NA * npad;
+    const int nseg = (nkb + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+    uint32_t ncols = 32;
+    while (ncols < (nseg > 1 ? 3 : 2) * acc_cols) ncols <<= 1;
+
+    if (warp == 0) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
+                     "r"(ncols));
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;");
+    }
+    if (threadIdx.x == 32) {
+        for (int i = 0; i < nst; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&accf[i], 1);
+            mbar_init(&acce[i], 4);
+        }
+        mbar_init(&fin, 1);
+        s_abort = 0;
+        mbar_fence_init();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = s_tmem;
+    pdl_trigger();
+    pdl_wait();   // the activation planes and the residual come from earlier kernels
+
+    if (warp == 0) {
+        if (lane == 0) {
+            long long g = 0;
+            bool stop = false;
+            for (int it = 0; it < nloc && !stop; ++it) {
+                const int y = (i0 + it) * 128;
+                for (int kb = 0; kb < nkb; ++kb, ++g) {
+                    const int s = (int)(g % nst);
+                    if (g >= nst && !mbar_wait(&empty[s], (uint32_t)((g / nst) - 1) & 1)) {
+                        set_status(a.status, OSPREY_ERR_TIMEOUT);
+                        atomicExch(&s_abort, 1);
+                        stop = true;
+                        break;
+                    }
+                    if (*(volatile int *)&s_abort) { stop = true; break; }
+                    uint8_t *st = sm + (size_t)s * stage;
+                    mbar_arrive_expect_tx(&full[s], stage);
+                    tma_2d(st, &wa, kb * 64, y, &full[s]);
+                    if (PAIR) tma_2d(st + TC_ABYTES, &wb, kb * 64, y, &full[s]);
+                    for (int p = 0; p < a.planes; ++p)
+                        tma_2d(st + NA * TC_ABYTES + (size_t)p * npad * 128, &xm, kb * 64, p * npad, &full[s]);
+                }
+            }
+            if (stop)   // let the copies this thread issued land before the CTA can exit
+                for (long long q = g - nst > 0 ? g - nst : 0; q < g; ++q)
+                    mbar_wait(&full[q % nst], (uint32_t)(q / nst) & 1, 200000000LL);
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // one accumulation unit = one segment of one tile, into buffer u & 1
+            const uint32_t idesc = tc_idesc(128, npad);
+            long long g = 0, u = 0;
+            bool stop = false;
+            for (int it = 0; it < nloc && !stop; ++it) {
+                for (int sg = 0; sg < nseg && !stop; ++sg, ++u) {
+                    const int buf = (int)(u & 1);
+                    if (u >= 2 && !mbar_wait(&acce[buf], (uint32_t)((u >> 1) - 1) & 1)) {
+                        set_status(a.status, OSPREY_ERR_TIMEOUT);
+                        atomicExch(&s_abort, 1);
+                        stop = true;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d0 = tmem + (uint32_t)buf * acc_cols, d1 = d0 + (uint32_t)npad;
+                    const int kb0 = sg * OSP_TC_SEGKB, kb1 = min(nkb, kb0 + OSP_TC_SEGKB);
+                    for (int kb = kb0; kb < kb1; ++kb, ++g) {
+                        const int s = (int)(g % nst);
+                        if (!mbar_wait(&full[s], (uint32_t)(g / nst) & 1) || *(volatile int *)&s_abort) {
+                            set_status(a.status, OSPREY_ERR_TIMEOUT);
+                            atomicExch(&s_abort, 1);
+                            stop = true;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t st = smem_u32(sm + (size_t)s * stage);
+                        const uint64_t da = tc_desc(st), da2 = tc_desc(st + TC_ABYTES);
+#pragma unroll
+                        for (int kk = 0; kk < 4; ++kk) {
+                            for (int p = 0; p < a.planes; ++p) {
+                                const uint64_t db = tc_desc(st + NA * TC_ABYTES + (uint32_t)p * npad * 128);
+                                const uint32_t acc = (kb != kb0) || kk || p;
+                                tc_mma(d0, da + 2 * kk, db + 2 * kk, idesc, acc);
+                                if (PAIR) tc_mma(d1, da2 + 2 * kk, db + 2 * kk, idesc, acc);
+                            }
+                        }
+                        tc_commit(&empty[s]);
+                    }
+                    if (!stop) tc_commit(&accf[buf]);
+                }
+            }
+            tc_commit(&fin);
+            mbar_wait(&fin, 0, 400000000LL);   // every MMA of this CTA has completed
+        }
+    } else {
+        // epilogue: TMEM lanes (warp % 4) * 32 .. + 31 hold output features m.
+        // Each segment's partial is added into the tile's running total in float32;
+        // the last segment's sum goes through the epilogue.
+        const int lg = (warp & 3) * 32;
+        const int m = lg + lane;
+        long long u = 0;
+        bool stop = false;
+        for (int it = 0; it < nloc && !stop; ++it) {
+            const int col = (i0 + it) * 128 + m;
+            const bool colok = col < a.nout;
+            const uint32_t tt = tmem + ((uint32_t)lg << 16) + 2u * acc_cols;
+            for (int sg = 0; sg < nseg; ++sg, ++u) {
+                const int buf = (int)(u & 1);
+                if (!mbar_wait(&accf[buf], (uint32_t)(u >> 1) & 1) || *(volatile int *)&s_abort) {
+                    set_status(a.status, OSPREY_ERR_TIMEOUT);
+                    atomicExch(&s_abort, 1);
+                    stop = true;
+                    break;
+                }
+                tc_fence_after();
+                const bool last = sg == nseg - 1;
+                const uint32_t t0 = tmem + ((uint32_t)lg << 16) + (uint32_t)buf * acc_cols;
+                for (int c0 = 0; c0 < npad; c0 += 16) {
+                    float v[16], w[16], tv[16], tw[16];
+                    tc_ld16(t0 + (uint32_t)c0, v);
+                    if (PAIR) tc_ld16(t0 + (uint32_t)npad + (uint32_t)c0, w);
+                    if (sg > 0) {
+                        tc_ld16(tt + (uint32_t)c0, tv);
+                        if (PAIR) tc_ld16(tt + (uint32_t)npad + (uint32_t)c0, tw);
+                    }
+                    tc_ld_wait();
+                    if (sg > 0) {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            v[j] += tv[j];
+                            if (PAIR) w[j] += tw[j];
+                        }
+                    }
+                    if (!last) {
+                        tc_st16(tt + (uint32_t)c0, v);
+                        if (PAIR) tc_st16(tt + (uint32_t)npad + (uint32_t)c0, w);
+                        continue;
+                    }
+#pragma unroll
+                    for (int j = 0; j < 16; ++j) {
+                        const int n = c0 + j;
+                        if (n >= a.R || !colok) continue;
+                        if (EPI == TC_STORE) {
+                            a.y[(size_t)n * a.ldy + col] = v[j];
+                        } else if (EPI == TC_RESID) {
+                            a.x[(size_t)n * a.ldy + col] += v[j];
+                        } else {
+                            const float g = v[j];
+                            const float h = g / (1.f + expf(-g)) * w[j];
+                            uint16_t q[TC_PLANES];
+                            tc_split(h, q);
+#pragma unroll
+                            for (int i = 0; i < TC_PLANES; ++i) a.h[((size_t)i * npad + n) * a.nout + col] = q[i];
+                        }
+                    }
+                }
+                if (!last) tc_st_wait();
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&acce[buf]);
+            }
+        }
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols));
+}
+
+// ---------------------------------------------------------------- operand planes
+__global__ void __launch_bounds__(256) planes_kernel(const PlaneArgs a) {
+    __shared__ float red[33];
+    const int r = blockIdx.x;
+    pdl_trigger();
+    pdl_wait();
+    bool act;
+    int srow;
+    if (a.last_of_seq) {
+        act = !a.valid || a.valid[r];
+        srow = act ? r * a.max_new + a.nnew[r] - 1 : 0;
+    } else {
+        const int b = r / a.rows_per_seq, j = r - b * a.rows_per_seq;
+        act = (!a.valid || a.valid[b]) && (a.rows_per_seq == 1 || j < a.nnew[b]);
+        srow = r;
+    }
+    const float *x = a.src + (size_t)srow * a.d;
+    float inv = 1.f;
+    if (a.gain) {
+        float ss = 0.f;
+        if (act)
+            for (int k = threadIdx.x; k < a.d; k += blockDim.x) ss = fmaf(x[k], x[k], ss);
+        ss = warp_sum(ss);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            float t = 0.f;
+            for (int w = 0; w < (int)(blockDim.x >> 5); ++w) t += red[w];
+            red[32] = rsqrtf(t / (float)a.d + a.eps);
+        }
+        __syncthreads();
+        inv = red[32];
+    }
+    uint16_t *p0 = a.dst + (size_t)r * a.ld + a.col0;
+    const size_t plane = (size_t)a.npad * a.ld;
+    for (int k = threadIdx.x; k < a.d; k += blockDim.x) {
+        float v = act ? x[k] : 0.f;
+        if (a.gain) v = v * inv * bf_to_f(a.gain[k]);
+        uint16_t q[TC_PLANES];
+        tc_split(v, q);
+#pragma unroll
+        for (int i = 0; i < TC_PLANES; ++i) p0[i * plane + k] = q[i];
+    }
+}
+
+// ---------------------------------------------------------------- RoPE + K/V write
+__global__ void __launch_bounds__(256) qkv_post_kernel(const QkvPostArgs a) {
+    const Dims &D = a.dim;
+    const int half = D.hd / 2;
+    const int per_row = (D.Hq + 2 * D.Hkv) * half;
+    pdl_trigger();
+    pdl_wait();
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)a.R * per_row) return;
+    const int r = (int)(idx / per_row), item = (int)(idx % per_row);
+    int b, pos;
+    if (!a.map.row(r, b, pos)) return;
+    const int h = item / half, ii = item % half;
+    const float *yr = a.y + (size_t)r * (D.Hq + 2 * D.Hkv) * D.hd + (size_t)h * D.hd;
+    float x1 = yr[ii], x2 = yr[ii + half];
+    if (h < D.Hq + D.Hkv) {
+        float c, sn;
+        rope_cs2(a.inv_freq[ii], pos, c, sn);
+        const float y1 = x1 * c - x2 * sn, y2 = x2 * c + x1 * sn;
+        x1 = y1;
+        x2 = y2;
+    }
+    if (h < D.Hq) {
+        float *q = a.q + (size_t)r * D.Hq * D.hd + (size_t)h * D.hd;
+        q[ii] = x1;
+        q[ii + half] = x2;
+    } else {
+        const bool is_k = h < D.Hq + D.Hkv;
+        const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
+        const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
+        uint16_t *dst = (is_k ? a.k_pages : a.v_pages) + (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * D.hd;
+        dst[ii] = f_to_bf(x1);
+        dst[ii + half] = f_to_bf(x2);
+    }
+}
+
+// ---------------------------------------------------------------- row sampler
+constexpr int RS_THREADS = 256;
+constexpr int RS_PER = 16;                      // logits per thread in a chunk
+constexpr int RS_CHUNK = RS_THREADS * RS_PER;   // 4096 ids
+
+int row_sample_chunks(int V) { return (V + RS_CHUNK - 1) / RS_CHUNK; }
+
+// Block-wide ordered pick over one weight per thread: the smallest index i
+// with t < C_i (inclusive cumulative weight, positive weights only); if
+// rounding leaves t past the total, the last index with weight.  Returns the
+// index and the cumulative weight before it in *before.
+__device__ int rs_pick(float w, int idx, float t, float *before, float *sh, int *si) {
+    float tot;
+    const float ex = block_excl_scan(w, sh, &tot);
+    if (threadIdx.x == 0) { si[0] = 0x7fffffff; si[1] = -1; }
+    __syncthreads();
+    if (w > 0.f && t < ex + w) atomicMin(&si[0], idx);
+    if (w > 0.f) atomicMax(&si[1], idx);
+    __syncthreads();
+    const int pick = si[0] != 0x7fffffff ? si[0] : (si[1] >= 0 ? si[1] : 0);
+    if (idx == pick) sh[32] = ex;
+    __syncthreads();
+    *before = sh[32];
+    __syncthreads();
+    return pick;
+}
+
+__global__ void __launch_bounds__(RS_THREADS) row_sample_kernel(const RowSampleArgs a) {
+    __shared__ MS sm_ms[RS_THREADS / 32];
+    __shared__ AM sm_am[RS_THREADS / 32];
+    __shared__ float sh[34];
+    __shared__ int si[2];
+    __shared__ int s_tok;
+    __shared__ float s_e;
+    const Dims &D = a.dim;
+    const int c = blockIdx.x, b = blockIdx.y, t = threadIdx.x;
+    pdl_trigger();
+    pdl_wait();
+    if (!a.valid[b]) return;   // every block of the row leaves here
+    const bool greedy = a.temperature == 0.f;
+    const float invT = greedy ? 1.f : 1.f / a.temperature;
+    const float *z = a.z + (size_t)b * a.ldz;
+    // chunk statistics of y = z / T: (max, sum exp(y - max)), argmax of z (lowest id)
+    const int base = c * RS_CHUNK + t * RS_PER;
+    float y[RS_PER];
+    float m = -INFINITY;
+    AM am{-INFINITY, 0x7fffffff};
+#pragma unroll
+    for (int k = 0; k < RS_PER; ++k) {
+        const int n = base + k;
+        const float zv = n < D.V ? __ldcg(z + n) : -INFINITY;
+        y[k] = zv * invT;
+        m = fmaxf(m, y[k]);
+        if (zv > am.v) am = AM{zv, n};
+    }
+    float s = 0.f;
+#pragma unroll
+    for (int k = 0; k < RS_PER; ++k) s += y[k] == -INFINITY ? 0.f : __expf(y[k] - m);
+    const MS ms = block_ms(MS{m, m == -INFINITY ? 0.f : s}, sm_ms);
+    const AM bam = block_am(am, sm_am);
+    if (t == 0) a.part[(size_t)b * a.nch + c] = make_float4(ms.m, ms.s, bam.v, __int_as_float(bam.i));
+    if (!arrive_last(a.ticket + b, a.nch)) return;
+
+    // last block of row b: level 1 over the chunk partials (one per thread)
+    const float4 pv = t < a.nch ? __ldcg(a.part + (size_t)b * a.nch + t) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+    const float M = block_ms(MS{pv.x, pv.y}, sm_ms).m;
+    const float cw = t < a.nch && pv.x != -INFINITY ? pv.y * __expf(pv.x - M) : 0.f;
+    int token;
+    float S, qx = 1.f;
+    if (greedy) {
+        token = block_am(AM{t < a.nch ? pv.z : -INFINITY, t < a.nch ? __float_as_int(pv.w) : 0x7fffffff}, sm_am).i;
+        S = block_ms(MS{0.f, cw}, sm_ms).s;
+    } else {
+        const float u = a.u_draft[(size_t)b * a.K + a.step];
+        float tot;
+        block_excl_scan(cw, sh, &tot);
+        S = tot;
+        const float target = u * S;
+        float before1;
+        const int ck = rs_pick(cw, t, target, &before1, sh, si);
+        // level 2: the chosen chunk, RS_PER consecutive ids per thread
+        const int b2 = ck * RS_CHUNK + t * RS_PER;
+        float e[RS_PER], mine = 0.f;
+#pragma unroll
+        for (int k = 0; k < RS_PER; ++k) {
+            const int n = b2 + k;
+            e[k] = n < D.V ? __expf(__ldcg(z + n) * invT - M) : 0.f;
+            mine += e[k];
+        }
+        float tot2;
+        const float ex = block_excl_scan(mine, sh, &tot2);
+        float cum = before1 + ex;
+        int found = 0x7fffffff, lastp = -1;
+        float efound = 0.f, elast = 0.f;
+#pragma unroll
+        for (int k = 0; k < RS_PER; ++k) {
+            cum += e[k];
+            if (e[k] > 0.f) { lastp = b2 + k; elast = e[k]; }
+            if (found == 0x7fffffff && e[k] > 0.f && target < cum) { found = b2 + k; efound = e[k]; }
+        }
+        if (t == 0) { si[0] = 0x7fffffff; si[1] = -1; }
+        __syncthreads();
+        if (found != 0x7fffffff) atomicMin(&si[0], found);
+        if (lastp >= 0) atomicMax(&si[1], lastp);
+        __syncthreads();
+        const int pick = si[0] != 0x7fffffff ? si[0] : (si[1] >= 0 ? si[1] : ck * RS_CHUNK);
+        if (found == pick) { s_tok = pick; s_e = efound; }
+        else if (si[0] == 0x7fffffff && lastp == pick) { s_tok = pick; s_e = elast; }
+        __syncthreads();
+        token = s_tok;
+        qx = s_e / S;
+    }
+    if (t == 0) {
+        a.tokens[(size_t)b * a.K + a.step] = token;
+        if (a.qx) a.qx[(size_t)b * a.K + a.step] = qx;
+        if (a.stats) {
+            a.stats[((size_t)b * a.K + a.step) * 2 + 0] = M;
+            a.stats[((size_t)b * a.K + a.step) * 2 + 1] = logf(S);
+        }
+    }
+    if (a.step + 1 < a.K) {
+        // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[token]
+        const int src = a.src_is_ext ? b * a.max_new + a.nnew[b] - 1 : b;
+        const float *xl = a.x_in + (size_t)src * D.d;
+        const uint16_t *er = a.embed + (size_t)token * D.d;
+        for (int k = t; k < D.d; k += RS_THREADS) {
+            const float xv = xl[k];
+            const float ev = bf_to_f(er[k]);
+            a.s_chain[(size_t)b * D.d + k] = xv;
+            a.x_chain[(size_t)b * D.d + k] = ev;
+        }
+    }
+}
+
+// ---------------------------------------------------------------- embedding rows
+__global__ void __launch_bounds__(256) embed_rows_kernel(const EmbedArgs a) {
+    const int r = blockIdx.x, b = r / a.max_new, j = r - b * a.max_new;
+    pdl_trigger();
+    pdl_wait();
+    if (!a.valid[b] || j >= a.nnew[b]) return;
+    const uint16_t *e = a.embed + (size_t)a.tokens[r] * a.d;   // ids checked by the prepare kernel
+    for (int k = threadIdx.x; k < a.d; k += blockDim.x) a.x[(size_t)r * a.d + k] = bf_to_f(e[k]);
+}
+
+// ---------------------------------------------------------------- host side
+static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
+static int g_encode_state = 0;   // 0 unknown, 1 ok, -1 unavailable
+
+bool tc_available() {
+    if (g_encode_state == 0) {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        const cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
+        g_encode = e == cudaSuccess && q == cudaDriverEntryPointSuccess ? (PFN_cuTensorMapEncodeTiled_v12000)fn : nullptr;
+        if (e != cudaSuccess) cudaGetLastError();
+        int dev = 0, major = 0;
+        if (cudaGetDevice(&dev) != cudaSuccess || cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) {
+            cudaGetLastError();
+            major = 0;
+        }
+        g_encode_state = g_encode && major >= 10 ? 1 : -1;
+    }
+    return g_encode_state == 1;
+}
+
+static bool encode2d(CUtensorMap *m, const void *base, uint64_t inner, uint64_t rows, uint32_t box_rows) {
+    if (!tc_available()) return false;
+    if (((uintptr_t)base & 15) || (inner * 2) % 16) return false;
+    cuuint64_t dims[2] = {(cuuint64_t)inner, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)inner * 2};
+    cuuint32_t box[2] = {64, box_rows};
+    cuuint32_t es[2] = {1, 1};
+    return g_encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, es,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                    CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool tc_encode_weight(CUtensorMap *m, const void *w, int rows, int K) { return encode2d(m, w, K, rows, 128); }
+bool tc_encode_rows(CUtensorMap *m, const void *x, int rows, int npad, int K) { return encode2d(m, x, K, rows, npad); }
+bool tc_encode_operand(CUtensorMap *m, const void *x, int planes, int npad, int K) {
+    return encode2d(m, x, K, (uint64_t)planes * npad, npad);
+}
+
+static int tc_stages(int npad, int planes, bool pair) {
+    const size_t stage = (size_t)(pair ? 2 : 1) * TC_ABYTES + (size_t)planes * npad * 128;
+    int n = (int)((TC_SMEM_CAP - 1024) / stage);
+    return n > TC_MAXST ? TC_MAXST : n;
+}
+size_t tc_smem_bytes(int npad, int planes, bool pair) {
+    const size_t stage = (size_t)(pair ? 2 : 1) * TC_ABYTES + (size_t)planes * npad * 128;
+    return (size_t)tc_stages(npad, planes, pair) * stage + 1024;
+}
+
+cudaError_t tc_set_attributes() {
+    const int bytes = (int)TC_SMEM_CAP;
+    cudaError_t e = cudaFuncSetAttribute(tc_kernel<TC_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    return e;
+}
+
+template <typename... P, typename... A>
+static cudaError_t pdl_launch(void (*k)(P...), dim3 grid, dim3 block, size_t smem, cudaStream_t s, const A &...args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, k, args...);
+    count_launch();
+    return e;
+}
+
+cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap *wb, const CUtensorMap &xm, int sms,
+                      cudaStream_t s) {
+    const bool pair = a.epi == TC_SWIGLU;
+    if (a.npad % 16 || a.npad < 16 || a.npad > (pair ? 128 : TC_MAX_ROWS) || a.K % 64 || a.R > a.npad)
+        return cudaErrorInvalidValue;
+    const int nst = tc_stages(a.npad, a.planes, pair);
+    if (nst < 2) return cudaErrorInvalidValue;
+    const int nseg = (a.K / 64 + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+    if ((nseg > 1 ? 3 : 2) * (pair ? 2 : 1) * a.npad > 512) return cudaErrorInvalidValue;   // TMEM columns
+    const int items = (a.nout + 127) / 128;
+    const int grid = items < sms ? items : sms;
+    const size_t smem = tc_smem_bytes(a.npad, a.planes, pair);
+    const CUtensorMap &b = wb ? *wb : wa;
+    switch (a.epi) {
+    case TC_STORE: return pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, b, xm, a, nst);
+    case TC_RESID: return pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, b, xm, a, nst);
+    default: return pdl_launch(tc_kernel<TC_SWIGLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, b, xm, a, nst);
+    }
+}
+
+cudaError_t launch_planes(const PlaneArgs &a, cudaStream_t s) {
+    return pdl_launch(planes_kernel, dim3(a.R), dim3(256), 0, s, a);
+}
+
+cudaError_t launch_qkv_post(const QkvPostArgs &a, cudaStream_t s) {
+    const long long n = (long long)a.R * (a.dim.Hq + 2 * a.dim.Hkv) * (a.dim.hd / 2);
+    return pdl_launch(qkv_post_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, a);
+}
+
+cudaError_t launch_embed_rows(const EmbedArgs &a, cudaStream_t s) {
+    return pdl_launch(embed_rows_kernel, dim3(a.R), dim3(256), 0, s, a);
+}
+
+cudaError_t launch_row_sample(const RowSampleArgs &a, cudaStream_t s) {
+    if (a.nch > RS_THREADS) return cudaErrorInvalidValue;
+    return pdl_launch(row_sample_kernel, dim3(a.nch, a.B), dim3(RS_THREADS), 0, s, a);
+}
+
+}  // namespace osp

@@ -1,0 +1,121 @@
+// Batched-row draft step on the 5th-generation tensor cores (tcgen05): the
+// projections of Sec. 3.3 (Eq. 1-3, the MLP and the LM head) as streamed
+// swap-AB GEMMs, Y[R x Nout] = X[R x K] . W[Nout x K]^T, for 3..80 rows.
+//
+// Weights are the M = 128 operand, streamed tile by tile with 2-D TMA (128-byte
+// swizzle); the R activation rows are the N operand (padded to a multiple of
+// 16).  Activations are float32 between kernels; for the tensor cores each is
+// split into three bf16 planes, q0 = bf16(x), q1 = bf16(x - q0), q2 =
+// bf16(x - q0 - q1), and every k-step issues one MMA per plane into the same
+// float32 accumulator, so the product keeps the 24 mantissa bits of x (bf16
+// inputs such as the target features use a single plane).  Two planes (16
+// bits) were not enough: attention over thousands of cached keys turns a 1e-5
+// relative error in q into logit errors two orders above the float32 path's.  The reduction is accumulated in segments of
+// 512 (a fresh TMEM accumulator each) whose float32 sum the epilogue keeps, so
+// no accumulation chain in the tensor core is longer than 32 MMA steps per
+// plane (a long chain loses precision against a float32 tree sum).
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "draft.cuh"
+
+namespace osp {
+
+enum TcEpi { TC_STORE = 0, TC_RESID = 1, TC_SWIGLU = 2 };
+
+constexpr int TC_MAX_ROWS = 80;    // activation rows per GEMM: three accumulators of the gate/up pair fit TMEM
+constexpr int TC_PLANES = 3;       // bf16 planes of a float32 operand
+
+struct TcArgs {
+    int epi;           // TcEpi
+    int R, npad;       // rows, rows padded to a multiple of 16
+    int K;             // reduction length (multiple of 64)
+    int nout;          // output features (tiles of 128, the last one may be partial)
+    int planes;        // 1 (bf16 input) or TC_PLANES (split float32 input)
+    float *y;          // TC_STORE: [R][ldy] float32 (columns col0 + m)
+    int ldy;
+    float *x;          // TC_RESID: [R][ldy] float32, +=
+    uint16_t *h;       // TC_SWIGLU: [TC_PLANES][npad][nout] bf16 planes of silu(gate) * up
+    int32_t *status;
+};
+
+// Host side.  Tensor maps: weights [rows][K] bf16 with a 64 x 128 box, operand
+// planes [planes * npad][K] bf16 with a 64 x npad box, both 128-byte swizzled.
+bool tc_available();   // the driver exposes tensor-map encoding and the device is sm_100+
+bool tc_encode_weight(CUtensorMap *m, const void *w, int rows, int K);
+bool tc_encode_operand(CUtensorMap *m, const void *x, int planes, int npad, int K);
+// a single bf16 plane of `rows` rows read in place (rows past `rows` read as zero)
+bool tc_encode_rows(CUtensorMap *m, const void *x, int rows, int npad, int K);
+size_t tc_smem_bytes(int npad, int planes, bool pair);
+cudaError_t tc_set_attributes();
+cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap *wb, const CUtensorMap &xm, int sms,
+                      cudaStream_t s);
+
+// Operand preparation: rows of float32 (optionally RMS-normalised with a bf16
+// gain) written as bf16 planes [TC_PLANES][npad][ld] starting at column col0.
+struct PlaneArgs {
+    const float *src;          // row r at src + src_row(r) * d
+    const uint16_t *gain;      // RMSNorm gain, or null for a plain copy
+    float eps;
+    int d, R, npad, ld, col0;
+    uint16_t *dst;
+    // row selection: r itself, or (LM at the extend step) b*max_new + n_new[b] - 1
+    const int *nnew;
+    int max_new, last_of_seq;
+    const int *valid;          // rows of invalid sequences are written as zeros (may be null)
+    int rows_per_seq;
+};
+cudaError_t launch_planes(const PlaneArgs &a, cudaStream_t s);
+
+// RoPE and the paged K/V write from the QKV GEMM output y [R][(Hq+2Hkv)hd].
+struct QkvPostArgs {
+    Dims dim;
+    RowMap map;
+    int R;
+    const float *y;
+    float *q;
+    uint16_t *k_pages, *v_pages;
+    const int32_t *page_table;
+    int max_pages;
+    double inv_freq[64];       // rotary frequencies theta^(-2i/hd)
+};
+cudaError_t launch_qkv_post(const QkvPostArgs &a, cudaStream_t s);
+
+// Sampling over B logits rows z [B][V] (Sec. 3.1 draft distribution q =
+// softmax(z / T)): inverse CDF at u_draft[b][step] over ascending ids, or the
+// argmax (T = 0); writes the token, q(token), (max, log-sum-exp) and, when a
+// next chain step follows, the next chain row (context slot = x_L, residual =
+// E[token]).
+struct RowSampleArgs {
+    Dims dim;
+    int B, K, step, max_new, src_is_ext;
+    const int *valid, *nnew;
+    const float *z;            // row b at z + b * ldz
+    long long ldz;
+    float temperature;
+    const float *u_draft;
+    int32_t *tokens;
+    float *qx, *stats;
+    const float *x_in;         // residual rows of the step (x_ext or x_chain)
+    float *x_chain, *s_chain;
+    const uint16_t *embed;
+    float4 *part;              // [B][nch] chunk partials
+    int *ticket;               // [B]
+    int nch;
+};
+int row_sample_chunks(int V);
+// x[r] = E[tokens[r]] (float32) for the active extend rows r = b*max_new + j, j < n_new[b].
+struct EmbedArgs {
+    int d, R, max_new;
+    const int *valid, *nnew;
+    const int32_t *tokens;
+    const uint16_t *embed;
+    float *x;
+};
+cudaError_t launch_embed_rows(const EmbedArgs &a, cudaStream_t s);
+cudaError_t launch_row_sample(const RowSampleArgs &a, cudaStream_t s);
+
+}  // namespace osp

@@ -63,14 +63,22 @@ def run_case(shape, ctx, K, T, seed, n_new=None, max_new=1, zero=False, peaked=F
 
 
 def oracle_for(case):
-    """Oracle on the sampled sequences, following the GPU's chain."""
+    """Oracle on the sampled sequences, following the GPU's chain: its tokens,
+    and the bf16 K/V rows it cached at this call's positions (each step is then
+    checked from the same cache state; the rows themselves are checked against
+    the oracle's own in check_case)."""
     idx = case["seqs"]
-    ctx, kv, di = case["ctx"], case["kv"], case["di"]
+    ctx, kv, di, g = case["ctx"], case["kv"], case["di"], case["g"]
     offs = np.concatenate([[0], np.cumsum(ctx)])
     rows = np.concatenate([np.arange(offs[b], offs[b + 1]) for b in idx]).astype(np.int64)
+    forced_kv = []
+    for b in idx:
+        pos = np.arange(ctx[b], ctx[b] + int(di["n_new"][b]) + case["K"] - 1)
+        forced_kv.append((gather_positions(g["k_pages"], kv["page_table"][b], pos),
+                          gather_positions(g["v_pages"], kv["page_table"][b], pos)))
     return od.draft_step(case["w"], case["shape"], kv["k_rows"][:, rows], kv["v_rows"][:, rows], ctx[idx],
                          di["tokens"][idx], di["feats"][idx], di["n_new"][idx], case["K"], case["T"],
-                         di["u_draft"][idx], forced_tokens=case["g"]["draft_tokens"][idx])
+                         di["u_draft"][idx], forced_tokens=g["draft_tokens"][idx], forced_kv=forced_kv)
 
 
 def check_case(case, o=None, min_checked_frac=0.5):
@@ -236,4 +244,13 @@ def test_attention_split_partials_in_global_memory(which, monkeypatch):
     else:
         shape = replace(TINY, head_dim=128, n_q_heads=8, n_kv_heads=2, d_model=512, vocab=5000)
         case = run_case(shape, [100, 1000, 17], 5, 0.7, 41, peaked=True)
+    check_case(case)
+
+
+def test_batched_rows_on_cuda_cores(monkeypatch):
+    """Batched rows on the CUDA-core GEMV (OSPREY_TC=0), the path used where the
+    tensor-core one cannot run, against the oracle."""
+    monkeypatch.setenv("OSPREY_TC", "0")
+    shape = replace(TINY, n_layers=2, n_q_heads=8, n_kv_heads=2)
+    case = run_case(shape, [5, 0, 31, 64], 3, 0.0, 31, n_new=[3, 1, 2, 3], max_new=3)
     check_case(case)

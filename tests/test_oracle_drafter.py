@@ -203,6 +203,25 @@ def test_forced_chain_matches_free_chain():
     assert np.abs(alt["logits"][0, 1] - free["logits"][0, 1]).max() > 1e-4
 
 
+def test_forced_cache_rows_match_free_chain():
+    """Forcing the cache rows a run wrote reproduces that run exactly; forcing a
+    changed row changes the later steps but not the rows this run computes at
+    that position."""
+    shape = SMALL
+    w, ctx, kv, di = _inputs(shape, 81)
+    free = _run(shape, w, ctx, kv, di, T=1.0)
+    own = [(k, v) for k, v in zip(free["new_k"], free["new_v"])]
+    forced = _run(shape, w, ctx, kv, di, T=1.0, forced_tokens=free["tokens"], forced_kv=own)
+    np.testing.assert_array_equal(free["logits"], forced["logits"])
+    np.testing.assert_array_equal(np.asarray(free["new_k"]), np.asarray(forced["new_k"]))
+    alt_k = [k.copy() for k, _ in own]
+    alt_k[0][0, 0] += 0.5                       # sequence 0, layer 0, first row written
+    alt = _run(shape, w, ctx, kv, di, T=1.0, forced_tokens=free["tokens"],
+               forced_kv=[(alt_k[b], own[b][1]) for b in range(len(own))])
+    np.testing.assert_array_equal(np.asarray(alt["new_k"])[0][0, 0], np.asarray(free["new_k"])[0][0, 0])
+    assert np.abs(alt["logits"][0] - free["logits"][0]).max() > 1e-6
+
+
 def test_sampling_stats_and_peaked_head():
     """q(token) and (M, log S) describe softmax(z/T); the peaked LM head makes the
     draft distribution concentrated (the sampled-draft parity case)."""
