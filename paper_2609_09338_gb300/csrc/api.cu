@@ -219,6 +219,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_xo = take(tcw ? 2ull * TC_PLANES * np * D.Hq * D.hd : 0), o_xg = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     size_t o_rp = take(tcw ? 16ull * B * row_sample_chunks(D.V) : 0), o_rt = take(tcw ? 4ull * B : 0);
+    size_t o_tg = take(tcw ? 4ull * np * D.F : 0);
     if (ws && base) {
         char *p = (char *)base;
         ws->seq_valid = (int *)(p + o_valid);
@@ -245,6 +246,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->tc_xl = (uint16_t *)(p + o_xl);
         ws->rs_part = (float4 *)(p + o_rp);
         ws->rs_ticket = (int *)(p + o_rt);
+        ws->tc_g = (float *)(p + o_tg);
         ws->n_splits_max = ns;
         ws->lm_warps_max = lm_warps;
     }
@@ -355,7 +357,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
     // tensor-core path for 3..TC_MAX_ROWS activation rows
     auto tc_rows = [&](int rows) { return ctx->tc && rows >= 3 && rows <= TC_MAX_ROWS; };
     auto npad_of = [](int rows) { return (rows + 15) / 16 * 16; };
-    auto tc_gemm = [&](int epi, int rows, int K_, int nout, int planes, const CUtensorMap &wa, const CUtensorMap *wb,
+    auto tc_gemm = [&](int epi, int rows, int K_, int nout, int planes, const CUtensorMap &wa,
                        const void *xbuf, bool in_place_rows, float *y, int ldy, uint16_t *h,
                        const char *what) -> int {
         const int np = npad_of(rows);
@@ -374,7 +376,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         ta.ldy = ldy;
         ta.h = h;
         ta.status = dev_status;
-        const cudaError_t e2 = launch_tc(ta, wa, wb, xm, ctx->sms, s);
+        const cudaError_t e2 = launch_tc(ta, wa, xm, ctx->sms, s);
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
     };
     auto planes = [&](const float *src, const uint16_t *gain, int d_, int rows, int ld, int col0, uint16_t *dst,
@@ -400,7 +402,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
     if (tc_rows(B * max_new)) {
         EmbedArgs ea{D.d, B * max_new, max_new, ws.seq_valid, ws.seq_nnew, tokens, (const uint16_t *)W.embed, ws.x_ext};
         if ((e = launch_embed_rows(ea, s)) != cudaSuccess) return cuda_fail(e, "embedding launch");
-        const int rc = tc_gemm(TC_STORE, B * max_new, D.feat, D.d, 1, ctx->tm_c, nullptr, feats, true, ws.s_ext, D.d,
+        const int rc = tc_gemm(TC_STORE, B * max_new, D.feat, D.d, 1, ctx->tm_c, feats, true, ws.s_ext, D.d,
                                nullptr, "feature projection launch");
         if (rc != OSPREY_OK) return rc;
     } else if ((e = launch_gemv(G_FEAT, g, gemv_rg(G_FEAT, D, g.R), ctx->sms, s)) != cudaSuccess) {
@@ -470,7 +472,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             if ((rc = planes(sb, nullptr, D.d, R, 2 * D.d, 0, ws.tc_xq, rows_per_seq, false, "qkv operand")) != OSPREY_OK ||
                 (rc = planes(x, (const uint16_t *)W.attn_norm[l], D.d, R, 2 * D.d, D.d, ws.tc_xq, rows_per_seq, false,
                              "qkv operand")) != OSPREY_OK ||
-                (rc = tc_gemm(TC_STORE, R, 2 * D.d, nqkv, TC_PLANES, ctx->tm_qkv[l], nullptr, ws.tc_xq, false, ws.tc_yq, nqkv,
+                (rc = tc_gemm(TC_STORE, R, 2 * D.d, nqkv, TC_PLANES, ctx->tm_qkv[l], ws.tc_xq, false, ws.tc_yq, nqkv,
                               nullptr, "qkv launch")) != OSPREY_OK)
                 return rc;
             QkvPostArgs qp{};
@@ -505,13 +507,15 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             const int ha = D.Hq * D.hd;
             if ((rc = planes(ws.attn_out, nullptr, ha, R, ha, 0, ws.tc_xo, rows_per_seq, false, "o-proj operand")) !=
                     OSPREY_OK ||
-                (rc = tc_gemm(TC_RESID, R, ha, D.d, TC_PLANES, ctx->tm_o[l], nullptr, ws.tc_xo, false, x, D.d, nullptr,
+                (rc = tc_gemm(TC_RESID, R, ha, D.d, TC_PLANES, ctx->tm_o[l], ws.tc_xo, false, x, D.d, nullptr,
                               "o-proj launch")) != OSPREY_OK ||
                 (rc = planes(x, (const uint16_t *)W.ffn_norm[l], D.d, R, D.d, 0, ws.tc_xg, rows_per_seq, false,
                              "gate/up operand")) != OSPREY_OK ||
-                (rc = tc_gemm(TC_SWIGLU, R, D.d, D.F, TC_PLANES, ctx->tm_gate[l], &ctx->tm_up[l], ws.tc_xg, false, nullptr, 0,
-                              ws.tc_xh, "gate/up launch")) != OSPREY_OK ||
-                (rc = tc_gemm(TC_RESID, R, D.F, D.d, TC_PLANES, ctx->tm_down[l], nullptr, ws.tc_xh, false, x, D.d, nullptr,
+                (rc = tc_gemm(TC_STORE, R, D.d, D.F, TC_PLANES, ctx->tm_gate[l], ws.tc_xg, false, ws.tc_g, D.F, nullptr,
+                              "gate launch")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_GLU, R, D.d, D.F, TC_PLANES, ctx->tm_up[l], ws.tc_xg, false, ws.tc_g, D.F, ws.tc_xh,
+                              "up launch")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_RESID, R, D.F, D.d, TC_PLANES, ctx->tm_down[l], ws.tc_xh, false, x, D.d, nullptr,
                               "down launch")) != OSPREY_OK)
                 return rc;
         }
@@ -585,7 +589,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             const long long ldz = draft_logits ? (long long)K * D.V : D.V;
             if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand")) !=
                     OSPREY_OK ||
-                (rc = tc_gemm(TC_STORE, B, D.d, D.V, TC_PLANES, ctx->tm_lm, nullptr, ws.tc_xl, false, zb, (int)ldz, nullptr,
+                (rc = tc_gemm(TC_STORE, B, D.d, D.V, TC_PLANES, ctx->tm_lm, ws.tc_xl, false, zb, (int)ldz, nullptr,
                               "lm head launch")) != OSPREY_OK)
                 return rc;
             RowSampleArgs rs{};

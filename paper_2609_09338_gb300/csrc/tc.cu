@@ -2,9 +2,9 @@
 // the projections of Sec. 3.3 (Eq. 1-3, MLP, LM head), operand preparation,
 // RoPE + paged K/V write, and per-row sampling of the draft token (Sec. 3.1).
 //
-// tc_kernel: persistent, one CTA per SM, 6 warps.
-//   warp 0     issues 2-D TMA copies of one 128-row weight tile (two for the
-//              gate/up pair) and the activation planes per 64-wide k-block into
+// tc_kernel: persistent, two CTAs per SM, 6 warps.
+//   warp 0     issues 2-D TMA copies of one 128-row weight tile and the
+//              activation planes per 64-wide k-block into
 //              an nst-slot shared-memory ring (128-byte swizzle);
 //   warp 1     issues tcgen05.mma (M 128, N npad, K 16, bf16 in, float32
 //              accumulate in TMEM) per k-block and plane, then commits the
@@ -28,7 +28,10 @@ namespace osp {
 constexpr int TC_THREADS = 192;
 constexpr int TC_ABYTES = 128 * 128;    // weight tile: 128 rows x 64 bf16
 constexpr int TC_MAXST = 8;
-constexpr size_t TC_SMEM_CAP = 200 * 1024;
+#ifndef OSP_TC_CTAS_PER_SM
+#define OSP_TC_CTAS_PER_SM 2   // two CTAs per SM: two TMA producers and two MMA chains per SM
+#endif
+constexpr size_t TC_SMEM_CAP = (OSP_TC_CTAS_PER_SM == 1 ? 200 : 100) * 1024;
 #ifndef OSP_TC_SEGKB
 #define OSP_TC_SEGKB 8   // k-blocks (64 wide) per accumulation segment
 #endif
@@ -102,11 +105,9 @@ __device__ __forceinline__ void tc_split(float x, uint16_t (&q)[TC_PLANES]) {
 
 // ---------------------------------------------------------------- GEMM kernel
 template <int EPI>
-__global__ void __launch_bounds__(TC_THREADS, 1)
-    tc_kernel(const __grid_constant__ CUtensorMap wa, const __grid_constant__ CUtensorMap wb,
-              const __grid_constant__ CUtensorMap xm, const TcArgs a, int nst) {
-    constexpr bool PAIR = EPI == TC_SWIGLU;
-    constexpr int NA = PAIR ? 2 : 1;
+__global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
+    tc_kernel(const __grid_constant__ CUtensorMap wa, const __grid_constant__ CUtensorMap xm, const TcArgs a, int nst) {
+    constexpr int NA = 1;
     extern __shared__ uint8_t raw[];
     uint8_t *sm = (uint8_t *)(((uintptr_t)raw + 1023) & ~(uintptr_t)1023);
     __shared__ __align__(8) uint64_t full[TC_MAXST], empty[TC_MAXST], accf[2], acce[2], fin;
@@ -169,7 +170,6 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                     uint8_t *st = sm + (size_t)s * stage;
                     mbar_arrive_expect_tx(&full[s], stage);
                     tma_2d(st, &wa, kb * 64, y, &full[s]);
-                    if (PAIR) tma_2d(st + TC_ABYTES, &wb, kb * 64, y, &full[s]);
                     for (int p = 0; p < a.planes; ++p)
                         tma_2d(st + NA * TC_ABYTES + (size_t)p * npad * 128, &xm, kb * 64, p * npad, &full[s]);
                 }
@@ -194,7 +194,7 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t d0 = tmem + (uint32_t)buf * acc_cols, d1 = d0 + (uint32_t)npad;
+                    const uint32_t d0 = tmem + (uint32_t)buf * acc_cols;
                     const int kb0 = sg * OSP_TC_SEGKB, kb1 = min(nkb, kb0 + OSP_TC_SEGKB);
                     for (int kb = kb0; kb < kb1; ++kb, ++g) {
                         const int s = (int)(g % nst);
@@ -206,14 +206,13 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                         }
                         tc_fence_after();
                         const uint32_t st = smem_u32(sm + (size_t)s * stage);
-                        const uint64_t da = tc_desc(st), da2 = tc_desc(st + TC_ABYTES);
+                        const uint64_t da = tc_desc(st);
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk) {
                             for (int p = 0; p < a.planes; ++p) {
                                 const uint64_t db = tc_desc(st + NA * TC_ABYTES + (uint32_t)p * npad * 128);
                                 const uint32_t acc = (kb != kb0) || kk || p;
                                 tc_mma(d0, da + 2 * kk, db + 2 * kk, idesc, acc);
-                                if (PAIR) tc_mma(d1, da2 + 2 * kk, db + 2 * kk, idesc, acc);
                             }
                         }
                         tc_commit(&empty[s]);
@@ -248,24 +247,16 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                 const bool last = sg == nseg - 1;
                 const uint32_t t0 = tmem + ((uint32_t)lg << 16) + (uint32_t)buf * acc_cols;
                 for (int c0 = 0; c0 < npad; c0 += 16) {
-                    float v[16], w[16], tv[16], tw[16];
+                    float v[16], tv[16];
                     tc_ld16(t0 + (uint32_t)c0, v);
-                    if (PAIR) tc_ld16(t0 + (uint32_t)npad + (uint32_t)c0, w);
-                    if (sg > 0) {
-                        tc_ld16(tt + (uint32_t)c0, tv);
-                        if (PAIR) tc_ld16(tt + (uint32_t)npad + (uint32_t)c0, tw);
-                    }
+                    if (sg > 0) tc_ld16(tt + (uint32_t)c0, tv);
                     tc_ld_wait();
                     if (sg > 0) {
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            v[j] += tv[j];
-                            if (PAIR) w[j] += tw[j];
-                        }
+                        for (int j = 0; j < 16; ++j) v[j] += tv[j];
                     }
                     if (!last) {
                         tc_st16(tt + (uint32_t)c0, v);
-                        if (PAIR) tc_st16(tt + (uint32_t)npad + (uint32_t)c0, w);
                         continue;
                     }
 #pragma unroll
@@ -276,9 +267,9 @@ __global__ void __launch_bounds__(TC_THREADS, 1)
                             a.y[(size_t)n * a.ldy + col] = v[j];
                         } else if (EPI == TC_RESID) {
                             a.x[(size_t)n * a.ldy + col] += v[j];
-                        } else {
-                            const float g = v[j];
-                            const float h = g / (1.f + expf(-g)) * w[j];
+                        } else {   // up projection: h = silu(gate) * up, gate from the previous pass
+                            const float g = a.y[(size_t)n * a.ldy + col];
+                            const float h = g / (1.f + expf(-g)) * v[j];
                             uint16_t q[TC_PLANES];
                             tc_split(h, q);
 #pragma unroll
@@ -577,7 +568,7 @@ cudaError_t tc_set_attributes() {
     const int bytes = (int)TC_SMEM_CAP;
     cudaError_t e = cudaFuncSetAttribute(tc_kernel<TC_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_SWIGLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_GLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     return e;
 }
 
@@ -598,23 +589,19 @@ static cudaError_t pdl_launch(void (*k)(P...), dim3 grid, dim3 block, size_t sme
     return e;
 }
 
-cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap *wb, const CUtensorMap &xm, int sms,
-                      cudaStream_t s) {
-    const bool pair = a.epi == TC_SWIGLU;
-    if (a.npad % 16 || a.npad < 16 || a.npad > (pair ? 128 : TC_MAX_ROWS) || a.K % 64 || a.R > a.npad)
-        return cudaErrorInvalidValue;
-    const int nst = tc_stages(a.npad, a.planes, pair);
+cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s) {
+    if (a.npad % 16 || a.npad < 16 || a.npad > TC_MAX_ROWS || a.K % 64 || a.R > a.npad) return cudaErrorInvalidValue;
+    const int nst = tc_stages(a.npad, a.planes, false);
     if (nst < 2) return cudaErrorInvalidValue;
     const int nseg = (a.K / 64 + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
-    if ((nseg > 1 ? 3 : 2) * (pair ? 2 : 1) * a.npad > 512) return cudaErrorInvalidValue;   // TMEM columns
+    if ((nseg > 1 ? 3 : 2) * a.npad > 512 / OSP_TC_CTAS_PER_SM) return cudaErrorInvalidValue;   // TMEM columns
     const int items = (a.nout + 127) / 128;
-    const int grid = items < sms ? items : sms;
-    const size_t smem = tc_smem_bytes(a.npad, a.planes, pair);
-    const CUtensorMap &b = wb ? *wb : wa;
+    const int grid = items < OSP_TC_CTAS_PER_SM * sms ? items : OSP_TC_CTAS_PER_SM * sms;
+    const size_t smem = tc_smem_bytes(a.npad, a.planes, false);
     switch (a.epi) {
-    case TC_STORE: return pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, b, xm, a, nst);
-    case TC_RESID: return pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, b, xm, a, nst);
-    default: return pdl_launch(tc_kernel<TC_SWIGLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, b, xm, a, nst);
+    case TC_STORE: return pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
+    case TC_RESID: return pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
+    default: return pdl_launch(tc_kernel<TC_GLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
     }
 }
 

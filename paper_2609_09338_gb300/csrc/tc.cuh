@@ -24,9 +24,9 @@
 
 namespace osp {
 
-enum TcEpi { TC_STORE = 0, TC_RESID = 1, TC_SWIGLU = 2 };
+enum TcEpi { TC_STORE = 0, TC_RESID = 1, TC_GLU = 2 };
 
-constexpr int TC_MAX_ROWS = 80;    // activation rows per GEMM: three accumulators of the gate/up pair fit TMEM
+constexpr int TC_MAX_ROWS = 80;    // activation rows per GEMM: three accumulators fit a CTA's 256 TMEM columns
 constexpr int TC_PLANES = 3;       // bf16 planes of a float32 operand
 
 struct TcArgs {
@@ -35,10 +35,10 @@ struct TcArgs {
     int K;             // reduction length (multiple of 64)
     int nout;          // output features (tiles of 128, the last one may be partial)
     int planes;        // 1 (bf16 input) or TC_PLANES (split float32 input)
-    float *y;          // TC_STORE: [R][ldy] float32 (columns col0 + m)
+    float *y;          // TC_STORE: [R][ldy] float32 output; TC_GLU: the gate values read
     int ldy;
     float *x;          // TC_RESID: [R][ldy] float32, +=
-    uint16_t *h;       // TC_SWIGLU: [TC_PLANES][npad][nout] bf16 planes of silu(gate) * up
+    uint16_t *h;       // TC_GLU: [TC_PLANES][npad][nout] bf16 planes of silu(gate) * up
     int32_t *status;
 };
 
@@ -51,8 +51,9 @@ bool tc_encode_operand(CUtensorMap *m, const void *x, int planes, int npad, int 
 bool tc_encode_rows(CUtensorMap *m, const void *x, int rows, int npad, int K);
 size_t tc_smem_bytes(int npad, int planes, bool pair);
 cudaError_t tc_set_attributes();
-cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap *wb, const CUtensorMap &xm, int sms,
-                      cudaStream_t s);
+// SwiGLU runs as two passes: the gate projection (TC_STORE into a float32
+// buffer), then the up projection whose epilogue (TC_GLU) forms silu(gate) * up.
+cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s);
 
 // Operand preparation: rows of float32 (optionally RMS-normalised with a bf16
 // gain) written as bf16 planes [TC_PLANES][npad][ld] starting at column col0.
