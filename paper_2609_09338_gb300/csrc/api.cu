@@ -417,6 +417,10 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         float *x = ext ? ws.x_ext : ws.x_chain;
         float *sb = ext ? ws.s_ext : ws.s_chain;
         const int ns = attn_splits(R, D.Hkv, max_ctx, ctx->sms);
+        // the on-chip-merge attention pays off while its clusters fit in one wave
+        // (one block per SM); beyond that the global-partials kernel keeps more
+        // loads in flight
+        const bool clu = ctx->attn_cs && (long long)R * D.Hkv * ctx->attn_cs <= ctx->sms;
         // activation rows per launch: the streamed kernels serve one or two
         const bool streamed = R <= 2;
         StreamArgs sa{};
@@ -491,7 +495,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.dim = D;
             at.map = map;
             at.R = R;
-            at.n_splits = ctx->attn_cs ? ctx->attn_cs : ns;
+            at.n_splits = clu ? ctx->attn_cs : ns;
             at.split_len = attn_split_len(max_ctx, at.n_splits);
             at.q = ws.q;
             at.k_pages = kp;
@@ -501,7 +505,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.part = ws.attn_part;
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
-            e = ctx->attn_cs ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
+            e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
             // x += W_o attn;  x += W_down (silu(W_g n) * W_u n),  n = RMSNorm(x)
             const int ha = D.Hq * D.hd;
@@ -536,7 +540,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.dim = D;
             at.map = map;
             at.R = R;
-            at.n_splits = ctx->attn_cs ? ctx->attn_cs : ns;
+            at.n_splits = clu ? ctx->attn_cs : ns;
             at.split_len = attn_split_len(max_ctx, at.n_splits);
             at.q = ws.q;
             at.k_pages = g.k_pages;
@@ -546,7 +550,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.part = ws.attn_part;
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
-            e = ctx->attn_cs ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
+            e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
             g.W = (const uint16_t *)W.W_o[l];
             g.xin = ws.attn_out;
