@@ -220,6 +220,22 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     size_t o_rp = take(tcw ? 16ull * B * row_sample_chunks(D.V) : 0), o_rt = take(tcw ? 4ull * B : 0);
     size_t o_tg = take(tcw ? 4ull * np * D.F : 0);
+    // split-K partials: the largest nsplit x rows x outputs of the call's projections
+    long long part = 0;
+    if (tcw) {
+        const long long rows = tc_rows;
+        auto need = [&](int nout, int K_) {
+            const int ns = tc_nsplit(nout, K_, ctx->sms);
+            if (ns > 1) part = std::max(part, (long long)ns * rows * nout);
+        };
+        need(D.d, D.feat);
+        need((D.Hq + 2 * D.Hkv) * D.hd, 2 * D.d);
+        need(D.d, D.Hq * D.hd);
+        need(D.F, D.d);
+        need(D.d, D.F);
+        need(D.V, D.d);
+    }
+    size_t o_tp = take(4ull * part);
     if (ws && base) {
         char *p = (char *)base;
         ws->seq_valid = (int *)(p + o_valid);
@@ -247,6 +263,8 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->rs_part = (float4 *)(p + o_rp);
         ws->rs_ticket = (int *)(p + o_rt);
         ws->tc_g = (float *)(p + o_tg);
+        ws->tc_part = (float *)(p + o_tp);
+        ws->tc_part_cap = part;
         ws->n_splits_max = ns;
         ws->lm_warps_max = lm_warps;
     }
@@ -376,6 +394,8 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         ta.ldy = ldy;
         ta.h = h;
         ta.status = dev_status;
+        ta.part = ws.tc_part;
+        ta.part_cap = ws.tc_part_cap;
         const cudaError_t e2 = launch_tc(ta, wa, xm, ctx->sms, s);
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
     };

@@ -36,6 +36,8 @@ struct DraftWs {
     uint16_t *tc_xo;                       // [P][np][Hq*hd] attention output
     uint16_t *tc_xg;                       // [P][np][d]     RMSNorm(x) for gate/up
     float *tc_g;                           // [np][F]        gate projection (float32)
+    float *tc_part;                        // split-K partials of the projections
+    long long tc_part_cap;
     uint16_t *tc_xh;                       // [P][np][F]     SwiGLU hidden (down operand)
     uint16_t *tc_xl;                       // [P][np][d]     final RMSNorm rows for the LM head
     float4 *rs_part;                       // [B][V/4096]    row-sampler chunk partials

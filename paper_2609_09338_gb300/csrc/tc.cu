@@ -114,18 +114,24 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int n_items = (a.nout + 127) / 128;
+    // work item = (output tile of 128 features, k-range); items of a CTA are contiguous
+    const int n_items = (a.nout + 127) / 128 * a.nsplit;
     const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
     const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
     const int nloc = i1 - i0, nkb = a.K / 64, npad = a.npad;
+    auto krange = [&](int item, int &lo, int &hi) {
+        const int sp = item % a.nsplit;
+        lo = sp * a.kbps;
+        hi = min(nkb, lo + a.kbps);
+    };
     const uint32_t bbytes = (uint32_t)a.planes * npad * 128;
     const uint32_t stage = NA * TC_ABYTES + bbytes;
     // TMEM: two segment buffers and (when a tile has several segments) the
     // running float32 total of the tile
     const uint32_t acc_cols = NA * npad;
-    const int nseg = (nkb + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+    const int nseg_max = (min(nkb, a.kbps) + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
     uint32_t ncols = 32;
-    while (ncols < (nseg > 1 ? 3 : 2) * acc_cols) ncols <<= 1;
+    while (ncols < (nseg_max > 1 ? 3 : 2) * acc_cols) ncols <<= 1;
 
     if (warp == 0) {
         asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(smem_u32(&s_tmem)),
@@ -157,8 +163,10 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
             long long g = 0;
             bool stop = false;
             for (int it = 0; it < nloc && !stop; ++it) {
-                const int y = (i0 + it) * 128;
-                for (int kb = 0; kb < nkb; ++kb, ++g) {
+                const int y = (i0 + it) / a.nsplit * 128;
+                int klo, khi;
+                krange(i0 + it, klo, khi);
+                for (int kb = klo; kb < khi; ++kb, ++g) {
                     const int s = (int)(g % nst);
                     if (g >= nst && !mbar_wait(&empty[s], (uint32_t)((g / nst) - 1) & 1)) {
                         set_status(a.status, OSPREY_ERR_TIMEOUT);
@@ -185,6 +193,9 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
             long long g = 0, u = 0;
             bool stop = false;
             for (int it = 0; it < nloc && !stop; ++it) {
+                int klo, khi;
+                krange(i0 + it, klo, khi);
+                const int nseg = (khi - klo + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
                 for (int sg = 0; sg < nseg && !stop; ++sg, ++u) {
                     const int buf = (int)(u & 1);
                     if (u >= 2 && !mbar_wait(&acce[buf], (uint32_t)((u >> 1) - 1) & 1)) {
@@ -195,7 +206,7 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     }
                     tc_fence_after();
                     const uint32_t d0 = tmem + (uint32_t)buf * acc_cols;
-                    const int kb0 = sg * OSP_TC_SEGKB, kb1 = min(nkb, kb0 + OSP_TC_SEGKB);
+                    const int kb0 = klo + sg * OSP_TC_SEGKB, kb1 = min(khi, kb0 + OSP_TC_SEGKB);
                     for (int kb = kb0; kb < kb1; ++kb, ++g) {
                         const int s = (int)(g % nst);
                         if (!mbar_wait(&full[s], (uint32_t)(g / nst) & 1) || *(volatile int *)&s_abort) {
@@ -232,9 +243,12 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
         long long u = 0;
         bool stop = false;
         for (int it = 0; it < nloc && !stop; ++it) {
-            const int col = (i0 + it) * 128 + m;
+            const int col = (i0 + it) / a.nsplit * 128 + m, sp = (i0 + it) % a.nsplit;
             const bool colok = col < a.nout;
             const uint32_t tt = tmem + ((uint32_t)lg << 16) + 2u * acc_cols;
+            int klo, khi;
+            krange(i0 + it, klo, khi);
+            const int nseg = (khi - klo + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
             for (int sg = 0; sg < nseg; ++sg, ++u) {
                 const int buf = (int)(u & 1);
                 if (!mbar_wait(&accf[buf], (uint32_t)(u >> 1) & 1) || *(volatile int *)&s_abort) {
@@ -263,7 +277,9 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     for (int j = 0; j < 16; ++j) {
                         const int n = c0 + j;
                         if (n >= a.R || !colok) continue;
-                        if (EPI == TC_STORE) {
+                        if (a.nsplit > 1) {   // partial of this k-range; tc_reduce applies the epilogue
+                            a.part[((size_t)sp * a.R + n) * a.nout + col] = v[j];
+                        } else if (EPI == TC_STORE) {
                             a.y[(size_t)n * a.ldy + col] = v[j];
                         } else if (EPI == TC_RESID) {
                             a.x[(size_t)n * a.ldy + col] += v[j];
@@ -288,6 +304,32 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
     __syncthreads();
     tc_fence_after();
     if (warp == 0) asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(ncols));
+}
+
+// ---------------------------------------------------------------- split-K reduction
+// out[n][col] = sum over the k-ranges (in order) of the partials, then the
+// GEMM's epilogue.
+template <int EPI>
+__global__ void __launch_bounds__(256) tc_reduce_kernel(const TcArgs a) {
+    pdl_trigger();
+    pdl_wait();
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)a.R * a.nout) return;
+    const int n = (int)(idx / a.nout), col = (int)(idx % a.nout);
+    float v = 0.f;
+    for (int sp = 0; sp < a.nsplit; ++sp) v += __ldcg(a.part + ((size_t)sp * a.R + n) * a.nout + col);
+    if (EPI == TC_STORE) {
+        a.y[(size_t)n * a.ldy + col] = v;
+    } else if (EPI == TC_RESID) {
+        a.x[(size_t)n * a.ldy + col] += v;
+    } else {
+        const float g = a.y[(size_t)n * a.ldy + col];
+        const float h = g / (1.f + expf(-g)) * v;
+        uint16_t q[TC_PLANES];
+        tc_split(h, q);
+#pragma unroll
+        for (int i = 0; i < TC_PLANES; ++i) a.h[((size_t)i * a.npad + n) * a.nout + col] = q[i];
+    }
 }
 
 // ---------------------------------------------------------------- operand planes
@@ -589,19 +631,43 @@ static cudaError_t pdl_launch(void (*k)(P...), dim3 grid, dim3 block, size_t sme
     return e;
 }
 
-cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s) {
+// k-ranges per output tile so that tiles x ranges fill the CTA slots (few
+// output tiles, long K: the layer projections); 1 for wide outputs.
+int tc_nsplit(int nout, int K, int sms) {
+    const int tiles = (nout + 127) / 128, nkb = K / 64;
+    int want = (OSP_TC_CTAS_PER_SM * sms + tiles - 1) / tiles;
+    if (want < 1) want = 1;
+    if (want > nkb) want = nkb;
+    const int kbps = (nkb + want - 1) / want;
+    return (nkb + kbps - 1) / kbps;
+}
+
+cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s) {
+    TcArgs a = a_in;
     if (a.npad % 16 || a.npad < 16 || a.npad > TC_MAX_ROWS || a.K % 64 || a.R > a.npad) return cudaErrorInvalidValue;
     const int nst = tc_stages(a.npad, a.planes, false);
     if (nst < 2) return cudaErrorInvalidValue;
-    const int nseg = (a.K / 64 + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+    const int nkb = a.K / 64;
+    a.nsplit = a.part ? tc_nsplit(a.nout, a.K, sms) : 1;
+    if ((long long)a.nsplit * a.R * a.nout > a.part_cap) a.nsplit = 1;
+    a.kbps = (nkb + a.nsplit - 1) / a.nsplit;
+    const int nseg = (a.kbps + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
     if ((nseg > 1 ? 3 : 2) * a.npad > 512 / OSP_TC_CTAS_PER_SM) return cudaErrorInvalidValue;   // TMEM columns
-    const int items = (a.nout + 127) / 128;
+    const int items = (a.nout + 127) / 128 * a.nsplit;
     const int grid = items < OSP_TC_CTAS_PER_SM * sms ? items : OSP_TC_CTAS_PER_SM * sms;
     const size_t smem = tc_smem_bytes(a.npad, a.planes, false);
+    cudaError_t e;
     switch (a.epi) {
-    case TC_STORE: return pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
-    case TC_RESID: return pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
-    default: return pdl_launch(tc_kernel<TC_GLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
+    case TC_STORE: e = pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    case TC_RESID: e = pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    default: e = pdl_launch(tc_kernel<TC_GLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    }
+    if (e != cudaSuccess || a.nsplit == 1) return e;
+    const unsigned rblocks = (unsigned)(((long long)a.R * a.nout + 255) / 256);
+    switch (a.epi) {
+    case TC_STORE: return pdl_launch(tc_reduce_kernel<TC_STORE>, dim3(rblocks), dim3(256), 0, s, a);
+    case TC_RESID: return pdl_launch(tc_reduce_kernel<TC_RESID>, dim3(rblocks), dim3(256), 0, s, a);
+    default: return pdl_launch(tc_reduce_kernel<TC_GLU>, dim3(rblocks), dim3(256), 0, s, a);
     }
 }
 

@@ -40,6 +40,10 @@ struct TcArgs {
     float *x;          // TC_RESID: [R][ldy] float32, +=
     uint16_t *h;       // TC_GLU: [TC_PLANES][npad][nout] bf16 planes of silu(gate) * up
     int32_t *status;
+    // split-K: per-range float32 partials [nsplit][R][nout] (null: no split)
+    float *part;
+    long long part_cap;   // floats available in part
+    int nsplit, kbps;     // set by launch_tc
 };
 
 // Host side.  Tensor maps: weights [rows][K] bf16 with a 64 x 128 box, operand
@@ -53,6 +57,10 @@ size_t tc_smem_bytes(int npad, int planes, bool pair);
 cudaError_t tc_set_attributes();
 // SwiGLU runs as two passes: the gate projection (TC_STORE into a float32
 // buffer), then the up projection whose epilogue (TC_GLU) forms silu(gate) * up.
+// Outputs narrower than the CTA slots are split along K (tc_nsplit ranges per
+// 128-feature tile); the float32 partials are then summed in range order by a
+// reduction kernel that applies the epilogue.
+int tc_nsplit(int nout, int K, int sms);
 cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s);
 
 // Operand preparation: rows of float32 (optionally RMS-normalised with a bf16
