@@ -525,6 +525,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.part = ws.attn_part;
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
+            at.status = dev_status;
             e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
             // x += W_o attn;  x += W_down (silu(W_g n) * W_u n),  n = RMSNorm(x)
@@ -570,6 +571,7 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.part = ws.attn_part;
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
+            at.status = dev_status;
             e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
             g.W = (const uint16_t *)W.W_o[l];

@@ -423,15 +423,16 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
 // ---------------------------------------------------------------------------
 // Split-KV GQA decode attention with the split merge kept on chip.  A cluster
 // of CS blocks takes one (row, KV head); block k of the cluster takes the k-th
-// key range, its 8 warps the range's pages round-robin.  Each block reduces its
-// warps in shared memory; after a cluster barrier every block merges one slice
-// of the G x HD outputs from all CS block partials through distributed shared
-// memory, and a second barrier keeps the partials alive until all slices are
-// done.  Every block of a cluster shares the row, so a block either reaches both
-// barriers or its whole cluster returns before the first.
-// Before griddepcontrol.wait (for G <= 2) a warp already loads its first page
-// id and the K/V rows of that page below pos0, the context committed before
-// this draft call, which no kernel of the call writes.
+// key range, its warps the range's pages round-robin.  Each warp streams its
+// pages through its own ring of ATTN_NSPW shared-memory stages with 1-D bulk
+// copies (one page of one head is P x HD contiguous bf16 for K and again for V);
+// the pages wholly below pos0, the context committed before this draft call
+// that no kernel of the call writes, are requested before griddepcontrol.wait.
+// Each block reduces its warps in shared memory and pushes its partial
+// (max, sum, G x HD accumulator) into block 0's shared memory through
+// distributed shared memory; block 0 merges the CS partials after one cluster
+// barrier.  Every block of a cluster shares the row, so either all of them
+// reach the barriers or the whole cluster returns before the first.
 #ifndef OSP_ATTN_CS
 #define OSP_ATTN_CS 8       // blocks per cluster (16 needs the non-portable cluster size)
 #endif
@@ -441,96 +442,118 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
 constexpr int ACT = OSP_ATTN_WARPS * 32;
 
 template <int HD, int G, int CS>
+struct AttnCluster {
+    static constexpr int NW = ACT / 32;
+    static constexpr int PB = 16 * HD * 2;   // bytes of one page of one head (K or V)
+    static constexpr int STATIC = NW * G * HD * 4 + CS * G * HD * 4 + 2 * (NW + CS) * G * 4 + 256;
+    static constexpr int NSPW = (200 * 1024 - STATIC) / (NW * 2 * PB) >= 2 ? 2 : 1;   // stages per warp
+    static constexpr int RING = NW * NSPW * 2 * PB;
+};
+
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait_acquire() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async_smem() {
+    asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+template <int HD, int G, int CS>
 __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
     namespace cg = cooperative_groups;
+    using C = AttnCluster<HD, G, CS>;
     constexpr int LPK = HD / 8;
     constexpr int KPL = 32 / LPK;
-    constexpr int NIT = 16 / KPL;     // loads per page (16 positions)
-    constexpr int NW = ACT / 32;
-    constexpr bool PREFETCH = G <= 2;
-    constexpr int SLICE = G * HD / CS;   // outputs merged by each block of the cluster
-    static_assert(SLICE <= ACT && SLICE * CS == G * HD, "slice");
+    constexpr int NIT = 16 / KPL;     // row loads per page (16 positions)
+    constexpr int NW = C::NW, NSPW = C::NSPW, PB = C::PB;
+    extern __shared__ __align__(128) uint8_t ring[];   // [NW][NSPW][K | V][PB]
+    __shared__ __align__(8) uint64_t full[NW][NSPW];
     __shared__ float sm_m[NW][G], sm_l[NW][G];
     __shared__ float sm_acc[NW][G][HD];
-    __shared__ float bm[G], bl[G];
-    __shared__ float bacc[G][HD];
+    __shared__ float gm[CS][G], gl[CS][G];   // block 0: the partials of the cluster
+    __shared__ float gacc[CS][G][HD];
     cg::cluster_group cluster = cg::this_cluster();
     const Dims &D = a.dim;
     const int split = (int)cluster.block_rank(), kvh = blockIdx.y, r = blockIdx.z;
-    pdl_trigger();   // the next projection may start streaming its weights
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    cluster_arrive_relaxed();   // this block has started: its shared memory may be written by the cluster
+    pdl_trigger();              // the next projection may start streaming its weights
     int b, pos;
     if (!a.map.row(r, b, pos)) return;   // the whole cluster (same row) leaves here
     const int n_keys = pos + 1, pos0 = a.map.pos0[b];
-    const int k_begin = split * a.split_len;
+    const int k_begin = split * a.split_len;   // a multiple of the page size
     const int k_end = min(n_keys, k_begin + a.split_len);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int pg0 = k_begin / 16;
+    const int npg = k_end > k_begin ? (k_end - k_begin + 15) / 16 : 0;
+    const int my_pages = npg > warp ? (npg - warp + NW - 1) / NW : 0;   // local pages warp + j * NW
     const int kg = lane / LPK, dl = (lane % LPK) * 8;
     const float scale = rsqrtf((float)HD);
     const size_t head_stride = (size_t)D.P * HD;
+    uint8_t *wring = ring + (size_t)warp * NSPW * 2 * PB;
+    const int32_t *ptab = a.page_table + (size_t)b * a.max_pages + pg0;
 
-    int pg = k_begin / D.P + warp;
-    // page ids of the warp's first pages (the page table is fixed for the call)
-    constexpr int NPID = 4;
-    int pid[NPID];
-#pragma unroll
-    for (int k = 0; k < NPID; ++k) {
-        const int pk = pg + k * NW;
-        pid[k] = pk * D.P < k_end ? __ldg(a.page_table + (size_t)b * a.max_pages + pk) : 0;
-    }
-    uint4 kr[NIT], vr[NIT];
-    const uint16_t *kb0 = nullptr, *vb0 = nullptr;
-    bool first = PREFETCH && pg * D.P < k_end;
-    if (first) {
-        const int page = pid[0];
-        kb0 = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
-        vb0 = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
-#pragma unroll
-        for (int it = 0; it < NIT; ++it) {
-            const int slot = it * KPL + kg;
-            if (pg * D.P + slot < pos0) {
-                kr[it] = ld_stream(kb0 + slot * HD + dl);
-                vr[it] = ld_stream(vb0 + slot * HD + dl);
-            }
-        }
+    auto issue = [&](int j) {   // lane 0: page j of this warp into stage j % NSPW
+        const int page = __ldg(ptab + warp + j * NW);
+        const int st = j % NSPW;
+        uint8_t *dst = wring + (size_t)st * 2 * PB;
+        mbar_arrive_expect_tx(&full[warp][st], 2 * PB);
+        bulk_g2s(dst, a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride, PB, &full[warp][st]);
+        bulk_g2s(dst + PB, a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride, PB, &full[warp][st]);
+    };
+    int issued = 0;
+    if (lane == 0) {
+        for (int st = 0; st < NSPW; ++st) mbar_init(&full[warp][st], 1);
+        mbar_fence_init();
+        const int first = min(NSPW, my_pages);
+        // committed pages: every position of the page below pos0
+        while (issued < first && (pg0 + warp + issued * NW + 1) * 16 <= pos0) issue(issued++);
     }
     pdl_wait();   // q and this call's K/V rows come from the QKV kernels
+    if (lane == 0)
+        for (; issued < min(NSPW, my_pages); ++issued) issue(issued);
+    __syncwarp();
 
     float q[G][8], acc[G][8], m_run[G], l[G];
 #pragma unroll
     for (int g = 0; g < G; ++g) {
         const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dl;
+        const float4 q0 = *(const float4 *)qp, q1 = *(const float4 *)(qp + 4);
+        q[g][0] = q0.x * scale; q[g][1] = q0.y * scale; q[g][2] = q0.z * scale; q[g][3] = q0.w * scale;
+        q[g][4] = q1.x * scale; q[g][5] = q1.y * scale; q[g][6] = q1.z * scale; q[g][7] = q1.w * scale;
 #pragma unroll
-        for (int e = 0; e < 8; ++e) { q[g][e] = qp[e] * scale; acc[g][e] = 0.f; }
+        for (int e = 0; e < 8; ++e) acc[g][e] = 0.f;
         m_run[g] = -INFINITY;
         l[g] = 0.f;
     }
-    for (int it_pg = 0; pg * D.P < k_end; pg += NW, ++it_pg) {
-        if (first) {
-            // the prefetched page: rows of this call now
-#pragma unroll
-            for (int it = 0; it < NIT; ++it) {
-                const int slot = it * KPL + kg;
-                if (pg * D.P + slot >= pos0) {
-                    kr[it] = ld_stream(kb0 + slot * HD + dl);
-                    vr[it] = ld_stream(vb0 + slot * HD + dl);
-                }
-            }
-            first = false;
-        } else {
-            int page = 0;
-#pragma unroll
-            for (int k = 0; k < NPID; ++k)
-                if (k == it_pg) page = pid[k];
-            if (it_pg >= NPID) page = a.page_table[(size_t)b * a.max_pages + pg];
-            const uint16_t *kb = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
-            const uint16_t *vb = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
-#pragma unroll
-            for (int it = 0; it < NIT; ++it) {
-                const int slot = it * KPL + kg;
-                kr[it] = ld_stream(kb + slot * HD + dl);
-                vr[it] = ld_stream(vb + slot * HD + dl);
-            }
+    int consumed = 0;
+    for (int j = 0; j < my_pages; ++j) {
+        const int st = j % NSPW;
+        if (!__all_sync(0xffffffffu, mbar_wait(&full[warp][st], (uint32_t)(j / NSPW) & 1))) {   // warp-uniform exit
+            if (lane == 0) set_status(a.status, OSPREY_ERR_TIMEOUT);
+            break;
         }
+        consumed = j + 1;
+        const uint16_t *ks = (const uint16_t *)(wring + (size_t)st * 2 * PB);
+        const uint16_t *vs = ks + 16 * HD;
+        uint4 kr[NIT], vr[NIT];
+#pragma unroll
+        for (int it = 0; it < NIT; ++it) {
+            const int slot = it * KPL + kg;
+            kr[it] = *(const uint4 *)(ks + slot * HD + dl);
+            vr[it] = *(const uint4 *)(vs + slot * HD + dl);
+        }
+        __syncwarp();
+        if (lane == 0 && j + NSPW < my_pages) {   // refill the stage once every lane has read it
+            fence_proxy_async_smem();
+            issue(j + NSPW);
+            issued = j + NSPW + 1;
+        }
+        const int key0 = (pg0 + warp + j * NW) * 16;
 #pragma unroll
         for (int g = 0; g < G; ++g) {
             float sc[NIT];
@@ -544,7 +567,7 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
                 for (int e = 0; e < 8; ++e) p = fmaf(q[g][e], kf[e], p);
 #pragma unroll
                 for (int o = LPK / 2; o; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
-                const int key = pg * D.P + it * KPL + kg;
+                const int key = key0 + it * KPL + kg;
                 sc[it] = key < k_end ? p : -INFINITY;
                 mx = fmaxf(mx, sc[it]);
             }
@@ -568,6 +591,9 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
             m_run[g] = m_new;
         }
     }
+    // after a timed-out wait: let the copies already requested land before the block can exit
+    if (lane == 0)
+        for (int j = consumed; j < issued; ++j) mbar_wait(&full[warp][j % NSPW], (uint32_t)(j / NSPW) & 1, 200000000LL);
     // merge the key groups of the warp, then the warps of the block
 #pragma unroll
     for (int g = 0; g < G; ++g) {
@@ -584,6 +610,10 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
         if (lane == 0) { sm_m[warp][g] = m_run[g]; sm_l[warp][g] = l[g]; }
     }
     __syncthreads();
+    cluster_wait_acquire();   // every block of the cluster has started
+    float *r_acc = cluster.map_shared_rank(&gacc[split][0][0], 0);
+    float *r_m = cluster.map_shared_rank(&gm[split][0], 0);
+    float *r_l = cluster.map_shared_rank(&gl[split][0], 0);
     for (int idx = threadIdx.x; idx < G * HD; idx += ACT) {
         const int g = idx / HD, dim = idx % HD;
         float M = -INFINITY;
@@ -597,33 +627,26 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
                 num = fmaf(f, sm_acc[w][g][dim], num);
                 den = fmaf(f, sm_l[w][g], den);
             }
-        bacc[g][dim] = num;
-        if (dim == 0) { bm[g] = M; bl[g] = den; }
+        r_acc[idx] = num;
+        if (dim == 0) { r_m[g] = M; r_l[g] = den; }
     }
-    cluster.sync();   // every block's partial is visible to its cluster
-    if (threadIdx.x < SLICE) {
-        const int idx = split * SLICE + threadIdx.x;
+    cluster_arrive_release();   // the pushed partial is visible to block 0 once it waits
+    if (split != 0) return;
+    cluster_wait_acquire();
+    for (int idx = threadIdx.x; idx < G * HD; idx += ACT) {
         const int g = idx / HD, dim = idx % HD;
-        float pm[CS], pl[CS], pa[CS];
-#pragma unroll
-        for (int k = 0; k < CS; ++k) {
-            pm[k] = *cluster.map_shared_rank(&bm[g], k);
-            pl[k] = *cluster.map_shared_rank(&bl[g], k);
-            pa[k] = *cluster.map_shared_rank(&bacc[g][dim], k);
-        }
         float M = -INFINITY;
 #pragma unroll
-        for (int k = 0; k < CS; ++k) M = fmaxf(M, pm[k]);
+        for (int k = 0; k < CS; ++k) M = fmaxf(M, gm[k][g]);
         float num = 0.f, den = 0.f;
 #pragma unroll
         for (int k = 0; k < CS; ++k) {
-            const float f = pm[k] == -INFINITY ? 0.f : __expf(pm[k] - M);
-            num = fmaf(f, pa[k], num);
-            den = fmaf(f, pl[k], den);
+            const float f = gm[k][g] == -INFINITY ? 0.f : __expf(gm[k][g] - M);
+            num = fmaf(f, gacc[k][g][dim], num);
+            den = fmaf(f, gl[k][g], den);
         }
         a.out[(size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num / den;
     }
-    cluster.sync();   // the partials stay readable until every slice is merged
 }
 
 // ---------------------------------------------------------------------------
@@ -981,6 +1004,7 @@ static cudaLaunchConfig_t attn_cluster_cfg(const AttnArgs &a, cudaStream_t s, cu
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(CS, a.dim.Hkv, a.R);
     cfg.blockDim = dim3(ACT);
+    cfg.dynamicSmemBytes = AttnCluster<HD, G, CS>::RING;
     cfg.stream = s;
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = CS;
@@ -1002,6 +1026,12 @@ static bool attn_cluster_ok(const Dims &D) {
         cudaGetLastError();
         return false;
     }
+    if (cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnCluster<HD, G, CS>::RING) !=
+        cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    if (D.P != 16) return false;   // the page loop takes 16 positions per page
     AttnArgs a{};
     a.dim = D;
     a.R = 1;

@@ -98,6 +98,7 @@ struct AttnArgs {
     float *part;
     float *out;
     int *ticket;
+    int32_t *status;
 };
 
 struct LmArgs {
