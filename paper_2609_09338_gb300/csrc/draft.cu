@@ -446,7 +446,8 @@ struct AttnCluster {
     static constexpr int NW = ACT / 32;
     static constexpr int PB = 16 * HD * 2;   // bytes of one page of one head (K or V)
     static constexpr int STATIC = NW * G * HD * 4 + CS * G * HD * 4 + 2 * (NW + CS) * G * 4 + 256;
-    static constexpr int NSPW = (200 * 1024 - STATIC) / (NW * 2 * PB) >= 2 ? 2 : 1;   // stages per warp
+    static constexpr int FIT = (220 * 1024 - STATIC) / (NW * 2 * PB);
+    static constexpr int NSPW = FIT > 4 ? 4 : (FIT < 1 ? 1 : FIT);   // stages per warp
     static constexpr int RING = NW * NSPW * 2 * PB;
 };
 
@@ -462,6 +463,33 @@ __device__ __forceinline__ void cluster_wait_acquire() {
 __device__ __forceinline__ void fence_proxy_async_smem() {
     asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
+
+// Transposed butterfly over a group of 2*O lanes holding N partial sums each:
+// every level hands half of the lane's values to its partner and adds the half
+// it receives, so after log2(2*O) levels each lane holds N / (2*O) complete
+// sums (for N < 2*O, one sum shared by 2*O / N lanes).  That is N - 1 shuffles
+// in place of N * log2(2*O).
+template <int N, int O, int NVV>
+struct AttnTrReduce {
+    static __device__ __forceinline__ void run(float (&v)[NVV], int lane) {
+        if constexpr (O >= 1) {
+            if constexpr (N >= 2) {
+                constexpr int H = N / 2;
+                const bool up = (lane & O) != 0;
+#pragma unroll
+                for (int i = 0; i < H; ++i) {
+                    const float send = up ? v[i] : v[i + H];
+                    const float keep = up ? v[i + H] : v[i];
+                    v[i] = keep + __shfl_xor_sync(0xffffffffu, send, O);
+                }
+                AttnTrReduce<H, O / 2, NVV>::run(v, lane);
+            } else {
+                v[0] += __shfl_xor_sync(0xffffffffu, v[0], O);
+                AttnTrReduce<1, O / 2, NVV>::run(v, lane);
+            }
+        }
+    }
+};
 
 template <int HD, int G, int CS>
 __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
@@ -479,7 +507,8 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
     __shared__ float gacc[CS][G][HD];
     cg::cluster_group cluster = cg::this_cluster();
     const Dims &D = a.dim;
-    const int split = (int)cluster.block_rank(), kvh = blockIdx.y, r = blockIdx.z;
+    const int split = (int)cluster.block_rank(), r = blockIdx.z;
+    const int qh0 = blockIdx.y * G, kvh = qh0 / (D.Hq / D.Hkv);   // the block's G query heads share a KV head
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     cluster_arrive_relaxed();   // this block has started: its shared memory may be written by the cluster
     pdl_trigger();              // the next projection may start streaming its weights
@@ -497,38 +526,58 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
     uint8_t *wring = ring + (size_t)warp * NSPW * 2 * PB;
     const int32_t *ptab = a.page_table + (size_t)b * a.max_pages + pg0;
 
-    auto issue = [&](int j) {   // lane 0: page j of this warp into stage j % NSPW
-        const int page = __ldg(ptab + warp + j * NW);
+    // lane i holds the page id of the warp's i-th page (the page table is fixed for the call)
+    const int my_pid = lane < my_pages ? __ldg(ptab + warp + lane * NW) : 0;
+    auto issue = [&](int j, int page) {   // lane 0: page j of this warp into stage j % NSPW
         const int st = j % NSPW;
         uint8_t *dst = wring + (size_t)st * 2 * PB;
         mbar_arrive_expect_tx(&full[warp][st], 2 * PB);
         bulk_g2s(dst, a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride, PB, &full[warp][st]);
         bulk_g2s(dst + PB, a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride, PB, &full[warp][st]);
     };
+    auto pid_of = [&](int j) {   // warp-wide
+        const int p = __shfl_sync(0xffffffffu, my_pid, j & 31);
+        return j < 32 ? p : __ldg(ptab + warp + j * NW);
+    };
+    const int first = min(NSPW, my_pages);
+    int pids[NSPW];
+#pragma unroll
+    for (int j = 0; j < NSPW; ++j) pids[j] = pid_of(j);
     int issued = 0;
     if (lane == 0) {
         for (int st = 0; st < NSPW; ++st) mbar_init(&full[warp][st], 1);
         mbar_fence_init();
-        const int first = min(NSPW, my_pages);
         // committed pages: every position of the page below pos0
-        while (issued < first && (pg0 + warp + issued * NW + 1) * 16 <= pos0) issue(issued++);
+#pragma unroll
+        for (int j = 0; j < NSPW; ++j)
+            if (j == issued && j < first && (pg0 + warp + j * NW + 1) * 16 <= pos0) issue(issued++, pids[j]);
     }
     pdl_wait();   // q and this call's K/V rows come from the QKV kernels
-    if (lane == 0)
-        for (; issued < min(NSPW, my_pages); ++issued) issue(issued);
+    if (lane == 0) {
+#pragma unroll
+        for (int j = 0; j < NSPW; ++j)
+            if (j >= issued && j < first) issue(j, pids[j]);
+        issued = first;
+    }
     __syncwarp();
 
-    float q[G][8], acc[G][8], m_run[G], l[G];
+    constexpr int NV = G * NIT;                    // partial dot products per lane and page
+    constexpr int NF = NV >= LPK ? NV / LPK : 1;   // complete scores per lane after the reduction
+    constexpr int REP = NV >= LPK ? 1 : LPK / NV;  // lanes holding the same score
+    constexpr int LPG = LPK / G;                   // lanes of a key group per query head
+    static_assert(G <= LPK && NF <= NIT, "score layout");
+    const int sbase = ((lane % LPK) / REP) * NF;   // the lane's scores: head sbase / NIT
+    float q[G][8], acc[G][8], m_run[G];
+    float m_own_run = -INFINITY, l_own = 0.f;      // the lane's head: running max, partial sum
 #pragma unroll
     for (int g = 0; g < G; ++g) {
-        const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dl;
+        const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(qh0 + g) * HD + dl;
         const float4 q0 = *(const float4 *)qp, q1 = *(const float4 *)(qp + 4);
         q[g][0] = q0.x * scale; q[g][1] = q0.y * scale; q[g][2] = q0.z * scale; q[g][3] = q0.w * scale;
         q[g][4] = q1.x * scale; q[g][5] = q1.y * scale; q[g][6] = q1.z * scale; q[g][7] = q1.w * scale;
 #pragma unroll
         for (int e = 0; e < 8; ++e) acc[g][e] = 0.f;
         m_run[g] = -INFINITY;
-        l[g] = 0.f;
     }
     int consumed = 0;
     for (int j = 0; j < my_pages; ++j) {
@@ -547,59 +596,95 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
             kr[it] = *(const uint4 *)(ks + slot * HD + dl);
             vr[it] = *(const uint4 *)(vs + slot * HD + dl);
         }
-        __syncwarp();
-        if (lane == 0 && j + NSPW < my_pages) {   // refill the stage once every lane has read it
-            fence_proxy_async_smem();
-            issue(j + NSPW);
-            issued = j + NSPW + 1;
+        if (j + NSPW < my_pages) {   // refill the stage once every lane has read it
+            const int pn = pid_of(j + NSPW);
+            __syncwarp();
+            if (lane == 0) {
+                fence_proxy_async_smem();
+                issue(j + NSPW, pn);
+                issued = j + NSPW + 1;
+            }
         }
         const int key0 = (pg0 + warp + j * NW) * 16;
+        // partial q.k over the lane's HD / LPK dimensions, each K chunk unpacked once
+        float v[NV];
+#pragma unroll
+        for (int it = 0; it < NIT; ++it) {
+            float kf[8];
+            unpack8(kr[it], kf);
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+                float d = 0.f;
+#pragma unroll
+                for (int e = 0; e < 8; ++e) d = fmaf(q[g][e], kf[e], d);
+                v[g * NIT + it] = d;
+            }
+        }
+        // complete the sums across the LPK lanes of each key group, leaving the
+        // lane NF consecutive scores (indices sbase .. sbase + NF - 1 of g * NIT + it)
+        AttnTrReduce<NV, LPK / 2, NV>::run(v, lane);
+        float mloc = -INFINITY;
+#pragma unroll
+        for (int i = 0; i < NF; ++i) {
+            const int key = key0 + ((sbase + i) % NIT) * KPL + kg;
+            v[i] = key < k_end ? v[i] : -INFINITY;
+            mloc = fmaxf(mloc, v[i]);
+        }
+        // page maximum of the lane's head, then of every head
+#pragma unroll
+        for (int o = 1; o < LPG; o <<= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+#pragma unroll
+        for (int o = LPK; o < 32; o <<= 1) mloc = fmaxf(mloc, __shfl_xor_sync(0xffffffffu, mloc, o));
+        float corr[G];
 #pragma unroll
         for (int g = 0; g < G; ++g) {
-            float sc[NIT];
-            float mx = -INFINITY;
+            const float mn = fmaxf(m_run[g], __shfl_sync(0xffffffffu, mloc, g * LPG));
+            corr[g] = mn == -INFINITY ? 1.f : __expf(m_run[g] - mn);
+            m_run[g] = mn;
+        }
+        const float m_own = fmaxf(m_own_run, mloc);
+        l_own *= m_own == -INFINITY ? 1.f : __expf(m_own_run - m_own);
+        m_own_run = m_own;
+        float p[NF];
 #pragma unroll
-            for (int it = 0; it < NIT; ++it) {
-                float kf[8];
-                unpack8(kr[it], kf);
-                float p = 0.f;
+        for (int i = 0; i < NF; ++i) {
+            p[i] = v[i] == -INFINITY ? 0.f : __expf(v[i] - m_own);
+            l_own += p[i];
+        }
 #pragma unroll
-                for (int e = 0; e < 8; ++e) p = fmaf(q[g][e], kf[e], p);
+        for (int g = 0; g < G; ++g)
 #pragma unroll
-                for (int o = LPK / 2; o; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
-                const int key = key0 + it * KPL + kg;
-                sc[it] = key < k_end ? p : -INFINITY;
-                mx = fmaxf(mx, sc[it]);
+            for (int e = 0; e < 8; ++e) acc[g][e] *= corr[g];
+        // p . V: each V chunk unpacked once, each weight fetched from the lane holding it
+#pragma unroll
+        for (int it = 0; it < NIT; ++it) {
+            float vf[8];
+            unpack8(vr[it], vf);
+#pragma unroll
+            for (int g = 0; g < G; ++g) {
+                const int vi = g * NIT + it;
+                const float pp = __shfl_sync(0xffffffffu, p[vi % NF], (lane & ~(LPK - 1)) | ((vi / NF) * REP));
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(pp, vf[e], acc[g][e]);
             }
-#pragma unroll
-            for (int o = LPK; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            const float m_new = fmaxf(m_run[g], mx);
-            if (m_new == -INFINITY) continue;   // no key of this page for the warp yet
-            const float corr = __expf(m_run[g] - m_new);
-            l[g] *= corr;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc[g][e] *= corr;
-#pragma unroll
-            for (int it = 0; it < NIT; ++it) {
-                const float p = __expf(sc[it] - m_new);
-                float vf[8];
-                unpack8(vr[it], vf);
-                l[g] += p;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p, vf[e], acc[g][e]);
-            }
-            m_run[g] = m_new;
         }
     }
     // after a timed-out wait: let the copies already requested land before the block can exit
     if (lane == 0)
         for (int j = consumed; j < issued; ++j) mbar_wait(&full[warp][j % NSPW], (uint32_t)(j / NSPW) & 1, 200000000LL);
-    // merge the key groups of the warp, then the warps of the block
+    // the warp's sums per head (REP lanes hold each score), then merge the key
+    // groups of the warp and the warps of the block
+#pragma unroll
+    for (int o = 1; o < LPG; o <<= 1) l_own += __shfl_xor_sync(0xffffffffu, l_own, o);
+#pragma unroll
+    for (int o = LPK; o < 32; o <<= 1) l_own += __shfl_xor_sync(0xffffffffu, l_own, o);
+    float l[G];
+#pragma unroll
+    for (int g = 0; g < G; ++g) l[g] = __shfl_sync(0xffffffffu, l_own, g * LPG) * (1.f / REP);
 #pragma unroll
     for (int g = 0; g < G; ++g) {
 #pragma unroll
         for (int o = LPK; o < 32; o <<= 1) {
-            l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
 #pragma unroll
             for (int e = 0; e < 8; ++e) acc[g][e] += __shfl_xor_sync(0xffffffffu, acc[g][e], o);
         }
@@ -645,7 +730,7 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
             num = fmaf(f, gacc[k][g][dim], num);
             den = fmaf(f, gl[k][g], den);
         }
-        a.out[(size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num / den;
+        a.out[(size_t)r * D.Hq * HD + (size_t)(qh0 + g) * HD + dim] = num / den;
     }
 }
 
@@ -1002,7 +1087,7 @@ cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s) {
 template <int HD, int G, int CS>
 static cudaLaunchConfig_t attn_cluster_cfg(const AttnArgs &a, cudaStream_t s, cudaLaunchAttribute (&attr)[2]) {
     cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(CS, a.dim.Hkv, a.R);
+    cfg.gridDim = dim3(CS, a.dim.Hq / G, a.R);
     cfg.blockDim = dim3(ACT);
     cfg.dynamicSmemBytes = AttnCluster<HD, G, CS>::RING;
     cfg.stream = s;
