@@ -436,17 +436,22 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
 #ifndef OSP_ATTN_CS
 #define OSP_ATTN_CS 8       // blocks per cluster (16 needs the non-portable cluster size)
 #endif
-#ifndef OSP_ATTN_WARPS
-#define OSP_ATTN_WARPS 8    // warps per block
+#ifndef OSP_ATTN_RING_KB
+#define OSP_ATTN_RING_KB 220   // shared memory budget of a block (ring + partials)
 #endif
-constexpr int ACT = OSP_ATTN_WARPS * 32;
+#ifndef OSP_ATTN_WARPS
+#define OSP_ATTN_WARPS 16   // warps per block for groups of up to two query heads (8 beyond)
+#endif
 
 template <int HD, int G, int CS>
 struct AttnCluster {
-    static constexpr int NW = ACT / 32;
+    // groups of <= 2 heads fit 128 registers: 16 warps, every page of a 2k-key
+    // range in flight at once; larger groups keep 8 warps and more stages each
+    static constexpr int NW = G <= 2 ? OSP_ATTN_WARPS : 8;
+    static constexpr int THREADS = NW * 32;
     static constexpr int PB = 16 * HD * 2;   // bytes of one page of one head (K or V)
     static constexpr int STATIC = NW * G * HD * 4 + CS * G * HD * 4 + 2 * (NW + CS) * G * 4 + 256;
-    static constexpr int FIT = (220 * 1024 - STATIC) / (NW * 2 * PB);
+    static constexpr int FIT = (OSP_ATTN_RING_KB * 1024 - STATIC) / (NW * 2 * PB);
     static constexpr int NSPW = FIT > 4 ? 4 : (FIT < 1 ? 1 : FIT);   // stages per warp
     static constexpr int RING = NW * NSPW * 2 * PB;
 };
@@ -492,7 +497,7 @@ struct AttnTrReduce {
 };
 
 template <int HD, int G, int CS>
-__global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
+__global__ void __launch_bounds__(AttnCluster<HD, G, CS>::THREADS, 1) attn_cluster_kernel(const AttnArgs a) {
     namespace cg = cooperative_groups;
     using C = AttnCluster<HD, G, CS>;
     constexpr int LPK = HD / 8;
@@ -699,7 +704,7 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
     float *r_acc = cluster.map_shared_rank(&gacc[split][0][0], 0);
     float *r_m = cluster.map_shared_rank(&gm[split][0], 0);
     float *r_l = cluster.map_shared_rank(&gl[split][0], 0);
-    for (int idx = threadIdx.x; idx < G * HD; idx += ACT) {
+    for (int idx = threadIdx.x; idx < G * HD; idx += C::THREADS) {
         const int g = idx / HD, dim = idx % HD;
         float M = -INFINITY;
 #pragma unroll
@@ -718,7 +723,7 @@ __global__ void __launch_bounds__(ACT) attn_cluster_kernel(const AttnArgs a) {
     cluster_arrive_release();   // the pushed partial is visible to block 0 once it waits
     if (split != 0) return;
     cluster_wait_acquire();
-    for (int idx = threadIdx.x; idx < G * HD; idx += ACT) {
+    for (int idx = threadIdx.x; idx < G * HD; idx += C::THREADS) {
         const int g = idx / HD, dim = idx % HD;
         float M = -INFINITY;
 #pragma unroll
@@ -1088,7 +1093,7 @@ template <int HD, int G, int CS>
 static cudaLaunchConfig_t attn_cluster_cfg(const AttnArgs &a, cudaStream_t s, cudaLaunchAttribute (&attr)[2]) {
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(CS, a.dim.Hq / G, a.R);
-    cfg.blockDim = dim3(ACT);
+    cfg.blockDim = dim3(AttnCluster<HD, G, CS>::THREADS);
     cfg.dynamicSmemBytes = AttnCluster<HD, G, CS>::RING;
     cfg.stream = s;
     attr[0].id = cudaLaunchAttributeClusterDimension;

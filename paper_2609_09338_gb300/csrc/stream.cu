@@ -44,6 +44,12 @@ namespace osp {
 #ifndef OSP_SG_BLOCKS_PER_SM
 #define OSP_SG_BLOCKS_PER_SM 2
 #endif
+#ifndef OSP_SG_GEMV_BPS
+#define OSP_SG_GEMV_BPS OSP_SG_BLOCKS_PER_SM   // blocks per SM of the layer GEMVs
+#endif
+#ifndef OSP_SG_MIN_BLOCKS
+#define OSP_SG_MIN_BLOCKS 2   // register budget: this many blocks (of any stream kernel) per SM
+#endif
 #ifndef OSP_SG_NPROD
 #define OSP_SG_NPROD 1   // producer lanes; lane p issues stages p, p + NPROD, ...
 #endif
@@ -419,7 +425,7 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
 // NRS = weight rows per stage (single modes: items; pair modes: 2 * items, the
 // second segment at row `items` of the slot).
 template <int MODE, int RG, int NRS>
-__global__ void __launch_bounds__(SG_THREADS, OSP_SG_BLOCKS_PER_SM) stream_kernel(const StreamArgs a) {
+__global__ void __launch_bounds__(SG_THREADS, OSP_SG_MIN_BLOCKS) stream_kernel(const StreamArgs a) {
     constexpr bool PAIR = MODE == G_QKV || MODE == G_GATEUP;
     constexpr int NI = PAIR ? NRS / 2 : NRS;   // items per full stage
     extern __shared__ __align__(128) uint8_t smem[];
@@ -698,7 +704,8 @@ StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms) {
         p.stage_bytes = rows * row_bytes;
     }
     p.n_stages = (p.n_items + p.items - 1) / p.items;
-    p.blocks = p.n_stages < sms * OSP_SG_BLOCKS_PER_SM ? p.n_stages : sms * OSP_SG_BLOCKS_PER_SM;
+    const int bps = mode == G_LM ? OSP_SG_BLOCKS_PER_SM : OSP_SG_GEMV_BPS;
+    p.blocks = p.n_stages < sms * bps ? p.n_stages : sms * bps;
     p.smem = (size_t)SG_NST * p.stage_bytes;
     return p;
 }
