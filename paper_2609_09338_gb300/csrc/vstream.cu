@@ -34,10 +34,25 @@ namespace osp {
 #define OSP_VS_BPS 2   // resident blocks per SM (grid = OSP_VS_BPS x SMs at most)
 #endif
 
+#ifndef OSP_VS_NST
+#define OSP_VS_NST 12  // ring slots per block
+#endif
+#ifndef OSP_VS_ROWB
+#define OSP_VS_ROWB 4096   // bytes of one row chunk (the workspace holds 4 KB float32 chunks at least)
+#endif
+
 constexpr int VS_CW = 8;
 constexpr int VS_THREADS = (VS_CW + 1) * 32;
-constexpr int VS_NST = 12;
-constexpr int VS_ROWB = 4096;              // bytes of one row chunk
+constexpr int VS_NST = OSP_VS_NST;
+constexpr int VS_ROWB = OSP_VS_ROWB;       // bytes of one row chunk
+static_assert(VS_ROWB % 4096 == 0, "row chunks are whole multiples of 4 KB");
+// Slot s serves tiles s, s + NST, s + 2 NST, ... and tile j belongs to warp
+// j % CW, so consecutive uses of a slot can belong to different warps.  A wait
+// on a phase parity is exact only while the barrier is at most one phase
+// behind: a warp reaching use u of a slot first waits for use u - 1 to be freed
+// (vs_wait_slot).  That wait is itself exact because use u - 2 belongs to the
+// same warp, which has freed it: 2 NST must be a multiple of CW.
+static_assert((2 * VS_NST) % VS_CW == 0, "ring slots: 2 x slots must be a multiple of the consumer warps");
 constexpr int VS_SLOT = 2 * VS_ROWB;       // target chunk + draft chunk
 constexpr int VS_NV = VS_ROWB / 16 / 32;   // 16-byte vectors per lane per row chunk (8)
 
@@ -48,6 +63,40 @@ __device__ __forceinline__ float vs_ex2(float x) {
     return y;
 }
 constexpr float VS_LOG2E = 1.4426950408889634f;
+
+// Consumer wait for tile j of a block: the slot's previous use (another warp's
+// tile) freed, then tile j's copy complete.  False when a bounded wait ran out.
+__device__ __forceinline__ bool vs_wait_slot(uint64_t *full, uint64_t *empty, int j) {
+    const int slot = j % VS_NST, use = j / VS_NST;
+    if (use > 0 && !mbar_wait(&empty[slot], (use - 1) & 1)) return false;
+    return mbar_wait(&full[slot], use & 1);
+}
+
+// Position of tile t = (row * nch + c) with row = b * rows_per_seq + i, advanced
+// incrementally: the 64-bit divisions run once per launch and once per row,
+// not once per tile.
+struct VsCur {
+    long long row;
+    int b, i, c;
+    __device__ __forceinline__ void set_row(int rows_per_seq) {
+        b = (int)(row / rows_per_seq);
+        i = (int)(row - (long long)b * rows_per_seq);
+    }
+    __device__ __forceinline__ void init(long long t, int nch, int rows_per_seq) {
+        row = t / nch;
+        c = (int)(t - row * nch);
+        set_row(rows_per_seq);
+    }
+    __device__ __forceinline__ void step(int n, int nch, int rows_per_seq) {
+        c += n;
+        if (c < nch) return;
+        do {
+            c -= nch;
+            ++row;
+        } while (c >= nch);
+        set_row(rows_per_seq);
+    }
+};
 
 template <typename T> struct VsT;
 template <> struct VsT<float> {
@@ -300,25 +349,20 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_stats(const VerifyArgs a) {
     __syncthreads();
     pdl_trigger();
     pdl_wait();
-    auto decode = [&](long long t, int &b, int &i, int &c) {
-        c = (int)(t % nch);
-        const long long ri = t / nch;
-        i = (int)(ri % (K + 1));
-        b = (int)(ri / (K + 1));
-    };
     if (warp == VS_CW) {
         if (lane == 0) {
             const uint64_t pol = policy_evict_first();
             int issued = 0;
-            for (int j = 0; j < n; ++j) {
+            VsCur cur;
+            cur.init(t0, nch, K + 1);
+            for (int j = 0; j < n; ++j, cur.step(1, nch, K + 1)) {
                 const int slot = j % VS_NST;
                 if (j >= VS_NST && !mbar_wait(&empty[slot], ((j / VS_NST) - 1) & 1)) {
                     set_status(a.status, OSPREY_ERR_TIMEOUT);
                     atomicExch(&s_abort, 1);
                     break;
                 }
-                int b, i, c;
-                decode(t0 + j, b, i, c);
+                const int b = cur.b, i = cur.i, c = cur.c;
                 const int nel = min(L::EL, V - c * L::EL);
                 uint8_t *dst = smem + (size_t)slot * VS_SLOT;
                 issued = j + 1;
@@ -347,17 +391,18 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_stats(const VerifyArgs a) {
     long long cur_row = -1;
     int pend = 0;
     bool aborted = false;
-    for (int j = warp; j < n; j += VS_CW) {
-        int b, i, c;
-        decode(t0 + j, b, i, c);
-        const long long row = (t0 + j) / nch;
+    VsCur cur;
+    cur.init(t0 + warp, nch, K + 1);
+    for (int j = warp; j < n; j += VS_CW, cur.step(VS_CW, nch, K + 1)) {
+        const int i = cur.i, c = cur.c;
+        const long long row = cur.row;
         if (row != cur_row) {
             if (pend) vs_row_done<GREEDY>(a, (size_t)cur_row, pend);
             cur_row = row;
             pend = 0;
         }
         const int slot = j % VS_NST;
-        if (!mbar_wait(&full[slot], (j / VS_NST) & 1)) {
+        if (!vs_wait_slot(full, empty, j)) {
             set_status(a.status, OSPREY_ERR_TIMEOUT);
             atomicExch(&s_abort, 1);
             mbar_wait(&full[slot], (j / VS_NST) & 1, 200000000LL);
@@ -618,15 +663,16 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_sample(const VerifyArgs a) {
         if (lane == 0) {
             const uint64_t pol = policy_evict_first();
             int issued = 0, rb = -1, r = -1;
-            for (int j = 0; j < n; ++j) {
+            VsCur cur;
+            cur.init(t0, nch, 1);
+            for (int j = 0; j < n; ++j, cur.step(1, nch, 1)) {
                 const int slot = j % VS_NST;
                 if (j >= VS_NST && !mbar_wait(&empty[slot], ((j / VS_NST) - 1) & 1)) {
                     set_status(a.status, OSPREY_ERR_TIMEOUT);
                     atomicExch(&s_abort, 1);
                     break;
                 }
-                const long long t = t0 + j;
-                const int b = (int)(t / nch), c = (int)(t % nch);
+                const int b = (int)cur.row, c = cur.c;
                 if (b != rb) {
                     r = __ldcg(&decs[b].r);
                     rb = b;
@@ -661,9 +707,11 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_sample(const VerifyArgs a) {
     int cur_b = -1, pend = 0;
     bool aborted = false;
     Decision d{};
-    for (int j = warp; j < n; j += VS_CW) {
+    VsCur cur;
+    cur.init(t0 + warp, nch, 1);
+    for (int j = warp; j < n; j += VS_CW, cur.step(VS_CW, nch, 1)) {
         const long long t = t0 + j;
-        const int b = (int)(t / nch), c = (int)(t % nch);
+        const int b = (int)cur.row, c = cur.c;
         if (b != cur_b) {
             if (pend && vs_arrive(a.ticket2 + cur_b, pend, nch) && d.r >= 0) vs_pick<T>(a, cur_b, d);
             cur_b = b;
@@ -672,7 +720,7 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_sample(const VerifyArgs a) {
             if (d.r > K) d.r = -1;   // corrupt decision (reported by the producer)
         }
         const int slot = j % VS_NST;
-        if (!mbar_wait(&full[slot], (j / VS_NST) & 1)) {
+        if (!vs_wait_slot(full, empty, j)) {
             set_status(a.status, OSPREY_ERR_TIMEOUT);
             atomicExch(&s_abort, 1);
             mbar_wait(&full[slot], (j / VS_NST) & 1, 200000000LL);
