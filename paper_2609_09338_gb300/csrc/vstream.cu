@@ -554,26 +554,29 @@ __device__ void vs_pick(const VerifyArgs &a, int b, const Decision &d) {
     const uint4 *gp = (const uint4 *)((const T *)a.target + rowp);
     const uint4 *gq = (const uint4 *)((const T *)a.draft + rowq);
     const int nel = min(L::EL, V - chunk * L::EL);   // a multiple of VW (rows are 16-byte multiples)
+    // in two halves, so that the loads in flight stay in registers next to the
+    // walk's state (the kernel keeps two blocks per SM)
     float seg[VS_NV];
-    {
-        uint4 vp[VS_NV], vq[VS_NV];
 #pragma unroll
-        for (int k = 0; k < VS_NV; ++k) {
-            const bool in = (lane + 32 * k) * L::VW < nel;
-            vp[k] = in ? __ldg(gp + lane + 32 * k) : make_uint4(0, 0, 0, 0);
-            vq[k] = in && residual ? __ldg(gq + lane + 32 * k) : make_uint4(0, 0, 0, 0);
+    for (int h = 0; h < VS_NV; h += VS_NV / 2) {
+        uint4 vp[VS_NV / 2], vq[VS_NV / 2];
+#pragma unroll
+        for (int k = 0; k < VS_NV / 2; ++k) {
+            const bool in = (lane + 32 * (h + k)) * L::VW < nel;
+            vp[k] = in ? __ldg(gp + lane + 32 * (h + k)) : make_uint4(0, 0, 0, 0);
+            vq[k] = in && residual ? __ldg(gq + lane + 32 * (h + k)) : make_uint4(0, 0, 0, 0);
         }
 #pragma unroll
-        for (int k = 0; k < VS_NV; ++k) {
+        for (int k = 0; k < VS_NV / 2; ++k) {
             float f[L::VW], g[L::VW];
             L::unpack(vp[k], f);
             L::unpack(vq[k], g);
             float w = 0.f;
-            if ((lane + 32 * k) * L::VW < nel) {
+            if ((lane + 32 * (h + k)) * L::VW < nel) {
 #pragma unroll
                 for (int e = 0; e < L::VW; ++e) w += vs_weight(f[e], g[e], nrm, residual, fallback);
             }
-            seg[k] = w;
+            seg[h + k] = w;
         }
     }
     // segment walk (every lane holds every segment's total)
