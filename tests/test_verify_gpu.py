@@ -92,6 +92,34 @@ def test_verify_workload_shapes(name):
         check_verify(g0["out_tokens"], g0["n_accepted"], o0, wl.K)
 
 
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_verify_ring_reuse_repeated(dtype):
+    """Hundreds of tiles per block, so every ring slot is reused many times by
+    different consumer warps: repeated calls (sampled and greedy) must all end
+    with status 0, give identical outputs, and match the oracle."""
+    from paper_2609_09338_gb300.session import VerifyBuffers
+    V, B, K = 65536, 128, 8
+    vi = syn.make_verify_inputs(V, B, K, 1.0, 0.7, seed=77)
+    conv = _dev if dtype == "f32" else _bf16
+    zp, zq = conv(vi["target_logits"]), conv(vi["draft_logits"])
+    toks, ua, us = _dev(vi["draft_tokens"]), _dev(vi["u_accept"]), _dev(vi["u_sample"])
+    for T in (1.0, 0.0):
+        vb = VerifyBuffers(B, K, V)
+        first = None
+        for rep in range(12):
+            vb.run(zp, zq if T > 0 else None, toks, T, ua, us)
+            torch.cuda.synchronize()
+            assert int(vb.status.item()) == 0, (T, rep)
+            got = (vb.out_tokens.cpu().numpy().copy(), vb.n_accepted.cpu().numpy().copy())
+            if first is None:
+                first = got
+                o = _oracle(vi, T, dtype)
+                check_verify(got[0], got[1], o, K)
+            else:
+                np.testing.assert_array_equal(got[0], first[0])
+                np.testing.assert_array_equal(got[1], first[1])
+
+
 def test_identical_drafter_accepts_everything():
     rng = np.random.default_rng(5)
     B, K, V = 6, 7, 151936
