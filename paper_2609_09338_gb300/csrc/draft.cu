@@ -239,223 +239,11 @@ __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
 }
 
 // ---------------------------------------------------------------------------
-// Split-KV GQA decode attention.  Block (split, kv head, row); 4 warps take the
-// split's pages round-robin.  HD/8 lanes share one key (8 dims, 16 bytes each).
-template <int HD, int G>
-__global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
-    constexpr int LPK = HD / 8;
-    constexpr int KPL = 32 / LPK;
-    constexpr int NIT = 16 / KPL;     // loads per page (16 positions)
-    __shared__ float sm_m[AT / 32][G], sm_l[AT / 32][G];
-    __shared__ float sm_acc[AT / 32][G][HD];
-    const Dims &D = a.dim;
-    const int split = blockIdx.x, kvh = blockIdx.y, r = blockIdx.z;
-    pdl_trigger();   // the next projection may start streaming its weights
-    pdl_wait();      // q and this step's K/V row come from the QKV kernel
-    int b, pos;
-    if (!a.map.row(r, b, pos)) return;
-    const int n_keys = pos + 1;
-    const int k_begin = split * a.split_len;
-    const int k_end = min(n_keys, k_begin + a.split_len);
-    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int kg = lane / LPK, dl = (lane % LPK) * 8;
-    const float scale = rsqrtf((float)HD);
-
-    float q[G][8], acc[G][8], m_run[G], l[G];
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-        const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(kvh * G + g) * HD + dl;
-#pragma unroll
-        for (int e = 0; e < 8; ++e) { q[g][e] = qp[e] * scale; acc[g][e] = 0.f; }
-        m_run[g] = -INFINITY;
-        l[g] = 0.f;
-    }
-    const size_t head_stride = (size_t)D.P * HD;
-    for (int pg = k_begin / D.P + warp; pg * D.P < k_end; pg += AT / 32) {
-        const int page = a.page_table[(size_t)b * a.max_pages + pg];
-        const uint16_t *kb = a.k_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
-        const uint16_t *vb = a.v_pages + ((size_t)page * D.Hkv + kvh) * head_stride;
-        uint4 kr[NIT], vr[NIT];
-#pragma unroll
-        for (int it = 0; it < NIT; ++it) {
-            const int slot = it * KPL + kg;
-            kr[it] = ld_stream(kb + slot * HD + dl);
-            vr[it] = ld_stream(vb + slot * HD + dl);
-        }
-#pragma unroll
-        for (int g = 0; g < G; ++g) {
-            float sc[NIT];
-            float mx = -INFINITY;
-#pragma unroll
-            for (int it = 0; it < NIT; ++it) {
-                float kf[8];
-                unpack8(kr[it], kf);
-                float p = 0.f;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) p = fmaf(q[g][e], kf[e], p);
-#pragma unroll
-                for (int o = LPK / 2; o; o >>= 1) p += __shfl_xor_sync(0xffffffffu, p, o);
-                const int key = pg * D.P + it * KPL + kg;
-                sc[it] = key < k_end ? p : -INFINITY;
-                mx = fmaxf(mx, sc[it]);
-            }
-#pragma unroll
-            for (int o = LPK; o < 32; o <<= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
-            const float m_new = fmaxf(m_run[g], mx);
-            const float corr = __expf(m_run[g] - m_new);
-            l[g] *= corr;
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc[g][e] *= corr;
-#pragma unroll
-            for (int it = 0; it < NIT; ++it) {
-                const float p = __expf(sc[it] - m_new);
-                float vf[8];
-                unpack8(vr[it], vf);
-                l[g] += p;
-#pragma unroll
-                for (int e = 0; e < 8; ++e) acc[g][e] = fmaf(p, vf[e], acc[g][e]);
-            }
-            m_run[g] = m_new;
-        }
-    }
-    // merge the key groups of the warp, then the warps of the block
-#pragma unroll
-    for (int g = 0; g < G; ++g) {
-#pragma unroll
-        for (int o = LPK; o < 32; o <<= 1) {
-            l[g] += __shfl_xor_sync(0xffffffffu, l[g], o);
-#pragma unroll
-            for (int e = 0; e < 8; ++e) acc[g][e] += __shfl_xor_sync(0xffffffffu, acc[g][e], o);
-        }
-        if (lane < LPK) {
-#pragma unroll
-            for (int e = 0; e < 8; ++e) sm_acc[warp][g][dl + e] = acc[g][e];
-        }
-        if (lane == 0) { sm_m[warp][g] = m_run[g]; sm_l[warp][g] = l[g]; }
-    }
-    __syncthreads();
-    const int Hq = D.Hq;
-    for (int idx = threadIdx.x; idx < G * HD; idx += AT) {
-        const int g = idx / HD, dim = idx % HD;
-        float M = -INFINITY;
-        for (int w = 0; w < AT / 32; ++w) M = fmaxf(M, sm_m[w][g]);
-        float num = 0.f, den = 0.f;
-        if (M != -INFINITY)
-            for (int w = 0; w < AT / 32; ++w) {
-                const float f = __expf(sm_m[w][g] - M);
-                num = fmaf(f, sm_acc[w][g][dim], num);
-                den = fmaf(f, sm_l[w][g], den);
-            }
-        float *pp = a.part + (((size_t)r * Hq + kvh * G + g) * a.n_splits + split) * (HD + 2);
-        pp[2 + dim] = num;
-        if (dim == 0) { pp[0] = M; pp[1] = den; }
-    }
-    if (!arrive_last(a.ticket + (size_t)r * D.Hkv + kvh, a.n_splits)) return;
-    // last split block of this (row, KV head): merge the split partials.  A
-    // thread issues every load it needs at once (split maxima and sums, and its
-    // accumulator values for up to SPR splits), so up to SPR splits cost one
-    // round trip to L2.
-    constexpr int IPT = (G * HD + AT - 1) / AT;            // (head, dim) items per thread
-    constexpr int SPR = IPT >= 8 ? 8 : (IPT >= 4 ? 16 : 32);  // splits per pass, <= 64 values held
-    __shared__ float s_w[G][ATTN_MAX_SPLITS], s_l[G][ATTN_MAX_SPLITS];
-    __shared__ float s_den[G];
-    const int ns = a.n_splits;
-    const float *base = a.part + ((size_t)r * Hq + kvh * G) * ns * (HD + 2);
-    for (int idx = threadIdx.x; idx < G * ns; idx += AT) {
-        const int g = idx / ns, sp = idx % ns;
-        const float *pp = base + ((size_t)g * ns + sp) * (HD + 2);
-        s_w[g][sp] = __ldcg(pp);
-        s_l[g][sp] = __ldcg(pp + 1);
-    }
-    float v[IPT][SPR];
-    auto load_pass = [&](int s0) {
-#pragma unroll
-        for (int it = 0; it < IPT; ++it) {
-            const int idx = threadIdx.x + it * AT;
-            const int g = idx / HD, dim = idx % HD;
-#pragma unroll
-            for (int k = 0; k < SPR; ++k)
-                v[it][k] = idx < G * HD && s0 + k < ns
-                               ? __ldcg(base + ((size_t)g * ns + s0 + k) * (HD + 2) + 2 + dim)
-                               : 0.f;
-        }
-    };
-    load_pass(0);
-    __syncthreads();
-    for (int g = warp; g < G; g += AT / 32) {
-        float M = -INFINITY;
-        for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, s_w[g][sp]);
-        M = warp_max(M);
-        float den = 0.f;
-        for (int sp = lane; sp < ns; sp += 32) {
-            const float ms = s_w[g][sp];
-            const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
-            den = fmaf(f, s_l[g][sp], den);
-            s_w[g][sp] = f;
-        }
-        den = warp_sum(den);
-        if (lane == 0) s_den[g] = den;
-    }
-    __syncthreads();
-    float num[IPT];
-#pragma unroll
-    for (int it = 0; it < IPT; ++it) num[it] = 0.f;
-    for (int s0 = 0; s0 < ns; s0 += SPR) {
-        if (s0 > 0) load_pass(s0);
-#pragma unroll
-        for (int it = 0; it < IPT; ++it) {
-            const int g = (threadIdx.x + it * AT) / HD;
-            if (g >= G) continue;
-#pragma unroll
-            for (int k = 0; k < SPR; ++k)
-                if (s0 + k < ns) num[it] = fmaf(s_w[g][s0 + k], v[it][k], num[it]);
-        }
-    }
-#pragma unroll
-    for (int it = 0; it < IPT; ++it) {
-        const int idx = threadIdx.x + it * AT;
-        if (idx >= G * HD) continue;
-        const int g = idx / HD, dim = idx % HD;
-        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num[it] / s_den[g];
-    }
-}
-
-// ---------------------------------------------------------------------------
-// Split-KV GQA decode attention with the split merge kept on chip.  A cluster
-// of CS blocks takes one (row, KV head); block k of the cluster takes the k-th
-// key range, its warps the range's pages round-robin.  Each warp streams its
-// pages through its own ring of ATTN_NSPW shared-memory stages with 1-D bulk
-// copies (one page of one head is P x HD contiguous bf16 for K and again for V);
-// the pages wholly below pos0, the context committed before this draft call
-// that no kernel of the call writes, are requested before griddepcontrol.wait.
-// Each block reduces its warps in shared memory and pushes its partial
-// (max, sum, G x HD accumulator) into block 0's shared memory through
-// distributed shared memory; block 0 merges the CS partials after one cluster
-// barrier.  Every block of a cluster shares the row, so either all of them
-// reach the barriers or the whole cluster returns before the first.
-#ifndef OSP_ATTN_CS
-#define OSP_ATTN_CS 8       // blocks per cluster (16 needs the non-portable cluster size)
-#endif
-#ifndef OSP_ATTN_RING_KB
-#define OSP_ATTN_RING_KB 220   // shared memory budget of a block (ring + partials)
-#endif
-#ifndef OSP_ATTN_WARPS
-#define OSP_ATTN_WARPS 16   // warps per block for groups of up to two query heads (8 beyond)
-#endif
-
-template <int HD, int G, int CS>
-struct AttnCluster {
-    // groups of <= 2 heads fit 128 registers: 16 warps, every page of a 2k-key
-    // range in flight at once; larger groups keep 8 warps and more stages each
-    static constexpr int NW = G <= 2 ? OSP_ATTN_WARPS : 8;
-    static constexpr int THREADS = NW * 32;
-    static constexpr int PB = 16 * HD * 2;   // bytes of one page of one head (K or V)
-    static constexpr int STATIC = NW * G * HD * 4 + CS * G * HD * 4 + 2 * (NW + CS) * G * 4 + 256;
-    static constexpr int FIT = (OSP_ATTN_RING_KB * 1024 - STATIC) / (NW * 2 * PB);
-    static constexpr int NSPW = FIT > 4 ? 4 : (FIT < 1 ? 1 : FIT);   // stages per warp
-    static constexpr int RING = NW * NSPW * 2 * PB;
-};
-
+// Split-KV GQA decode attention (Sec. 4, paged serving).  Both kernels below
+// give a block (key range, KV head, row) and its warps the range's pages
+// round-robin (attn_warp_pages); HD/8 lanes share one key (8 dims, 16 bytes
+// each).  attn_kernel merges the ranges through global partials (the last block
+// of a (row, KV head) merges); attn_cluster_kernel merges them on chip.
 __device__ __forceinline__ void cluster_arrive_relaxed() {
     asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
@@ -496,32 +284,24 @@ struct AttnTrReduce {
     }
 };
 
-template <int HD, int G, int CS>
-__global__ void __launch_bounds__(AttnCluster<HD, G, CS>::THREADS, 1) attn_cluster_kernel(const AttnArgs a) {
-    namespace cg = cooperative_groups;
-    using C = AttnCluster<HD, G, CS>;
+// One warp's share of a key range [k_begin, k_end) of row r, KV head kvh: its
+// pages (warp, warp + NW, ...) stream through the warp's own NSPW shared-memory
+// stages with 1-D bulk copies; pages wholly below pos0 (the context committed
+// before this draft call, which no kernel of the call writes) are requested
+// before griddepcontrol.wait, which this function executes.  Per page each K/V
+// chunk is unpacked once for the G query heads and the q.k sums are completed
+// by a transposed butterfly (one score per lane).  Leaves the warp's partial
+// (max, sum, G x HD accumulator) in sm_m / sm_l / sm_acc[warp].
+template <int HD, int G, int NW, int NSPW>
+__device__ __forceinline__ void attn_warp_pages(const AttnArgs &a, int b, int r, int kvh, int qh0, int k_begin,
+                                                int k_end, int pos0, uint8_t *ring, uint64_t (*full)[NSPW],
+                                                float (*sm_m)[G], float (*sm_l)[G], float (*sm_acc)[G][HD]) {
     constexpr int LPK = HD / 8;
     constexpr int KPL = 32 / LPK;
     constexpr int NIT = 16 / KPL;     // row loads per page (16 positions)
-    constexpr int NW = C::NW, NSPW = C::NSPW, PB = C::PB;
-    extern __shared__ __align__(128) uint8_t ring[];   // [NW][NSPW][K | V][PB]
-    __shared__ __align__(8) uint64_t full[NW][NSPW];
-    __shared__ float sm_m[NW][G], sm_l[NW][G];
-    __shared__ float sm_acc[NW][G][HD];
-    __shared__ float gm[CS][G], gl[CS][G];   // block 0: the partials of the cluster
-    __shared__ float gacc[CS][G][HD];
-    cg::cluster_group cluster = cg::this_cluster();
+    constexpr int PB = 16 * HD * 2;   // bytes of one page of one head (K or V)
     const Dims &D = a.dim;
-    const int split = (int)cluster.block_rank(), r = blockIdx.z;
-    const int qh0 = blockIdx.y * G, kvh = qh0 / (D.Hq / D.Hkv);   // the block's G query heads share a KV head
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    cluster_arrive_relaxed();   // this block has started: its shared memory may be written by the cluster
-    pdl_trigger();              // the next projection may start streaming its weights
-    int b, pos;
-    if (!a.map.row(r, b, pos)) return;   // the whole cluster (same row) leaves here
-    const int n_keys = pos + 1, pos0 = a.map.pos0[b];
-    const int k_begin = split * a.split_len;   // a multiple of the page size
-    const int k_end = min(n_keys, k_begin + a.split_len);
     const int pg0 = k_begin / 16;
     const int npg = k_end > k_begin ? (k_end - k_begin + 15) / 16 : 0;
     const int my_pages = npg > warp ? (npg - warp + NW - 1) / NW : 0;   // local pages warp + j * NW
@@ -699,6 +479,180 @@ __global__ void __launch_bounds__(AttnCluster<HD, G, CS>::THREADS, 1) attn_clust
         }
         if (lane == 0) { sm_m[warp][g] = m_run[g]; sm_l[warp][g] = l[g]; }
     }
+}
+
+// Stages per warp of the global-partials attention (4 warps per block): two
+// or three blocks fit an SM next to the ring.
+template <int HD>
+struct AttnSplit {
+    static constexpr int PB = 16 * HD * 2;
+    static constexpr int NSPW = HD == 128 ? 2 : 4;
+    static constexpr int RING = (AT / 32) * NSPW * 2 * PB;
+};
+
+template <int HD, int G>
+__global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
+    constexpr int NW = AT / 32, NSPW = AttnSplit<HD>::NSPW;
+    extern __shared__ __align__(128) uint8_t ring[];   // [NW][NSPW][K | V][PB]
+    __shared__ __align__(8) uint64_t full[NW][NSPW];
+    __shared__ float sm_m[NW][G], sm_l[NW][G];
+    __shared__ float sm_acc[NW][G][HD];
+    const Dims &D = a.dim;
+    const int split = blockIdx.x, kvh = blockIdx.y, r = blockIdx.z;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    pdl_trigger();   // the next projection may start streaming its weights
+    int b, pos;
+    if (!a.map.row(r, b, pos)) return;   // the row map was written by the prepare kernel
+    const int n_keys = pos + 1, pos0 = a.map.pos0[b];
+    const int k_begin = split * a.split_len;   // a multiple of the page size
+    const int k_end = min(n_keys, k_begin + a.split_len);
+    attn_warp_pages<HD, G, NW, NSPW>(a, b, r, kvh, kvh * G, k_begin, k_end, pos0, ring, full, sm_m, sm_l, sm_acc);
+    __syncthreads();
+    const int Hq = D.Hq;
+    for (int idx = threadIdx.x; idx < G * HD; idx += AT) {
+        const int g = idx / HD, dim = idx % HD;
+        float M = -INFINITY;
+        for (int w = 0; w < AT / 32; ++w) M = fmaxf(M, sm_m[w][g]);
+        float num = 0.f, den = 0.f;
+        if (M != -INFINITY)
+            for (int w = 0; w < AT / 32; ++w) {
+                const float f = __expf(sm_m[w][g] - M);
+                num = fmaf(f, sm_acc[w][g][dim], num);
+                den = fmaf(f, sm_l[w][g], den);
+            }
+        float *pp = a.part + (((size_t)r * Hq + kvh * G + g) * a.n_splits + split) * (HD + 2);
+        pp[2 + dim] = num;
+        if (dim == 0) { pp[0] = M; pp[1] = den; }
+    }
+    if (!arrive_last(a.ticket + (size_t)r * D.Hkv + kvh, a.n_splits)) return;
+    // last split block of this (row, KV head): merge the split partials.  A
+    // thread issues every load it needs at once (split maxima and sums, and its
+    // accumulator values for up to SPR splits), so up to SPR splits cost one
+    // round trip to L2.
+    constexpr int IPT = (G * HD + AT - 1) / AT;            // (head, dim) items per thread
+    constexpr int SPR = IPT >= 8 ? 8 : (IPT >= 4 ? 16 : 32);  // splits per pass, <= 64 values held
+    __shared__ float s_w[G][ATTN_MAX_SPLITS], s_l[G][ATTN_MAX_SPLITS];
+    __shared__ float s_den[G];
+    const int ns = a.n_splits;
+    const float *base = a.part + ((size_t)r * Hq + kvh * G) * ns * (HD + 2);
+    for (int idx = threadIdx.x; idx < G * ns; idx += AT) {
+        const int g = idx / ns, sp = idx % ns;
+        const float *pp = base + ((size_t)g * ns + sp) * (HD + 2);
+        s_w[g][sp] = __ldcg(pp);
+        s_l[g][sp] = __ldcg(pp + 1);
+    }
+    float v[IPT][SPR];
+    auto load_pass = [&](int s0) {
+#pragma unroll
+        for (int it = 0; it < IPT; ++it) {
+            const int idx = threadIdx.x + it * AT;
+            const int g = idx / HD, dim = idx % HD;
+#pragma unroll
+            for (int k = 0; k < SPR; ++k)
+                v[it][k] = idx < G * HD && s0 + k < ns
+                               ? __ldcg(base + ((size_t)g * ns + s0 + k) * (HD + 2) + 2 + dim)
+                               : 0.f;
+        }
+    };
+    load_pass(0);
+    __syncthreads();
+    for (int g = warp; g < G; g += AT / 32) {
+        float M = -INFINITY;
+        for (int sp = lane; sp < ns; sp += 32) M = fmaxf(M, s_w[g][sp]);
+        M = warp_max(M);
+        float den = 0.f;
+        for (int sp = lane; sp < ns; sp += 32) {
+            const float ms = s_w[g][sp];
+            const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
+            den = fmaf(f, s_l[g][sp], den);
+            s_w[g][sp] = f;
+        }
+        den = warp_sum(den);
+        if (lane == 0) s_den[g] = den;
+    }
+    __syncthreads();
+    float num[IPT];
+#pragma unroll
+    for (int it = 0; it < IPT; ++it) num[it] = 0.f;
+    for (int s0 = 0; s0 < ns; s0 += SPR) {
+        if (s0 > 0) load_pass(s0);
+#pragma unroll
+        for (int it = 0; it < IPT; ++it) {
+            const int g = (threadIdx.x + it * AT) / HD;
+            if (g >= G) continue;
+#pragma unroll
+            for (int k = 0; k < SPR; ++k)
+                if (s0 + k < ns) num[it] = fmaf(s_w[g][s0 + k], v[it][k], num[it]);
+        }
+    }
+#pragma unroll
+    for (int it = 0; it < IPT; ++it) {
+        const int idx = threadIdx.x + it * AT;
+        if (idx >= G * HD) continue;
+        const int g = idx / HD, dim = idx % HD;
+        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num[it] / s_den[g];
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Split-KV GQA decode attention with the split merge kept on chip.  A cluster
+// of CS blocks takes one (row, KV head); block k of the cluster takes the k-th
+// key range, its warps the range's pages round-robin.  Each warp streams its
+// pages through its own ring of ATTN_NSPW shared-memory stages with 1-D bulk
+// copies (one page of one head is P x HD contiguous bf16 for K and again for V);
+// the pages wholly below pos0, the context committed before this draft call
+// that no kernel of the call writes, are requested before griddepcontrol.wait.
+// Each block reduces its warps in shared memory and pushes its partial
+// (max, sum, G x HD accumulator) into block 0's shared memory through
+// distributed shared memory; block 0 merges the CS partials after one cluster
+// barrier.  Every block of a cluster shares the row, so either all of them
+// reach the barriers or the whole cluster returns before the first.
+#ifndef OSP_ATTN_CS
+#define OSP_ATTN_CS 8       // blocks per cluster (16 needs the non-portable cluster size)
+#endif
+#ifndef OSP_ATTN_RING_KB
+#define OSP_ATTN_RING_KB 220   // shared memory budget of a block (ring + partials)
+#endif
+#ifndef OSP_ATTN_WARPS
+#define OSP_ATTN_WARPS 16   // warps per block for groups of up to two query heads (8 beyond)
+#endif
+
+template <int HD, int G, int CS>
+struct AttnCluster {
+    // groups of <= 2 heads fit 128 registers: 16 warps, every page of a 2k-key
+    // range in flight at once; larger groups keep 8 warps and more stages each
+    static constexpr int NW = G <= 2 ? OSP_ATTN_WARPS : 8;
+    static constexpr int THREADS = NW * 32;
+    static constexpr int PB = 16 * HD * 2;   // bytes of one page of one head (K or V)
+    static constexpr int STATIC = NW * G * HD * 4 + CS * G * HD * 4 + 2 * (NW + CS) * G * 4 + 256;
+    static constexpr int FIT = (OSP_ATTN_RING_KB * 1024 - STATIC) / (NW * 2 * PB);
+    static constexpr int NSPW = FIT > 4 ? 4 : (FIT < 1 ? 1 : FIT);   // stages per warp
+    static constexpr int RING = NW * NSPW * 2 * PB;
+};
+
+template <int HD, int G, int CS>
+__global__ void __launch_bounds__(AttnCluster<HD, G, CS>::THREADS, 1) attn_cluster_kernel(const AttnArgs a) {
+    namespace cg = cooperative_groups;
+    using C = AttnCluster<HD, G, CS>;
+    constexpr int NW = C::NW, NSPW = C::NSPW;
+    extern __shared__ __align__(128) uint8_t ring[];   // [NW][NSPW][K | V][PB]
+    __shared__ __align__(8) uint64_t full[NW][NSPW];
+    __shared__ float sm_m[NW][G], sm_l[NW][G];
+    __shared__ float sm_acc[NW][G][HD];
+    __shared__ float gm[CS][G], gl[CS][G];   // block 0: the partials of the cluster
+    __shared__ float gacc[CS][G][HD];
+    cg::cluster_group cluster = cg::this_cluster();
+    const Dims &D = a.dim;
+    const int split = (int)cluster.block_rank(), r = blockIdx.z;
+    const int qh0 = blockIdx.y * G, kvh = qh0 / (D.Hq / D.Hkv);   // the block's G query heads share a KV head
+    cluster_arrive_relaxed();   // this block has started: its shared memory may be written by the cluster
+    pdl_trigger();              // the next projection may start streaming its weights
+    int b, pos;
+    if (!a.map.row(r, b, pos)) return;   // the whole cluster (same row) leaves here
+    const int n_keys = pos + 1, pos0 = a.map.pos0[b];
+    const int k_begin = split * a.split_len;   // a multiple of the page size
+    const int k_end = min(n_keys, k_begin + a.split_len);
+    attn_warp_pages<HD, G, NW, NSPW>(a, b, r, kvh, qh0, k_begin, k_end, pos0, ring, full, sm_m, sm_l, sm_acc);
     __syncthreads();
     cluster_wait_acquire();   // every block of the cluster has started
     float *r_acc = cluster.map_shared_rank(&gacc[split][0][0], 0);
@@ -1055,9 +1009,19 @@ cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaS
 
 template <int HD, int G>
 static cudaError_t launch_attn_t(const AttnArgs &a, cudaStream_t s) {
+    static int attr_dev = -1;   // the ring's dynamic shared memory, opted into once per device
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (attr_dev != dev) {
+        e = cudaFuncSetAttribute(attn_kernel<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnSplit<HD>::RING);
+        if (e != cudaSuccess) return e;
+        attr_dev = dev;
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.n_splits, a.dim.Hkv, a.R);
     cfg.blockDim = dim3(AT);
+    cfg.dynamicSmemBytes = AttnSplit<HD>::RING;
     cfg.stream = s;
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
