@@ -32,12 +32,12 @@ sys.path.insert(0, ROOT)
 from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
 from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: E402
 
-# dram__bytes_read.sum + dram__bytes_write.sum of one LM-head launch (mean of
-# two captured launches of this workload under ncu --set full); valid
-# only for the stream.cu it was taken on.
+# dram__bytes_read.sum + dram__bytes_write.sum of one LM-head launch of this
+# workload (the first LM head of a bench run, ncu --set full); valid only for
+# the stream.cu it was taken on.
 LM_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/stream.cu",
-              "sha256": "6d2d8e13865a495755e07e57e7d0dc969b35d6497914adcb89b08b88e1e83221",
-              "bytes_per_launch": 314_518_784}
+              "sha256": "90d10a609dc3cdd6796755d7c6ff7213e7e7ddeb5064fcb5779e04778e7230de",
+              "bytes_per_launch": 314_359_808}
 
 
 def _sha(path):
