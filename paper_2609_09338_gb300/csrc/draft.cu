@@ -597,12 +597,10 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
 // ---------------------------------------------------------------------------
 // Split-KV GQA decode attention with the split merge kept on chip.  A cluster
 // of CS blocks takes one (row, KV head); block k of the cluster takes the k-th
-// key range, its warps the range's pages round-robin.  Each warp streams its
-// pages through its own ring of ATTN_NSPW shared-memory stages with 1-D bulk
-// copies (one page of one head is P x HD contiguous bf16 for K and again for V);
-// the pages wholly below pos0, the context committed before this draft call
-// that no kernel of the call writes, are requested before griddepcontrol.wait.
-// Each block reduces its warps in shared memory and pushes its partial
+// key range, its warps the range's pages round-robin (attn_warp_pages: each
+// warp streams its pages through its own AttnCluster::NSPW shared-memory stages
+// with 1-D bulk copies, one page of one head being P x HD contiguous bf16 for K
+// and again for V).  Each block reduces its warps in shared memory and pushes its partial
 // (max, sum, G x HD accumulator) into block 0's shared memory through
 // distributed shared memory; block 0 merges the CS partials after one cluster
 // barrier.  Every block of a cluster shares the row, so either all of them

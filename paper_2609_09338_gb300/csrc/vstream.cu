@@ -18,8 +18,9 @@
 // vs_sample: a tile is (sequence b, chunk c) of the decision row r only.  The
 //   warp sums the draw weights max(0, p_r - q_r) (p_K for the bonus) and p_r;
 //   the warp that completes the sequence's count walks the chunk sums in id
-//   order, loads the chosen chunk once and walks its 8 segments, then its
-//   lanes, then one lane's elements (inverse CDF at u_sample[r]).
+//   order, loads the chosen chunk (two halves of loads in flight) and walks its
+//   8 segments, then its lanes, then one lane's elements (inverse CDF at
+//   u_sample[r]).
 // Both kernels are launched as programmatic dependents: barrier set-up overlaps
 // the previous kernel's tail, and every global read follows griddepcontrol.wait.
 #include <math.h>
