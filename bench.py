@@ -171,6 +171,17 @@ def cpu_baseline(wl, ctx, w, kv, di, vi, budget_s=10.0):
                       f"weights widened once ({setup:.1f}s, untimed); {os.cpu_count()} host cores visible"}
 
 
+def max_over_ranks(x: float, world: int, device="cpu") -> float:
+    """The job's time is its slowest replica's: MAX over the ranks (identity for one rank)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
     if rank != 0:
@@ -370,11 +381,7 @@ def main():
     if world > 1:
         dist.barrier()
     step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
-    ms = sum(step_ms) / len(step_ms)
-    if world > 1:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
+    ms = max_over_ranks(sum(step_ms) / len(step_ms), world, dev)
 
     # verify alone (same inputs, L2 flushed): verify GB/s
     vgraph = torch.cuda.CUDAGraph()
@@ -411,7 +418,7 @@ def main():
             h_out["n_accepted"].copy_(vb.n_accepted, non_blocking=True)
             ee[i].record(stream)
     torch.cuda.synchronize()
-    e2e_ms = sum(s.elapsed_time(e) for s, e in zip(es, ee)) / args.steps
+    e2e_ms = max_over_ranks(sum(s.elapsed_time(e) for s, e in zip(es, ee)) / args.steps, world, dev)
     h2d = sum(v.numel() * v.element_size() for v in h_in.values())
     d2h = sum(v.numel() * v.element_size() for v in h_out.values())
 
