@@ -711,11 +711,12 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_sample(const VerifyArgs a) {
     int cur_b = -1, pend = 0;
     bool aborted = false;
     Decision d{};
-    VsCur cur;
-    cur.init(t0 + warp, nch, 1);
-    for (int j = warp; j < n; j += VS_CW, cur.step(VS_CW, nch, 1)) {
+    // the consumer warps divide per tile: with the incremental cursor here the
+    // sampling walk's loads of the chosen chunk measured 4.9 us instead of 1.4 us
+    // at batch 1 (cause not identified)
+    for (int j = warp; j < n; j += VS_CW) {
         const long long t = t0 + j;
-        const int b = (int)cur.row, c = cur.c;
+        const int b = (int)(t / nch), c = (int)(t % nch);
         if (b != cur_b) {
             if (pend && vs_arrive(a.ticket2 + cur_b, pend, nch) && d.r >= 0) vs_pick<T>(a, cur_b, d);
             cur_b = b;
