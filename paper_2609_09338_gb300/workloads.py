@@ -78,6 +78,13 @@ LARGE_VOCAB_DRAFTER = DrafterShape(d_model=1024, n_layers=1, n_q_heads=16, n_kv_
                                    head_dim=128, ffn_dim=3072, vocab=200064,
                                    feat_dim=3 * 3072, rope_theta=1e6)
 
+# The paper's own drafter body (Sec. 3.2; Appendix "Draft Model Sizes"): two
+# Qwen3-4B-shaped blocks, d 2560, 32/8 heads of 128, FFN 9728, on a
+# Qwen3-8B-shaped target (3 x 4096 feature columns, vocabulary 151936).
+OSPREY_PAPER_DRAFTER = DrafterShape(d_model=2560, n_layers=2, n_q_heads=32, n_kv_heads=8,
+                                    head_dim=128, ffn_dim=9728, vocab=151936,
+                                    feat_dim=3 * 4096, rope_theta=1e6)
+
 WORKLOADS = {
     # tiny correctness case: fits the oracle in well under a second
     "tiny-d256-v4096-b1-k4": Workload("tiny-d256-v4096-b1-k4", TINY, batch=1, K=4,
@@ -95,6 +102,11 @@ WORKLOADS = {
     "llama70b-d2048-v128256-b16-k7": Workload("llama70b-d2048-v128256-b16-k7", LLAMA70B_DRAFTER,
                                               batch=16, K=7, ctx_lo=2048, ctx_hi=8192,
                                               temperature=0.7, sigma_p=0.5, seed=1003),
+    # the paper-shaped drafter, one stream; each call extends by 3 accepted rows
+    # (an acceptance length of about 3) before its 7-token chain
+    "osprey-d2560-v151936-b1-k7-ext3": Workload("osprey-d2560-v151936-b1-k7-ext3", OSPREY_PAPER_DRAFTER,
+                                                batch=1, K=7, ctx_lo=2048, ctx_hi=2048, temperature=1.0,
+                                                sigma_p=0.7, seed=1005, n_new=3),
     # large vocabulary, verify-heavy
     "large-vocab-d1024-v200064-b64-k8": Workload("large-vocab-d1024-v200064-b64-k8",
                                                  LARGE_VOCAB_DRAFTER, batch=64, K=8,

@@ -225,10 +225,21 @@ def test_capacity_violation_skips_only_that_sequence():
     ("large-vocab-d1024-v200064-b64-k8", 1.0, [7, 63]),
 ])
 def test_workload_full_size(name, T, sample):
-    """Each workload at its full size; the oracle checks sampled sequences."""
+    """Each workload at its full size, with its extend rows; the oracle checks sampled sequences."""
     wl = WORKLOADS[name]
     ctx = syn.make_contexts(wl)
-    case = run_case(wl.shape, ctx, wl.K, T, wl.seed, sample_seqs=sample)
+    case = run_case(wl.shape, ctx, wl.K, T, wl.seed, n_new=[wl.n_new] * wl.batch, max_new=wl.n_new,
+                    sample_seqs=sample)
+    check_case(case)
+
+
+def test_paper_shaped_body_extend_rows():
+    """The paper's drafter body (two blocks, d 2560, 32/8 heads of 128, FFN 9728,
+    12288 feature columns) at a reduced vocabulary and context: 3 extend rows
+    (tensor-core projections) then a 7-token chain (streamed GEMVs), sampled."""
+    from dataclasses import replace
+    shape = replace(WORKLOADS["osprey-d2560-v151936-b1-k7-ext3"].shape, vocab=16384)
+    case = run_case(shape, [512], 7, 1.0, 1105, n_new=[3], max_new=3)
     check_case(case)
 
 
