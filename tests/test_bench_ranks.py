@@ -55,3 +55,25 @@ def test_reference_arm_prints_only_on_rank_zero():
                         "--warmup", "1"], env=env, capture_output=True, text=True, timeout=300)
     assert r.returncode == 0, r.stderr[-2000:]
     assert r.stdout.strip() == ""
+
+
+def test_reference_arm_line_on_rank_zero():
+    """The reference arm (the float64 oracle on the host cores) prints one JSON
+    line with the same metric and workload as the CUDA arm, and its own
+    cpu_baseline and zero-copy e2e fields."""
+    import json
+    sys.path.insert(0, ROOT)
+    from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD
+    env = {k: v for k, v in os.environ.items() if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK")}
+    r = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                        "--warmup", "1"], env=env, capture_output=True, text=True, timeout=900)
+    assert r.returncode == 0, r.stderr[-2000:]
+    line = json.loads(r.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference"
+    assert line["metric"] == "draft+verify steps/s" and line["unit"] == "steps/s"
+    assert line["higher_is_better"] is True and line["value"] > 0
+    assert line["config"]["workload"] == BENCH_WORKLOAD
+    assert line["cpu_baseline"]["kind"] == "oracle" and line["cpu_baseline"]["cores"] >= 1
+    assert line["cpu_baseline"]["value"] == line["value"]
+    assert line["e2e"] == {"value": line["value"], "unit": "steps/s", "h2d_bytes_per_step": 0,
+                           "d2h_bytes_per_step": 0}
