@@ -105,6 +105,15 @@ typedef struct osprey_ctx osprey_ctx;
 const char *osprey_last_error(void);
 
 /* Validate the shape and weight pointers and make a context (host memory only).
+ * The context picks the kernels a draft call uses:
+ *   rows <= 2 per chain step: TMA-streamed GEMVs (weights read once per step);
+ *   3..80 rows: tcgen05 tensor-core GEMMs, float32 activations split into three
+ *     bf16 planes (24 mantissa bits) so results match the GEMV path's;
+ *   attention: clusters merged on chip while they fit one wave, else global
+ *     partials.
+ * Two environment variables, read here, select the alternatives for testing:
+ * OSPREY_TC=0 (CUDA-core GEMVs for batched rows) and OSPREY_ATTN_CLUSTER=0
+ * (global-partials attention).
  * Errors: INVALID_ARG (null), SHAPE (unsupported dimension). */
 int osprey_create(const osprey_config *cfg, const osprey_weights *w, osprey_ctx **out);
 void osprey_destroy(osprey_ctx *ctx);
