@@ -46,6 +46,7 @@ struct osprey_ctx {
     int sms;
     int attn_cs;    // cluster size of the attention kernel (0: split partials in global memory)
     bool tc;        // batched rows (3..80) run their projections on tcgen05
+    bool fused_mlp; // batch-1 chain steps run O-proj, gate/up and down as one launch
     CUtensorMap tm_c, tm_lm, tm_qkv[OSPREY_MAX_LAYERS], tm_o[OSPREY_MAX_LAYERS], tm_gate[OSPREY_MAX_LAYERS],
         tm_up[OSPREY_MAX_LAYERS], tm_down[OSPREY_MAX_LAYERS];
     double inv_freq[64];
@@ -123,6 +124,10 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
                  tc_encode_weight(&ctx->tm_up[l], W.W_up[l], D.F, D.d) &&
                  tc_encode_weight(&ctx->tm_down[l], W.W_down[l], D.d, D.F);
         ctx->tc = tc;
+        // OSPREY_FUSED_MLP=1 runs O-proj, gate/up and down of a batch-1 chain
+        // step as one launch with grid barriers (not yet the default)
+        const char *menv = std::getenv("OSPREY_FUSED_MLP");
+        ctx->fused_mlp = menv && menv[0] == '1' && mlp_fused_supported(D, ctx->sms);
         cudaGetLastError();
     }
     if (e != cudaSuccess) {
@@ -200,6 +205,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
     size_t o_valid = take(4ull * B), o_pos0 = take(4ull * B), o_nn = take(4ull * B);
     size_t o_at = take(4ull * R_ext * D.Hkv), o_lt = take(4ull * B);
+    size_t o_gb = take(2 * sizeof(unsigned));   // grid barrier of the fused layer tail
     size_t o_xe = take(4ull * R_ext * D.d), o_se = take(4ull * R_ext * D.d);
     size_t o_xc = take(4ull * B * D.d), o_sc = take(4ull * B * D.d);
     size_t o_q = take(4ull * R_ext * D.Hq * D.hd);
@@ -243,6 +249,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->seq_nnew = (int *)(p + o_nn);
         ws->attn_ticket = (int *)(p + o_at);
         ws->lm_ticket = (int *)(p + o_lt);
+        ws->grid_bar = (unsigned *)(p + o_gb);
         ws->x_ext = (float *)(p + o_xe);
         ws->s_ext = (float *)(p + o_se);
         ws->x_chain = (float *)(p + o_xc);
@@ -574,6 +581,24 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             at.status = dev_status;
             e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+            if (streamed && R == 1 && ctx->fused_mlp) {
+                MlpArgs ma{};
+                ma.dim = D;
+                ma.map = map;
+                ma.W_o = (const uint16_t *)W.W_o[l];
+                ma.W_gate = (const uint16_t *)W.W_gate[l];
+                ma.W_up = (const uint16_t *)W.W_up[l];
+                ma.W_down = (const uint16_t *)W.W_down[l];
+                ma.ffn_norm = (const uint16_t *)W.ffn_norm[l];
+                ma.attn = ws.attn_out;
+                ma.x = x;
+                ma.h = ws.ffn_h;
+                ma.bar_count = ws.grid_bar;
+                ma.bar_gen = ws.grid_bar + 1;
+                ma.status = dev_status;
+                if ((e = launch_mlp_fused(ma, ctx->sms, s)) != cudaSuccess) return cuda_fail(e, "fused mlp launch");
+                continue;
+            }
             g.W = (const uint16_t *)W.W_o[l];
             g.xin = ws.attn_out;
             if ((rc = gemv(G_OPROJ, "o-proj launch")) != OSPREY_OK) return rc;

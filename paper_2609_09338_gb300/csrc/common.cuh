@@ -188,4 +188,42 @@ __device__ __forceinline__ void set_status(int32_t *status, int code) {
     if (status) atomicCAS((int *)status, 0, code);
 }
 
+__device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
+    unsigned v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+    return v;
+}
+__device__ __forceinline__ void st_release_gpu(unsigned *p, unsigned v) {
+    asm volatile("st.release.gpu.global.u32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Barrier over every block of a grid whose blocks are all resident at once.
+// `count` is zero between uses (the last block to arrive resets it) and `gen`
+// advances once per use; a block reads `gen` before arriving, so the release
+// cannot be missed.  The wait is bounded (about a second of SM clocks): on
+// expiry the status word gets OSPREY_ERR_TIMEOUT and the block goes on.
+__device__ __forceinline__ void grid_sync(unsigned *count, unsigned *gen, int32_t *status) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        const unsigned g = ld_acquire_gpu(gen);
+        __threadfence();   // this block's writes, ordered before the arrival
+        if (atomicAdd(count, 1u) == gridDim.x - 1) {
+            atomicExch(count, 0u);
+            __threadfence();
+            st_release_gpu(gen, g + 1u);
+        } else {
+            const long long t0 = clock64();
+            while (ld_acquire_gpu(gen) == g) {
+                if (clock64() - t0 > 2000000000LL) {
+                    set_status(status, OSPREY_ERR_TIMEOUT);
+                    break;
+                }
+                __nanosleep(64);
+            }
+        }
+        __threadfence();
+    }
+    __syncthreads();
+}
+
 }  // namespace osp

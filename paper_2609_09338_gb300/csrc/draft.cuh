@@ -19,6 +19,7 @@ struct DraftWs {
     int *seq_valid, *seq_pos0, *seq_nnew;  // [B]
     int *attn_ticket;                      // [R_ext * Hkv]
     int *lm_ticket;                        // [groups]
+    unsigned *grid_bar;                    // [2] grid barrier (count, generation)
     float *x_ext;                          // [B*max_new][d]  residual stream, extend rows
     float *s_ext;                          // [B*max_new][d]  context slot (c)
     float *x_chain;                        // [B][d]          residual stream, chain rows
@@ -165,6 +166,22 @@ struct StreamPlan {
     int items, n_items, n_stages, stage_bytes, blocks;
     size_t smem;
 };
+
+// Batch-1 chain steps: O-proj + residual, RMSNorm + gate/up + SwiGLU and
+// down + residual of one layer in one launch (one block per SM, every block's
+// weight slices requested before griddepcontrol.wait, two grid barriers).
+struct MlpArgs {
+    Dims dim;
+    RowMap map;                       // row 0 of the step
+    const uint16_t *W_o, *W_gate, *W_up, *W_down, *ffn_norm;
+    const float *attn;                // [Hq hd] attention output of the row
+    float *x;                         // [d] residual stream of the row
+    float *h;                         // [F] SwiGLU hidden (scratch)
+    unsigned *bar_count, *bar_gen;    // grid barrier words; count zero between uses
+    int32_t *status;
+};
+bool mlp_fused_supported(const Dims &D, int sms);
+cudaError_t launch_mlp_fused(const MlpArgs &a, int sms, cudaStream_t s);
 
 StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms);
 bool stream_supported(GemvMode mode, const Dims &D, int rg, int sms);
