@@ -24,7 +24,7 @@ import numpy as np
 
 from .workloads import DrafterShape, Workload
 
-_CHUNK = 1 << 24
+_CHUNK = 1 << 20   # elements per pass; buffers of a few MB are reused, not re-faulted
 
 
 def bf16_bits(x: np.ndarray) -> np.ndarray:
@@ -32,24 +32,33 @@ def bf16_bits(x: np.ndarray) -> np.ndarray:
     x = np.ascontiguousarray(x, dtype=np.float32)
     out = np.empty(x.shape, dtype=np.uint16)
     xf, of = x.reshape(-1), out.reshape(-1)
+    t = np.empty(min(_CHUNK, xf.size), dtype=np.uint32)
+    r = np.empty_like(t)
     for s in range(0, xf.size, _CHUNK):
-        u = xf[s:s + _CHUNK].view(np.uint32)
-        r = ((u >> 16) & 1) + np.uint32(0x7FFF)
-        of[s:s + _CHUNK] = ((u + r) >> 16).astype(np.uint16)
+        n = min(_CHUNK, xf.size - s)
+        u, tn, rn = xf[s:s + n].view(np.uint32), t[:n], r[:n]
+        np.right_shift(u, 16, out=rn)
+        np.bitwise_and(rn, 1, out=rn)
+        np.add(rn, np.uint32(0x7FFF), out=rn)
+        np.add(u, rn, out=tn)            # wraps like uint32 arithmetic
+        np.right_shift(tn, 16, out=tn)
+        of[s:s + n] = tn
     return out
 
 
 def _normal_bf16(rng: np.random.Generator, shape, std: float = 1.0, mean: float = 0.0) -> np.ndarray:
     out = np.empty(shape, dtype=np.uint16)
     of = out.reshape(-1)
+    v = np.empty(min(_CHUNK, of.size), dtype=np.float32)
     for s in range(0, of.size, _CHUNK):
         n = min(_CHUNK, of.size - s)
-        v = rng.standard_normal(n, dtype=np.float32)
+        vn = v[:n]
+        rng.standard_normal(n, dtype=np.float32, out=vn)
         if std != 1.0:
-            v *= np.float32(std)
+            vn *= np.float32(std)
         if mean != 0.0:
-            v += np.float32(mean)
-        of[s:s + n] = bf16_bits(v)
+            vn += np.float32(mean)
+        of[s:s + n] = bf16_bits(vn)
     return out
 
 
