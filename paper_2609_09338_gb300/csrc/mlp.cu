@@ -175,13 +175,15 @@ bool mlp_fused_supported(const Dims &D, int sms) {
 cudaError_t launch_mlp_fused(const MlpArgs &a, int sms, cudaStream_t s) {
     const MlpPlan p = mlp_plan(a.dim, sms);
     static int attr_dev = -1;
+    static size_t attr_smem = 0;   // the opt-in grows with the largest shape launched so far
     int dev = 0;
     cudaError_t e = cudaGetDevice(&dev);
     if (e != cudaSuccess) return e;
-    if (attr_dev != dev) {
+    if (attr_dev != dev || p.smem > attr_smem) {
         e = cudaFuncSetAttribute(mlp_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
         if (e != cudaSuccess) return e;
         attr_dev = dev;
+        attr_smem = p.smem;
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(sms);
