@@ -8,6 +8,7 @@ logits (band 1e-5) and against the oracle's logits (band from the measured
 error).  The oracle follows the GPU's chain (teacher forcing) so a flagged
 position does not desynchronise the rows after it.
 """
+import os
 from dataclasses import replace
 
 import numpy as np
@@ -233,11 +234,22 @@ def test_workload_full_size(name, T, sample):
     check_case(case)
 
 
+@pytest.mark.skipif(os.environ.get("OSPREY_TEST_FUSED_MLP") != "1",
+                    reason="the fused layer tail (OSPREY_FUSED_MLP) is off by default; set OSPREY_TEST_FUSED_MLP=1")
+@pytest.mark.parametrize("T", [0.0, 1.0])
+def test_fused_layer_tail_matches_oracle(T, monkeypatch):
+    """Batch-1 chain steps with O-proj, gate/up and down fused into one launch
+    (grid barriers between the phases), Qwen3-8B-shaped drafter."""
+    monkeypatch.setenv("OSPREY_FUSED_MLP", "1")
+    wl = WORKLOADS["qwen3-8b-d1024-v151936-b1-k7"]
+    case = run_case(wl.shape, syn.make_contexts(wl), wl.K, T, wl.seed)
+    check_case(case)
+
+
 def test_paper_shaped_body_extend_rows():
     """The paper's drafter body (two blocks, d 2560, 32/8 heads of 128, FFN 9728,
     12288 feature columns) at a reduced vocabulary and context: 3 extend rows
     (tensor-core projections) then a 7-token chain (streamed GEMVs), sampled."""
-    from dataclasses import replace
     shape = replace(WORKLOADS["osprey-d2560-v151936-b1-k7-ext3"].shape, vocab=16384)
     case = run_case(shape, [512], 7, 1.0, 1105, n_new=[3], max_new=3)
     check_case(case)
