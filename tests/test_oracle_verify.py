@@ -237,3 +237,29 @@ def test_inverse_cdf_point_on_edge_takes_next_bin():
     assert r["out_tokens"][0, 1] == 2
     r = ov.verify(zp2, zp2[:, :1], np.array([[2]]), 1.0, np.array([[0.1]]), np.array([[0.5, 0.25]]))
     assert r["out_tokens"][0, 1] == 1
+
+
+def test_emitted_tokens_pass_chi_square():
+    """Monte Carlo on a 16-token vocabulary: draft tokens x_i ~ q_i, random
+    uniforms; the first emitted token follows p_0 and, among the sequences that
+    accepted position 0, the second follows p_1 (Pearson chi-square).  The same
+    counts reject q_0, so the test can tell the two apart."""
+    from scipy.stats import chisquare
+    rng = np.random.default_rng(11)
+    V, K, N = 16, 3, 40000
+    zp = (rng.standard_normal((K + 1, V)) * 1.5).astype(np.float32)
+    zq = (zp[:K] + rng.standard_normal((K, V)).astype(np.float32)).astype(np.float32)
+    p = sp_softmax(zp.astype(np.float64), axis=-1)
+    q = sp_softmax(zq.astype(np.float64), axis=-1)
+    ud = rng.random((N, K))
+    cq = np.cumsum(q, axis=-1)
+    x = np.stack([np.minimum(np.searchsorted(cq[i], ud[:, i] * cq[i, -1], side="right"), V - 1)
+                  for i in range(K)], 1).astype(np.int32)
+    o = ov.verify(np.broadcast_to(zp, (N, K + 1, V)).copy(), np.broadcast_to(zq, (N, K, V)).copy(), x, 1.0,
+                  rng.random((N, K), dtype=np.float32), rng.random((N, K + 1), dtype=np.float32))
+    first = np.bincount(o["out_tokens"][:, 0], minlength=V)
+    assert chisquare(first, N * p[0]).pvalue > 1e-3
+    assert chisquare(first, N * q[0]).pvalue < 1e-6
+    reached = o["n_accepted"] >= 1
+    second = np.bincount(o["out_tokens"][reached, 1], minlength=V)
+    assert chisquare(second, reached.sum() * p[1]).pvalue > 1e-3
