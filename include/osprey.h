@@ -232,6 +232,17 @@ int osprey_probe_enable(osprey_ctx *ctx, int n_slots);
 int osprey_probe_read(osprey_ctx *ctx, float *ms, int n);
 int64_t osprey_launch_count(void);
 
+/* ---- self-test of the failure path (not part of the method) ------------------
+ * Every device-side wait of the library (mbarrier phases of the TMA rings,
+ * tensor-core commits, grid barriers) is bounded: when the limit runs out the
+ * kernel writes OSPREY_ERR_TIMEOUT to the caller's status word and returns, so
+ * the context stays usable.  This call launches one block that waits on a
+ * barrier nothing completes, for about limit_cycles SM clocks (1 .. 2e9), and
+ * then takes that path: dev_status (device int32, first error wins) reads
+ * OSPREY_ERR_TIMEOUT once the stream reaches it.
+ * Host errors: INVALID_ARG (limit out of range, null status). */
+int osprey_selftest_wait_timeout(int64_t limit_cycles, int32_t *dev_status, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -80,11 +80,12 @@ _c_verify_static = _sig("osprey_verify_static", ctypes.c_int,
 _c_probe_enable = _sig("osprey_probe_enable", ctypes.c_int, [_vp, ctypes.c_int])
 _c_probe_read = _sig("osprey_probe_read", ctypes.c_int, [_vp, ctypes.POINTER(_f32), ctypes.c_int])
 _c_launch_count = _sig("osprey_launch_count", _i64, [])
+_c_selftest_wait = _sig("osprey_selftest_wait_timeout", ctypes.c_int, [_i64, _vp, _vp])
 
 EXPORTED = ["osprey_last_error", "osprey_create", "osprey_destroy", "osprey_draft_workspace_bytes",
             "osprey_kv_append", "osprey_draft_step", "osprey_verify_workspace_bytes", "osprey_verify",
             "osprey_verify_static",
-            "osprey_probe_enable", "osprey_probe_read", "osprey_launch_count"]
+            "osprey_probe_enable", "osprey_probe_read", "osprey_launch_count", "osprey_selftest_wait_timeout"]
 
 
 def osprey_last_error() -> str:
@@ -334,3 +335,9 @@ def osprey_probe_read(ctx: Ctx, n: int) -> list:
 
 def osprey_launch_count() -> int:
     return int(_c_launch_count())
+
+
+def osprey_selftest_wait_timeout(limit_cycles: int, status: torch.Tensor, stream=None):
+    """Run the bounded-wait failure path once: status reads OSPREY_ERR_TIMEOUT afterwards."""
+    _need(status, torch.int32, (1,), "status")
+    _check(_c_selftest_wait(int(limit_cycles), _ptr(status), _stream(stream)))

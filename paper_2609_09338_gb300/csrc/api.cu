@@ -7,9 +7,11 @@
 #include <cstring>
 #include <new>
 
+#include "common.cuh"
 #include "draft.cuh"
 #include "tc.cuh"
 #include "internal.h"
+#include "tma.cuh"
 #include "osprey.h"
 
 namespace osp {
@@ -56,6 +58,28 @@ struct osprey_ctx {
 
 extern "C" const char *osprey_last_error(void) { return g_err; }
 extern "C" int64_t osprey_launch_count(void) { return g_launches.load(); }
+
+// One block waiting on an mbarrier that nothing arrives on, bounded like every
+// wait of the library; on expiry it reports the timeout and returns.
+__global__ void selftest_wait_kernel(long long limit_cycles, int32_t *status) {
+    __shared__ __align__(8) uint64_t bar;
+    if (threadIdx.x == 0) {
+        osp::mbar_init(&bar, 1);
+        osp::mbar_fence_init();
+    }
+    __syncthreads();
+    if (threadIdx.x == 0 && !osp::mbar_wait(&bar, 0, limit_cycles)) osp::set_status(status, OSPREY_ERR_TIMEOUT);
+}
+
+extern "C" int osprey_selftest_wait_timeout(int64_t limit_cycles, int32_t *dev_status, void *stream) {
+    g_err[0] = 0;
+    if (limit_cycles < 1 || limit_cycles > 2000000000LL || !dev_status)
+        return fail(OSPREY_ERR_INVALID_ARG, "limit_cycles in 1..2e9 and a status word required");
+    selftest_wait_kernel<<<1, 32, 0, (cudaStream_t)stream>>>((long long)limit_cycles, dev_status);
+    osp::count_launch();
+    const cudaError_t e = cudaGetLastError();
+    return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "self-test launch");
+}
 
 static bool is_pow2_multiple(int x, int m) { return x > 0 && x % m == 0; }
 

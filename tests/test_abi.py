@@ -78,3 +78,12 @@ def test_kv_append_and_draft_reject_null_pointers(lib):
     assert ob._c_kv_append(None, ctypes.byref(kv), 1, None, 0, None, None, None, None) == -1
     assert ob._c_draft(None, ctypes.byref(kv), 1, 1, 1, None, None, None, 1.0, None, None, None, None, None,
                        None, 0, None, None) == -1
+
+
+def test_selftest_wait_timeout_validates_on_host(lib):
+    from paper_2609_09338_gb300 import binding as ob
+    f = ob._c_selftest_wait
+    assert f(0, ctypes.c_void_p(16), None) == -1               # INVALID_ARG, before any launch
+    assert f(3_000_000_000, ctypes.c_void_p(16), None) == -1
+    assert f(1000, None, None) == -1
+    assert "limit_cycles" in ob.osprey_last_error()
