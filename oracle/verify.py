@@ -129,6 +129,33 @@ def verify(target_logits: np.ndarray, draft_logits: np.ndarray | None, draft_tok
     return {"out_tokens": out, "n_accepted": n_acc, "flags": flags, "p_x": p_x, "q_x": q_x}
 
 
+def draft_logits_from_hidden(hidden: np.ndarray, lm_head: np.ndarray, final_norm: np.ndarray,
+                             eps: float) -> np.ndarray:
+    """Draft logits of the rows a drafter chain produced, from the state it kept.
+
+    Sec. 3.3-3.4: draft token i is sampled from q_i = softmax(z^q_i / T) with
+    z^q_i = W_lm (RMSNorm(g_i) * gamma_f), g_i being the last layer's residual
+    output (before the final norm) of the row that drafted it.  hidden [B, K, d]
+    holds the g_i; lm_head [V, d] and final_norm [d] are bf16 bits or floats.
+    Returns z^q [B, K, V] in float64.
+    """
+    g = np.asarray(hidden, np.float64)
+    n = g / np.sqrt(np.mean(g * g, axis=-1, keepdims=True) + eps) * widen(final_norm)
+    return n @ widen(lm_head).T
+
+
+def verify_hidden(target_logits: np.ndarray, hidden: np.ndarray, lm_head: np.ndarray, final_norm: np.ndarray,
+                  eps: float, draft_tokens: np.ndarray, temperature: float, u_accept: np.ndarray,
+                  u_sample: np.ndarray, ratio_band: float = 1e-5, cdf_band: float = 1e-5) -> dict:
+    """The sampled rule of ``verify`` with the draft rows q_i defined by the
+    drafter's final norm and LM head applied to the kept states g_i instead of
+    stored draft logits (same outputs as ``verify``).  temperature > 0."""
+    assert temperature > 0.0, "the draft rows matter only for sampled verification"
+    zq = draft_logits_from_hidden(hidden, lm_head, final_norm, eps)
+    return verify(target_logits, zq, draft_tokens, temperature, u_accept, u_sample,
+                  ratio_band=ratio_band, cdf_band=cdf_band)
+
+
 def emission_distribution(p: np.ndarray, q: np.ndarray) -> dict:
     """The rule integrated over its uniforms, for one sequence.
 
