@@ -165,6 +165,47 @@ int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int ma
                       float *draft_qx, float *draft_stats, float *draft_logits,
                       void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
 
+/* osprey_draft_step with draft_logits NULL that also keeps, for every draft
+ * token, the state it was drafted from, for osprey_verify_hidden:
+ *   draft_hidden [B][K][d_model] float (device, 16-byte aligned): row k of
+ *          sequence b is the last layer's residual output before the final
+ *          norm (Sec. 3.4's g) of the row whose LM head drew token k; zeros
+ *          for a sequence the call skipped.
+ * Everything else as osprey_draft_step (same workspace size). */
+int osprey_draft_step_hidden(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
+                             const int32_t *n_new, const int32_t *tokens, const void *feats,
+                             float temperature, const float *u_draft, int32_t *draft_tokens,
+                             float *draft_qx, float *draft_stats, float *draft_hidden,
+                             void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
+
+/* Bytes of workspace osprey_verify_hidden needs.  0 on bad arguments. */
+size_t osprey_verify_hidden_workspace_bytes(const osprey_ctx *ctx, int B, int K);
+
+/* Sampled verification (the rule of osprey_verify, temperature > 0) without
+ * draft logits in memory.  The acceptance test at i reads the draft step's own
+ * q_i(x_i) (draft_qx); the one draft row the rule needs in full, q_r at the
+ * first rejected position r < K, is recomputed on the tensor cores from the
+ * kept state (draft_hidden row r) through ctx's final RMSNorm and LM head, and
+ * normalised with the draft step's (M, log S) of that row (draft_stats).  The
+ * draft logits, B*K*V floats, are neither written by the draft step nor read
+ * here; the LM head is read once per 80 sequences instead.
+ *   ctx: the drafter whose draft step produced the inputs (V = its vocab)
+ *   target_logits [B][K+1][V], logits_dtype OSPREY_F32 or OSPREY_BF16
+ *   draft_hidden [B][K][d_model], draft_qx [B][K], draft_stats [B][K][2]
+ *          float: as written by osprey_draft_step_hidden at the same T
+ *   draft_tokens, u_accept, u_sample, out_tokens, n_accepted, flags, probs:
+ *          as osprey_verify (probs' q column is draft_qx)
+ *   workspace: osprey_verify_hidden_workspace_bytes(ctx, B, K) bytes, zeroed
+ *          before the first call (its arrival counters return to zero)
+ * Host errors: INVALID_ARG (null pointer, T <= 0), SHAPE (the context has no
+ * tensor-core path: OSPREY_TC=0 or a device without tcgen05), CAPACITY. */
+int osprey_verify_hidden(osprey_ctx *ctx, int B, int K, int logits_dtype, const void *target_logits,
+                         const float *draft_hidden, const float *draft_qx, const float *draft_stats,
+                         const int32_t *draft_tokens, float temperature, const float *u_accept,
+                         const float *u_sample, int32_t *out_tokens, int32_t *n_accepted, uint8_t *flags,
+                         float *probs, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                         void *stream);
+
 /* Bytes of workspace osprey_verify needs.  0 on bad arguments. */
 size_t osprey_verify_workspace_bytes(int B, int K, int V);
 

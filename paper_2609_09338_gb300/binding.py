@@ -70,6 +70,13 @@ _c_kv_append = _sig("osprey_kv_append", ctypes.c_int, [_vp, ctypes.POINTER(ospre
 _c_draft = _sig("osprey_draft_step", ctypes.c_int,
                 [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32, _vp,
                  _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp])
+_c_draft_hidden = _sig("osprey_draft_step_hidden", ctypes.c_int,
+                       [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32,
+                        _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp])
+_c_verify_hidden_ws = _sig("osprey_verify_hidden_workspace_bytes", _sz, [_vp, ctypes.c_int, ctypes.c_int])
+_c_verify_hidden = _sig("osprey_verify_hidden", ctypes.c_int,
+                        [_vp, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
+                         _vp, _vp, _vp, _vp, _sz, _vp, _vp])
 _c_verify_ws = _sig("osprey_verify_workspace_bytes", _sz, [ctypes.c_int, ctypes.c_int, ctypes.c_int])
 _c_verify = _sig("osprey_verify", ctypes.c_int,
                  [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32, _vp, _vp, _vp, _vp,
@@ -83,8 +90,8 @@ _c_launch_count = _sig("osprey_launch_count", _i64, [])
 _c_selftest_wait = _sig("osprey_selftest_wait_timeout", ctypes.c_int, [_i64, _vp, _vp])
 
 EXPORTED = ["osprey_last_error", "osprey_create", "osprey_destroy", "osprey_draft_workspace_bytes",
-            "osprey_kv_append", "osprey_draft_step", "osprey_verify_workspace_bytes", "osprey_verify",
-            "osprey_verify_static",
+            "osprey_kv_append", "osprey_draft_step", "osprey_draft_step_hidden", "osprey_verify_workspace_bytes",
+            "osprey_verify", "osprey_verify_static", "osprey_verify_hidden_workspace_bytes", "osprey_verify_hidden",
             "osprey_probe_enable", "osprey_probe_read", "osprey_launch_count", "osprey_selftest_wait_timeout"]
 
 
@@ -260,6 +267,74 @@ def osprey_draft_step(ctx: Ctx, kv: KvCache, n_new: torch.Tensor, tokens: torch.
     _check(_c_draft(ctx.handle, ctypes.byref(kvs), B, K, max_new, _ptr(n_new), _ptr(tokens), _ptr(feats),
                     float(temperature), _ptr(u_draft), _ptr(draft_tokens), _ptr(draft_qx), _ptr(draft_stats),
                     _ptr(draft_logits), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+
+
+def osprey_draft_step_hidden(ctx: Ctx, kv: KvCache, n_new: torch.Tensor, tokens: torch.Tensor, feats: torch.Tensor,
+                             temperature: float, u_draft, draft_tokens: torch.Tensor, draft_qx: torch.Tensor,
+                             draft_stats: torch.Tensor, draft_hidden: torch.Tensor, workspace: torch.Tensor = None,
+                             status: torch.Tensor = None, stream=None):
+    """osprey_draft_step without draft logits, keeping the state behind every
+    draft token in draft_hidden [B, K, d] float32 (for osprey_verify_hidden)."""
+    s = ctx.shape
+    B, max_new = tokens.shape
+    K = draft_tokens.shape[1]
+    _need(n_new, torch.int32, (B,), "n_new")
+    _need(tokens, torch.int32, (B, max_new), "tokens")
+    _need(feats, torch.bfloat16, (B, max_new, s.feat_dim), "feats")
+    _need(draft_tokens, torch.int32, (B, K), "draft_tokens")
+    if u_draft is not None:
+        _need(u_draft, torch.float32, (B, K), "u_draft")
+    if draft_qx is not None:
+        _need(draft_qx, torch.float32, (B, K), "draft_qx")
+    if draft_stats is not None:
+        _need(draft_stats, torch.float32, (B, K, 2), "draft_stats")
+    _need(draft_hidden, torch.float32, (B, K, s.d_model), "draft_hidden")
+    _need(workspace, torch.uint8, None, "workspace")
+    _need(status, torch.int32, (1,), "status")
+    if kv.page_table.shape[0] != B:
+        raise ValueError("page table rows must equal the batch")
+    kvs = kv.c_struct()
+    _check(_c_draft_hidden(ctx.handle, ctypes.byref(kvs), B, K, max_new, _ptr(n_new), _ptr(tokens), _ptr(feats),
+                           float(temperature), _ptr(u_draft), _ptr(draft_tokens), _ptr(draft_qx), _ptr(draft_stats),
+                           _ptr(draft_hidden), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+
+
+def osprey_verify_hidden_workspace_bytes(ctx: Ctx, B: int, K: int) -> int:
+    return int(_c_verify_hidden_ws(ctx.handle, B, K))
+
+
+def osprey_verify_hidden(ctx: Ctx, target_logits: torch.Tensor, draft_hidden: torch.Tensor, draft_qx: torch.Tensor,
+                         draft_stats: torch.Tensor, draft_tokens: torch.Tensor, temperature: float,
+                         u_accept: torch.Tensor, u_sample: torch.Tensor, out_tokens: torch.Tensor,
+                         n_accepted: torch.Tensor, flags: torch.Tensor, probs=None, workspace: torch.Tensor = None,
+                         status: torch.Tensor = None, stream=None):
+    """Sampled verification without draft logits: the decision row's draft
+    logits are recomputed from draft_hidden by ctx's LM head."""
+    B, K1, V = target_logits.shape
+    K = K1 - 1
+    dt = {torch.float32: OSPREY_F32, torch.bfloat16: OSPREY_BF16}.get(target_logits.dtype)
+    if dt is None:
+        raise TypeError("logits must be float32 or bfloat16")
+    if V != ctx.shape.vocab:
+        raise ValueError(f"target vocab {V} differs from the drafter's {ctx.shape.vocab}")
+    _need(target_logits, target_logits.dtype, (B, K + 1, V), "target_logits")
+    _need(draft_hidden, torch.float32, (B, K, ctx.shape.d_model), "draft_hidden")
+    _need(draft_qx, torch.float32, (B, K), "draft_qx")
+    _need(draft_stats, torch.float32, (B, K, 2), "draft_stats")
+    _need(draft_tokens, torch.int32, (B, K), "draft_tokens")
+    _need(u_accept, torch.float32, (B, K), "u_accept")
+    _need(u_sample, torch.float32, (B, K + 1), "u_sample")
+    _need(out_tokens, torch.int32, (B, K + 1), "out_tokens")
+    _need(n_accepted, torch.int32, (B,), "n_accepted")
+    _need(flags, torch.uint8, (B, K + 1), "flags")
+    if probs is not None:
+        _need(probs, torch.float32, (B, K, 2), "probs")
+    _need(workspace, torch.uint8, None, "workspace")
+    _need(status, torch.int32, (1,), "status")
+    _check(_c_verify_hidden(ctx.handle, B, K, dt, _ptr(target_logits), _ptr(draft_hidden), _ptr(draft_qx),
+                            _ptr(draft_stats), _ptr(draft_tokens), float(temperature), _ptr(u_accept),
+                            _ptr(u_sample), _ptr(out_tokens), _ptr(n_accepted), _ptr(flags), _ptr(probs),
+                            _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
 
 
 def osprey_verify_workspace_bytes(B: int, K: int, V: int) -> int:

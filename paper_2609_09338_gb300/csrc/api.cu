@@ -351,12 +351,11 @@ extern "C" int osprey_kv_append(const osprey_ctx *ctx, const osprey_kv *kv, int 
 }
 
 // ------------------------------------------------------------------ draft step
-extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
-                                 const int32_t *n_new, const int32_t *tokens, const void *feats,
-                                 float temperature, const float *u_draft, int32_t *draft_tokens,
-                                 float *draft_qx, float *draft_stats, float *draft_logits,
-                                 void *workspace, size_t workspace_bytes, int32_t *dev_status,
-                                 void *stream) {
+static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
+                           const int32_t *n_new, const int32_t *tokens, const void *feats, float temperature,
+                           const float *u_draft, int32_t *draft_tokens, float *draft_qx, float *draft_stats,
+                           float *draft_logits, float *draft_hidden, void *workspace, size_t workspace_bytes,
+                           int32_t *dev_status, void *stream) {
     g_err[0] = 0;
     if (!ctx || !kv) return fail(OSPREY_ERR_INVALID_ARG, "null context or kv");
     if (B == 0) return OSPREY_OK;
@@ -369,8 +368,8 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
         return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
     if (temperature > 0.f && !u_draft) return fail(OSPREY_ERR_INVALID_ARG, "u_draft is required when temperature > 0");
     if (kv->n_pages < 1) return fail(OSPREY_ERR_INVALID_ARG, "empty page pool");
-    if (((uintptr_t)feats | (uintptr_t)workspace) % 16)
-        return fail(OSPREY_ERR_INVALID_ARG, "feats and workspace must be 16-byte aligned");
+    if (((uintptr_t)feats | (uintptr_t)workspace | (uintptr_t)draft_hidden) % 16)
+        return fail(OSPREY_ERR_INVALID_ARG, "feats, workspace and draft_hidden must be 16-byte aligned");
     DraftWs ws{};
     const size_t need = draft_layout(ctx, B, K, max_new, kv->max_pages_per_seq, &ws, workspace);
     if (workspace_bytes < need)
@@ -636,6 +635,10 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
             g.xin = ws.ffn_h;
             if ((rc = gemv(G_DOWN, "down launch")) != OSPREY_OK) return rc;
         }
+        if (draft_hidden &&
+            (e = launch_keep_hidden(x, ext, B, K, step, max_new, D.d, ws.seq_valid, ws.seq_nnew, draft_hidden, s)) !=
+                cudaSuccess)
+            return cuda_fail(e, "keep-hidden launch");
         const bool probe = step < ctx->n_probe;
         if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
@@ -726,6 +729,30 @@ extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, in
     return OSPREY_OK;
 }
 
+extern "C" int osprey_draft_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
+                                 const int32_t *n_new, const int32_t *tokens, const void *feats,
+                                 float temperature, const float *u_draft, int32_t *draft_tokens,
+                                 float *draft_qx, float *draft_stats, float *draft_logits,
+                                 void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                 void *stream) {
+    return draft_step_impl(ctx, kv, B, K, max_new, n_new, tokens, feats, temperature, u_draft, draft_tokens, draft_qx,
+                           draft_stats, draft_logits, nullptr, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" int osprey_draft_step_hidden(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
+                                        const int32_t *n_new, const int32_t *tokens, const void *feats,
+                                        float temperature, const float *u_draft, int32_t *draft_tokens,
+                                        float *draft_qx, float *draft_stats, float *draft_hidden,
+                                        void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                        void *stream) {
+    if (!draft_hidden) {
+        g_err[0] = 0;
+        return fail(OSPREY_ERR_INVALID_ARG, "draft_hidden is required");
+    }
+    return draft_step_impl(ctx, kv, B, K, max_new, n_new, tokens, feats, temperature, u_draft, draft_tokens, draft_qx,
+                           draft_stats, nullptr, draft_hidden, workspace, workspace_bytes, dev_status, stream);
+}
+
 // ------------------------------------------------------------------ verify
 extern "C" size_t osprey_verify_workspace_bytes(int B, int K, int V) {
     if (B < 1 || K < 1 || K > 15 || V < 1) return 0;
@@ -773,4 +800,149 @@ extern "C" int osprey_verify(int B, int K, int V, int logits_dtype, const void *
     a.status = dev_status;
     cudaError_t e = launch_verify(a, (cudaStream_t)stream);
     return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "verify launch");
+}
+
+// ------------------------------------------------------------------ logits-free verify
+// Workspace: the verify layout (counters, partials, decisions, chunk sums), then
+// for one group of up to TC_MAX_ROWS sequences the gathered kept states
+// [rows][d] float, their operand planes [TC_PLANES][npad][d] bf16, the
+// recomputed decision-row logits [rows][V] float and the split-K partials of
+// that GEMM (the draft step's LM-head split, so the rows come out the same).
+struct HiddenWs {
+    float *rows;
+    uint16_t *planes;
+    float *z;
+    float *part;
+    long long part_cap;
+    int group, npad;
+};
+
+static size_t verify_hidden_layout(const osprey_ctx *ctx, int B, int K, VerifyArgs *a, void *base, HiddenWs *hw) {
+    const Dims &D = ctx->dim;
+    size_t off = align256(verify_workspace_layout(B, K, D.V, a, base));
+    const int group = B < TC_MAX_ROWS ? B : TC_MAX_ROWS;
+    const int npad = (group + 15) / 16 * 16;
+    const size_t o_r = off;
+    off = align256(off + 4ull * group * D.d);
+    const size_t o_p = off;
+    off = align256(off + 2ull * TC_PLANES * npad * D.d);
+    const size_t o_z = off;
+    off = align256(off + 4ull * group * D.V);
+    const int ns = tc_nsplit(D.V, D.d, ctx->sms);
+    const long long part = ns > 1 ? (long long)ns * group * D.V : 0;
+    const size_t o_t = off;
+    off = align256(off + 4ull * part);
+    if (hw && base) {
+        char *p = (char *)base;
+        hw->rows = (float *)(p + o_r);
+        hw->planes = (uint16_t *)(p + o_p);
+        hw->z = (float *)(p + o_z);
+        hw->part = part ? (float *)(p + o_t) : nullptr;
+        hw->part_cap = part;
+        hw->group = group;
+        hw->npad = npad;
+    }
+    return off;
+}
+
+extern "C" size_t osprey_verify_hidden_workspace_bytes(const osprey_ctx *ctx, int B, int K) {
+    if (!ctx || B < 1 || K < 1 || K > 15) return 0;
+    return verify_hidden_layout(ctx, B, K, nullptr, nullptr, nullptr);
+}
+
+extern "C" int osprey_verify_hidden(osprey_ctx *ctx, int B, int K, int logits_dtype, const void *target_logits,
+                                    const float *draft_hidden, const float *draft_qx, const float *draft_stats,
+                                    const int32_t *draft_tokens, float temperature, const float *u_accept,
+                                    const float *u_sample, int32_t *out_tokens, int32_t *n_accepted, uint8_t *flags,
+                                    float *probs, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                                    void *stream) {
+    g_err[0] = 0;
+    if (!ctx) return fail(OSPREY_ERR_INVALID_ARG, "null context");
+    if (B == 0) return OSPREY_OK;
+    const Dims &D = ctx->dim;
+    const int V = D.V;
+    if (B < 0 || K < 1 || K > 15) return fail(OSPREY_ERR_INVALID_ARG, "B >= 0 and K in 1..15 required");
+    if (logits_dtype != OSPREY_F32 && logits_dtype != OSPREY_BF16)
+        return fail(OSPREY_ERR_DTYPE, "logits_dtype must be OSPREY_F32 or OSPREY_BF16");
+    if (!(temperature > 0.f) || !std::isfinite(temperature))
+        return fail(OSPREY_ERR_INVALID_ARG,
+                    "temperature must be finite and > 0 (greedy verification reads no draft rows: osprey_verify)");
+    if (!target_logits || !draft_hidden || !draft_qx || !draft_stats || !draft_tokens || !u_accept || !u_sample ||
+        !out_tokens || !n_accepted || !flags || !workspace)
+        return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
+    if ((uintptr_t)workspace % 16) return fail(OSPREY_ERR_INVALID_ARG, "workspace must be 16-byte aligned");
+    if (!ctx->tc)
+        return fail(OSPREY_ERR_SHAPE, "the decision rows are recomputed on the tensor cores; this context has no "
+                                      "tensor-core path (OSPREY_TC=0 or no tcgen05)");
+    if ((long long)V * (K + 1) * B > (1LL << 40)) return fail(OSPREY_ERR_SHAPE, "logits too large");
+    if ((long long)((V + 8191) / 8192) * (K + 1) * B >= (1LL << 31))
+        return fail(OSPREY_ERR_SHAPE, "too many (sequence, row, chunk) blocks");
+    VerifyArgs a{};
+    HiddenWs hw{};
+    const size_t need = verify_hidden_layout(ctx, B, K, &a, workspace, &hw);
+    if (workspace_bytes < need)
+        return fail(OSPREY_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
+    a.B = B;
+    a.K = K;
+    a.V = V;
+    a.dtype = logits_dtype;
+    a.temperature = temperature;
+    a.target = target_logits;
+    a.draft = nullptr;
+    a.tokens = draft_tokens;
+    a.u_accept = u_accept;
+    a.u_sample = u_sample;
+    a.out_tokens = out_tokens;
+    a.n_accepted = n_accepted;
+    a.flags = flags;
+    a.probs = probs;
+    a.status = dev_status;
+    a.qx_in = draft_qx;
+    a.stats_in = draft_stats;
+    a.zrec = hw.z;
+    cudaStream_t s = (cudaStream_t)stream;
+    cudaError_t e;
+    // 1. target row statistics, the acceptance chain and the decision row r
+    if ((e = launch_verify_hidden_stats(a, s)) != cudaSuccess) return cuda_fail(e, "verify launch");
+    for (int b0 = 0; b0 < B; b0 += hw.group) {
+        const int n = B - b0 < hw.group ? B - b0 : hw.group;
+        const int npad = (n + 15) / 16 * 16;
+        // 2. the kept state of each decision row -> final RMSNorm -> bf16 planes
+        if ((e = launch_decision_rows(a.dec, draft_hidden, K, D.d, b0, n, hw.rows, s)) != cudaSuccess)
+            return cuda_fail(e, "decision-row launch");
+        PlaneArgs pl{};
+        pl.src = hw.rows;
+        pl.gain = (const uint16_t *)ctx->w.final_norm;
+        pl.eps = D.eps;
+        pl.d = D.d;
+        pl.R = n;
+        pl.npad = npad;
+        pl.ld = D.d;
+        pl.col0 = 0;
+        pl.dst = hw.planes;
+        pl.max_new = 1;
+        pl.rows_per_seq = 1;
+        if ((e = launch_planes(pl, s)) != cudaSuccess) return cuda_fail(e, "decision-row operand launch");
+        // 3. their draft logits on the tensor cores (the draft step's LM head GEMM)
+        CUtensorMap xm;
+        if (!tc_encode_operand(&xm, hw.planes, TC_PLANES, npad, D.d))
+            return fail(OSPREY_ERR_INVALID_ARG, "decision-row tensor map encoding failed");
+        TcArgs ta{};
+        ta.epi = TC_STORE;
+        ta.R = n;
+        ta.npad = npad;
+        ta.K = D.d;
+        ta.nout = V;
+        ta.planes = TC_PLANES;
+        ta.y = hw.z;
+        ta.x = hw.z;
+        ta.ldy = V;
+        ta.status = dev_status;
+        ta.part = hw.part;
+        ta.part_cap = hw.part_cap;
+        if ((e = launch_tc(ta, ctx->tm_lm, xm, ctx->sms, s)) != cudaSuccess) return cuda_fail(e, "decision-row lm head");
+        // 4. the emitted token of each sequence of the group
+        if ((e = launch_verify_hidden_sample(a, b0, n, s)) != cudaSuccess) return cuda_fail(e, "verify sample launch");
+    }
+    return OSPREY_OK;
 }

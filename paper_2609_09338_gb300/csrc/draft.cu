@@ -1171,6 +1171,23 @@ cudaError_t launch_lm(const LmArgs &a, int rg, int blocks, cudaStream_t s) {
     return cudaGetLastError();
 }
 
+__global__ void __launch_bounds__(256) keep_hidden_kernel(const float *x, int ext, int K, int step, int max_new,
+                                                          int d, const int *valid, const int *nnew, float *hidden) {
+    const int b = blockIdx.x;
+    const bool ok = valid[b] != 0;   // then 1 <= nnew[b] <= max_new
+    const float *src = x + (size_t)(ok ? (ext ? b * max_new + nnew[b] - 1 : b) : 0) * d;
+    float *dst = hidden + ((size_t)b * K + step) * d;
+    for (int k = threadIdx.x * 4; k < d; k += blockDim.x * 4)   // d is a multiple of 256
+        *(float4 *)(dst + k) = ok ? *(const float4 *)(src + k) : make_float4(0.f, 0.f, 0.f, 0.f);
+}
+
+cudaError_t launch_keep_hidden(const float *x, bool ext, int B, int K, int step, int max_new, int d,
+                               const int *valid, const int *nnew, float *hidden, cudaStream_t s) {
+    keep_hidden_kernel<<<B, 256, 0, s>>>(x, ext ? 1 : 0, K, step, max_new, d, valid, nnew, hidden);
+    count_launch();
+    return cudaGetLastError();
+}
+
 cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s) {
     prepare_kernel<<<a.B, 128, 0, s>>>(a);
     count_launch();

@@ -189,6 +189,11 @@ cudaError_t launch_stream(GemvMode mode, const StreamArgs &a, int rg, cudaStream
 cudaError_t stream_set_attributes();
 
 cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s);
+// hidden[b][step] <- the last layer's output row that feeds draft token `step`
+// of sequence b (extend step: row b*max_new + n_new[b] - 1; chain: row b);
+// zeros for a sequence the call skipped
+cudaError_t launch_keep_hidden(const float *x, bool ext, int B, int K, int step, int max_new, int d,
+                               const int *valid, const int *nnew, float *hidden, cudaStream_t s);
 cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaStream_t s);
 cudaError_t launch_attn(const AttnArgs &a, cudaStream_t s);
 // Cluster size (16 or 8) the on-chip-merge attention can run with on the

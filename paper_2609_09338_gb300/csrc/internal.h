@@ -47,11 +47,24 @@ struct VerifyArgs {
     void *rowstat;  // [B][K+1] float4 row summaries
     int nch3;
     size_t counter_bytes;   // ticket1, ticket2 and trow are one block from ticket1 on
+    // logits-free form: q_i(x_i) [B][K] and (M, log S) [B][K][2] from the draft
+    // step; the decision rows' draft logits of sequences b0.. are rows of zrec [.][V]
+    const float *qx_in, *stats_in;
+    const float *zrec;
+    int b0;
 };
 cudaError_t launch_verify_stream(const VerifyArgs &a, int sms, cudaStream_t s);
 bool verify_stream_ok(const VerifyArgs &a);
 size_t verify_workspace_layout(int B, int K, int V, VerifyArgs *a, void *base);
 cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s);
+// logits-free form: target statistics and the decision for every sequence, then
+// per group of n sequences from b0 (after zrec holds their decision rows) the draw
+cudaError_t launch_verify_hidden_stats(const VerifyArgs &a, cudaStream_t s);
+cudaError_t launch_verify_hidden_sample(const VerifyArgs &a, int b0, int n, cudaStream_t s);
+// the kept state of each sequence's decision row r < K (zeros otherwise) as
+// rows 0..n-1 of dst [n][d], for the sequences b0..b0+n-1
+cudaError_t launch_decision_rows(const void *dec, const float *hidden, int K, int d, int b0, int n, float *dst,
+                                 cudaStream_t s);
 
 // ---------------------------------------------------------------- kv append
 struct KvAppendArgs {

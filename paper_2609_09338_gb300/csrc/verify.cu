@@ -11,6 +11,10 @@
 //   re-reads only row r and sums the weights max(0, p_r - q_r) (or p_K for the
 //   bonus) per chunk; the last block picks the chunk holding u * S and scans it
 //   in id order for the token.
+// Logits-free form (HIDDEN): no draft rows in memory.  verify_stats reads the
+//   target rows only and the decision takes q_i(x_i) from the draft step;
+//   verify_sample reads the decision row's draft logits from `zrec`, recomputed
+//   for a group of sequences by the tensor-core LM head (api.cu).
 #include <float.h>
 #include <math.h>
 
@@ -104,7 +108,7 @@ __device__ __forceinline__ float ld_logit(const void *base, int dtype, size_t id
 
 // The last block of sequence b: combine the partials of all K+1 rows, run the
 // acceptance chain and write everything but the token emitted at r.
-template <bool GREEDY>
+template <bool GREEDY, bool HIDDEN>
 __device__ void decide(const VerifyArgs &a, int b) {
     __shared__ float sMp[16], sSp[16], sMq[16], sSq[16];
     __shared__ int sAm[16];
@@ -161,7 +165,8 @@ __device__ void decide(const VerifyArgs &a, int b) {
         const float invT = 1.f / a.temperature;
         const size_t rowp = ((size_t)b * (K + 1) + lane) * V, rowq = ((size_t)b * K + lane) * V;
         const float px = expf(ld_logit(a.target, a.dtype, rowp + xi) * invT - sMp[lane]) / sSp[lane];
-        const float qx = expf(ld_logit(a.draft, a.dtype, rowq + xi) * invT - sMq[lane]) / sSq[lane];
+        const float qx = HIDDEN ? a.qx_in[(size_t)b * K + lane]
+                                : expf(ld_logit(a.draft, a.dtype, rowq + xi) * invT - sMq[lane]) / sSq[lane];
         if (a.probs) {
             a.probs[((size_t)b * K + lane) * 2 + 0] = px;
             a.probs[((size_t)b * K + lane) * 2 + 1] = qx;
@@ -178,13 +183,18 @@ __device__ void decide(const VerifyArgs &a, int b) {
         if (!GREEDY) {
             dec->r = r;
             dec->Mp = sMp[r]; dec->Sp = sSp[r];
-            dec->Mq = r < K ? sMq[r] : 0.f;
-            dec->Sq = r < K ? sSq[r] : 1.f;
+            if (HIDDEN) {   // (M, log S) of the draft row, from the draft step
+                dec->Mq = r < K ? a.stats_in[((size_t)b * K + r) * 2 + 0] : 0.f;
+                dec->Sq = r < K ? expf(a.stats_in[((size_t)b * K + r) * 2 + 1]) : 1.f;
+            } else {
+                dec->Mq = r < K ? sMq[r] : 0.f;
+                dec->Sq = r < K ? sSq[r] : 1.f;
+            }
         }
     }
 }
 
-template <typename T, bool VEC, bool GREEDY>
+template <typename T, bool VEC, bool GREEDY, bool HIDDEN = false>
 __global__ void __launch_bounds__(VT) verify_stats(VerifyArgs a) {
     __shared__ MS shm[VT / 32];
     __shared__ AM sha[VT / 32];
@@ -208,14 +218,14 @@ __global__ void __launch_bounds__(VT) verify_stats(VerifyArgs a) {
         const float invT = 1.f / a.temperature;
         float f[VPER], g[VPER];
         load_chunk<T, VEC>(zp, start, V, f);
-        const bool has_q = i < K;
+        const bool has_q = !HIDDEN && i < K;
         if (has_q) load_chunk<T, VEC>((const T *)a.draft + ((size_t)b * K + i) * V, start, V, g);
         MS p = block_ms(thread_ms(f, invT), shm);
         MS q{-INFINITY, 0.f};
         if (has_q) q = block_ms(thread_ms(g, invT), shm);
         if (threadIdx.x == 0) *part = make_float4(p.m, p.s, q.m, q.s);
     }
-    if (arrive_last(a.ticket1 + b, a.nch * (K + 1))) decide<GREEDY>(a, b);
+    if (arrive_last(a.ticket1 + b, a.nch * (K + 1))) decide<GREEDY, HIDDEN>(a, b);
 }
 
 // Weight of id e in the decision row's draw: max(0, p - q) (residual) or p.
@@ -227,14 +237,16 @@ __device__ __forceinline__ float sample_weight(float zp, float zq, const Decisio
     return fmaxf(0.f, p - q);
 }
 
-template <typename T, bool VEC>
+// HIDDEN: blocks cover the group of sequences b0 .. b0 + n - 1 and the draft
+// row r of sequence b is row b - b0 of zrec (float32 logits, TQ = float).
+template <typename T, bool VEC, typename TQ = T, bool HIDDEN = false>
 __global__ void __launch_bounds__(VT) verify_sample(VerifyArgs a) {
     __shared__ float sh[33];
     __shared__ float2 shs[VT / 32];
     __shared__ int s_chunk, s_tok, s_flag;
     __shared__ float s_t, s_before;
     const int K = a.K, V = a.V, nch = a.nch;
-    const int c = (int)(blockIdx.x % nch), b = (int)(blockIdx.x / nch);
+    const int c = (int)(blockIdx.x % nch), b = (HIDDEN ? a.b0 : 0) + (int)(blockIdx.x / nch);
     const Decision d = ((const Decision *)a.dec)[b];   // written by verify_stats
     const float invT = 1.f / a.temperature;
     // a decision outside [-1, K] means the workspace was not produced by
@@ -244,13 +256,14 @@ __global__ void __launch_bounds__(VT) verify_sample(VerifyArgs a) {
     const int r = valid ? d.r : 0;
     const bool residual = r < K;
     const T *zp = (const T *)a.target + ((size_t)b * (K + 1) + r) * V;
-    const T *zq = residual ? (const T *)a.draft + ((size_t)b * K + r) * V : zp;
+    const TQ *zq = HIDDEN ? (residual ? (const TQ *)a.zrec + (size_t)(b - a.b0) * V : nullptr)
+                          : (residual ? (const TQ *)a.draft + ((size_t)b * K + r) * V : (const TQ *)zp);
     const int start = c * VCHUNK;
     float2 *csum = (float2 *)a.csum + (size_t)b * nch;
     if (valid) {
         float f[VPER], g[VPER];
         load_chunk<T, VEC>(zp, start, V, f);
-        if (residual) load_chunk<T, VEC>(zq, start, V, g);
+        if (residual) load_chunk<TQ, VEC>(zq, start, V, g);
         float sw = 0.f, sp = 0.f;
 #pragma unroll
         for (int j = 0; j < VPER; ++j) {
@@ -413,6 +426,59 @@ static cudaError_t launch_t(const VerifyArgs &a, cudaStream_t s) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     verify_sample<T, VEC><<<(unsigned)a.nch * a.B, VT, 0, s>>>(a);
+    count_launch();
+    return cudaGetLastError();
+}
+
+// ---------------------------------------------------------------- logits-free form
+static bool hidden_vec(const VerifyArgs &a) {
+    // both element types vectorised: 8 bf16 or 2 x 4 float per 16 bytes
+    return a.V % 8 == 0 && ((uintptr_t)a.target % 16) == 0 && ((uintptr_t)a.zrec % 16) == 0;
+}
+
+cudaError_t launch_verify_hidden_stats(const VerifyArgs &a, cudaStream_t s) {
+    const unsigned g1 = (unsigned)a.nch * (a.K + 1) * a.B;
+    const bool vec = hidden_vec(a);
+    if (a.dtype == OSPREY_F32) {
+        if (vec) verify_stats<float, true, false, true><<<g1, VT, 0, s>>>(a);
+        else verify_stats<float, false, false, true><<<g1, VT, 0, s>>>(a);
+    } else {
+        if (vec) verify_stats<uint16_t, true, false, true><<<g1, VT, 0, s>>>(a);
+        else verify_stats<uint16_t, false, false, true><<<g1, VT, 0, s>>>(a);
+    }
+    count_launch();
+    return cudaGetLastError();
+}
+
+cudaError_t launch_verify_hidden_sample(const VerifyArgs &a_in, int b0, int n, cudaStream_t s) {
+    VerifyArgs a = a_in;
+    a.b0 = b0;
+    const unsigned g2 = (unsigned)a.nch * n;
+    const bool vec = hidden_vec(a);
+    if (a.dtype == OSPREY_F32) {
+        if (vec) verify_sample<float, true, float, true><<<g2, VT, 0, s>>>(a);
+        else verify_sample<float, false, float, true><<<g2, VT, 0, s>>>(a);
+    } else {
+        if (vec) verify_sample<uint16_t, true, float, true><<<g2, VT, 0, s>>>(a);
+        else verify_sample<uint16_t, false, float, true><<<g2, VT, 0, s>>>(a);
+    }
+    count_launch();
+    return cudaGetLastError();
+}
+
+__global__ void __launch_bounds__(256) decision_rows_kernel(const Decision *dec, const float *hidden, int K, int d,
+                                                            int b0, float *dst) {
+    const int j = blockIdx.x, b = b0 + j;
+    const int r = dec[b].r;   // written by verify_stats
+    const bool act = r >= 0 && r < K;
+    const float *src = hidden + ((size_t)b * K + (act ? r : 0)) * d;
+    float *out = dst + (size_t)j * d;
+    for (int k = threadIdx.x; k < d; k += blockDim.x) out[k] = act ? src[k] : 0.f;
+}
+
+cudaError_t launch_decision_rows(const void *dec, const float *hidden, int K, int d, int b0, int n, float *dst,
+                                 cudaStream_t s) {
+    decision_rows_kernel<<<n, 256, 0, s>>>((const Decision *)dec, hidden, K, d, b0, dst);
     count_launch();
     return cudaGetLastError();
 }

@@ -45,6 +45,12 @@ class DraftSession:
                              out["draft_qx"], out["draft_stats"], out["draft_logits"], self.workspace,
                              self.status, stream)
 
+    def draft_hidden(self, n_new, tokens, feats, temperature: float, u_draft, out: dict, hidden, stream=None):
+        """The draft call without logits, keeping each draft token's state in hidden [B, K, d]."""
+        ob.osprey_draft_step_hidden(self.ctx, self.kv, n_new, tokens, feats, temperature, u_draft,
+                                    out["draft_tokens"], out["draft_qx"], out["draft_stats"], hidden, self.workspace,
+                                    self.status, stream)
+
 
 class VerifyBuffers:
     def __init__(self, B: int, K: int, V: int, device: str = "cuda"):
@@ -58,3 +64,18 @@ class VerifyBuffers:
     def run(self, target, draft, tokens, temperature, u_accept, u_sample, stream=None):
         ob.osprey_verify(target, draft, tokens, temperature, u_accept, u_sample, self.out_tokens,
                          self.n_accepted, self.flags, self.probs, self.workspace, self.status, stream)
+
+
+class VerifyHiddenBuffers(VerifyBuffers):
+    """Outputs and workspace of the logits-free verify for one drafter context."""
+
+    def __init__(self, ctx: "ob.Ctx", B: int, K: int, device: str = "cuda"):
+        super().__init__(B, K, ctx.shape.vocab, device)
+        self.ctx = ctx
+        self.workspace = torch.zeros(ob.osprey_verify_hidden_workspace_bytes(ctx, B, K), dtype=torch.uint8,
+                                     device=device)
+
+    def run_hidden(self, target, hidden, qx, stats, tokens, temperature, u_accept, u_sample, stream=None):
+        ob.osprey_verify_hidden(self.ctx, target, hidden, qx, stats, tokens, temperature, u_accept, u_sample,
+                                self.out_tokens, self.n_accepted, self.flags, self.probs, self.workspace,
+                                self.status, stream)

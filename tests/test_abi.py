@@ -87,3 +87,19 @@ def test_selftest_wait_timeout_validates_on_host(lib):
     assert f(3_000_000_000, ctypes.c_void_p(16), None) == -1
     assert f(1000, None, None) == -1
     assert "limit_cycles" in ob.osprey_last_error()
+
+
+def test_logits_free_entry_points_validate_on_host(lib):
+    from paper_2609_09338_gb300 import binding as ob
+    kv = ob.osprey_kv()
+    p = ctypes.c_void_p(256)
+    # draft_step_hidden without the hidden buffer, and with a null context
+    assert ob._c_draft_hidden(p, ctypes.byref(kv), 1, 1, 1, p, p, p, 1.0, p, p, p, p, None, p, 1 << 20, None,
+                              None) == -1
+    assert "draft_hidden" in ob.osprey_last_error()
+    assert ob._c_draft_hidden(None, ctypes.byref(kv), 1, 1, 1, p, p, p, 1.0, p, p, p, p, p, p, 1 << 20, None,
+                              None) == -1
+    # verify_hidden: null context; no workspace size without a context
+    f = ob._c_verify_hidden
+    assert f(None, 1, 2, 0, p, p, p, p, p, 1.0, p, p, p, p, p, None, p, 1 << 20, None, None) == -1
+    assert ob._c_verify_hidden_ws(None, 1, 2) == 0
