@@ -56,6 +56,8 @@ def parse():
     p.add_argument("--temperature", type=float, default=None, help="override the workload's temperature")
     p.add_argument("--verify-sweep", action="store_true",
                    help="time verify alone over batch x K at V=200064 (fp32 and bf16 logits)")
+    p.add_argument("--verify-hidden", action="store_true",
+                   help="compare draft (logits written) + verify against draft (states kept) + logits-free verify")
     return p.parse_args()
 
 
@@ -280,12 +282,97 @@ def verify_sweep(args):
                       "verify_sweep": points}))
 
 
+def verify_hidden_compare(args):
+    """One sampled draft+verify step two ways on the workload's drafter: the draft
+    step writes its logits [B, K, V] and osprey_verify reads them, or the draft
+    step keeps each token's state [B, K, d] and osprey_verify_hidden recomputes
+    only the decision rows.  Target logits are the workload's synthetic rows."""
+    import torch
+    import __graft_entry__
+    __graft_entry__.build()
+    from paper_2609_09338_gb300 import binding as ob
+    from paper_2609_09338_gb300.session import DraftSession, VerifyBuffers, VerifyHiddenBuffers
+    torch.cuda.set_device(0)
+    wl = WORKLOADS[args.workload]
+    if args.temperature is not None:
+        wl = wl.with_(temperature=args.temperature)
+    if wl.temperature <= 0:
+        raise SystemExit("--verify-hidden needs a sampled workload (temperature > 0)")
+    sh, B, K, T = wl.shape, wl.batch, wl.K, wl.temperature
+    ctx, w, kv, di, vi = make_inputs(wl)
+    dev = "cuda"
+    T_ = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
+    target = T_(vi["target_logits"]) if wl.logits_dtype == "f32" else \
+        ob.to_device_bf16(syn.bf16_bits(vi["target_logits"]))
+    d_in = (T_(di["n_new"]), T_(di["tokens"]), ob.to_device_bf16(di["feats"]), T, T_(di["u_draft"]))
+    u_acc, u_smp = T_(vi["u_accept"]), T_(vi["u_sample"])
+    flush_w = torch.empty(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    flush_r = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device=dev)
+    res = {}
+    for mode in ("logits", "hidden"):
+        sess = DraftSession(sh, w, kv["page_table"], kv["n_pages"], K, wl.n_new)
+        sess.append(ctx, kv["k_rows"], kv["v_rows"])
+        torch.cuda.synchronize()
+        seq0 = sess.kv.seq_len.clone()
+        out = sess.draft_buffers(with_logits=mode == "logits")
+        hidden = torch.zeros((B, K, sh.d_model), dtype=torch.float32, device=dev)
+        vb = VerifyBuffers(B, K, sh.vocab) if mode == "logits" else VerifyHiddenBuffers(sess.ctx, B, K)
+        # osprey_verify reads both rows in one dtype and the draft step writes float32
+        tgt = target if mode == "hidden" or wl.logits_dtype == "f32" else target.float()
+
+        def step():
+            sess.kv.seq_len.copy_(seq0)
+            if mode == "logits":
+                sess.draft(*d_in, out)
+                vb.run(tgt, out["draft_logits"], out["draft_tokens"], T, u_acc, u_smp)
+            else:
+                sess.draft_hidden(*d_in, out, hidden)
+                vb.run_hidden(tgt, hidden, out["draft_qx"], out["draft_stats"], out["draft_tokens"], T, u_acc,
+                              u_smp)
+        st = torch.cuda.Stream()
+        st.wait_stream(torch.cuda.current_stream())
+        with torch.cuda.stream(st):
+            step()
+        torch.cuda.synchronize()
+        assert int(sess.status.item()) == 0 and int(vb.status.item()) == 0
+        g = torch.cuda.CUDAGraph()
+        n0 = ob.osprey_launch_count()
+        with torch.cuda.graph(g, stream=st):
+            step()
+        launches = ob.osprey_launch_count() - n0
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps + max(args.warmup, 3))]
+        with torch.cuda.stream(st):
+            for s_, e_ in ev:
+                flush_w.zero_()
+                flush_r.sum()
+                s_.record(st)
+                g.replay()
+                e_.record(st)
+        torch.cuda.synchronize()
+        assert int(sess.status.item()) == 0 and int(vb.status.item()) == 0
+        ev = ev[max(args.warmup, 3):]
+        res[mode] = {"ms_per_step": sum(s_.elapsed_time(e_) for s_, e_ in ev) / len(ev),
+                     "launches_per_step": launches,
+                     "mean_accepted": float(vb.n_accepted.float().mean().item())}
+        del sess, vb, g
+        torch.cuda.empty_cache()
+    s_ = 4 if wl.logits_dtype == "f32" else 2
+    print(json.dumps({"metric": "draft+verify ms per step, draft logits vs kept states",
+                      "workload": wl.name, "temperature": T, "logits": wl.logits_dtype, "steps": args.steps,
+                      "l2": "flushed before every step", **res,
+                      "draft_logits_bytes": B * K * sh.vocab * 4,
+                      "decision_row_lm_bytes": -(-B // 80) * sh.vocab * sh.d_model * 2 + B * sh.vocab * s_}))
+
+
 def main():
     args = parse()
     if args.impl == "reference":
         return run_reference(args)
     if args.verify_sweep:
         return verify_sweep(args)
+    if args.verify_hidden:
+        return verify_hidden_compare(args)
     import torch
     import torch.distributed as dist
     world = int(os.environ.get("WORLD_SIZE", "1"))
