@@ -49,6 +49,7 @@ struct osprey_ctx {
     int attn_cs;    // cluster size of the attention kernel (0: split partials in global memory)
     bool tc;        // batched rows (3..80) run their projections on tcgen05
     bool fused_mlp; // batch-1 chain steps run O-proj, gate/up and down as one launch
+    bool fused_layer; // batch-1 chain steps run each whole layer as one launch
     CUtensorMap tm_c, tm_lm, tm_qkv[OSPREY_MAX_LAYERS], tm_o[OSPREY_MAX_LAYERS], tm_gate[OSPREY_MAX_LAYERS],
         tm_up[OSPREY_MAX_LAYERS], tm_down[OSPREY_MAX_LAYERS];
     double inv_freq[64];
@@ -152,6 +153,10 @@ extern "C" int osprey_create(const osprey_config *cfg, const osprey_weights *w, 
         // step as one launch with grid barriers (not yet the default)
         const char *menv = std::getenv("OSPREY_FUSED_MLP");
         ctx->fused_mlp = menv && menv[0] == '1' && mlp_fused_supported(D, ctx->sms);
+        // OSPREY_FUSED_LAYER=1 runs each whole layer of a batch-1 chain step as
+        // one launch with grid barriers (not yet the default)
+        const char *lenv = std::getenv("OSPREY_FUSED_LAYER");
+        ctx->fused_layer = lenv && lenv[0] == '1' && layer_fused_supported(D, ctx->sms);
         cudaGetLastError();
     }
     if (e != cudaSuccess) {
@@ -575,6 +580,37 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
                 return rc;
         }
         for (int l = 0; l < D.L && !tcp; ++l) {
+            if (streamed && R == 1 && ctx->fused_layer) {
+                LayerArgs la{};
+                la.dim = D;
+                la.map = map;
+                la.W_qkv = (const uint16_t *)W.W_qkv[l];
+                la.attn_norm = (const uint16_t *)W.attn_norm[l];
+                la.W_o = (const uint16_t *)W.W_o[l];
+                la.W_gate = (const uint16_t *)W.W_gate[l];
+                la.W_up = (const uint16_t *)W.W_up[l];
+                la.W_down = (const uint16_t *)W.W_down[l];
+                la.ffn_norm = (const uint16_t *)W.ffn_norm[l];
+                la.x = x;
+                la.s = sb;
+                la.q = ws.q;
+                la.k_pages = (uint16_t *)kv->k_pages + l * layer_pages;
+                la.v_pages = (uint16_t *)kv->v_pages + l * layer_pages;
+                la.page_table = kv->page_table;
+                la.max_pages = kv->max_pages_per_seq;
+                la.n_splits = layer_fused_splits(D, max_ctx, ctx->sms);
+                la.split_len = attn_split_len(max_ctx, la.n_splits);
+                la.attn_part = ws.attn_part;
+                la.attn_out = ws.attn_out;
+                la.attn_ticket = ws.attn_ticket;
+                la.h = ws.ffn_h;
+                la.bar_count = ws.grid_bar;
+                la.bar_gen = ws.grid_bar + 1;
+                la.status = dev_status;
+                for (int i = 0; i < D.hd / 2; ++i) la.inv_freq[i] = ctx->inv_freq[i];
+                if ((e = launch_layer_fused(la, ctx->sms, s)) != cudaSuccess) return cuda_fail(e, "fused layer launch");
+                continue;
+            }
             g.map = map;
             g.R = R;
             g.x = x;

@@ -292,7 +292,8 @@ struct AttnTrReduce {
 // chunk is unpacked once for the G query heads and the q.k sums are completed
 // by a transposed butterfly (one score per lane).  Leaves the warp's partial
 // (max, sum, G x HD accumulator) in sm_m / sm_l / sm_acc[warp].
-template <int HD, int G, int NW, int NSPW>
+// QCG: read q through L2 (q written by other blocks of the same grid).
+template <int HD, int G, int NW, int NSPW, bool QCG = false>
 __device__ __forceinline__ void attn_warp_pages(const AttnArgs &a, int b, int r, int kvh, int qh0, int k_begin,
                                                 int k_end, int pos0, uint8_t *ring, uint64_t (*full)[NSPW],
                                                 float (*sm_m)[G], float (*sm_l)[G], float (*sm_acc)[G][HD]) {
@@ -357,7 +358,8 @@ __device__ __forceinline__ void attn_warp_pages(const AttnArgs &a, int b, int r,
 #pragma unroll
     for (int g = 0; g < G; ++g) {
         const float *qp = a.q + (size_t)r * D.Hq * HD + (size_t)(qh0 + g) * HD + dl;
-        const float4 q0 = *(const float4 *)qp, q1 = *(const float4 *)(qp + 4);
+        const float4 q0 = QCG ? __ldcg((const float4 *)qp) : *(const float4 *)qp;
+        const float4 q1 = QCG ? __ldcg((const float4 *)(qp + 4)) : *(const float4 *)(qp + 4);
         q[g][0] = q0.x * scale; q[g][1] = q0.y * scale; q[g][2] = q0.z * scale; q[g][3] = q0.w * scale;
         q[g][4] = q1.x * scale; q[g][5] = q1.y * scale; q[g][6] = q1.z * scale; q[g][7] = q1.w * scale;
 #pragma unroll
@@ -1228,6 +1230,396 @@ cudaError_t draft_set_attributes() {
     if ((e = allow_smem(lm_head_kernel<2>))) return e;
     if ((e = allow_smem(lm_head_kernel<4>))) return e;
     return allow_smem(lm_head_kernel<8>);
+}
+
+// ---------------------------------------------------------------------------
+// Fused batch-1 layer: a whole drafter layer of one chain row (Sec. 3.3 Eq. 2-3
+// and the transferred block) in one launch, one block per SM.  Block c owns
+// pair units [u0, u1) of the expanded QKV rows (rows i and i + hd/2 of a head,
+// so the rotation stays in the block), KV head c / n_splits and key range
+// c % n_splits of the attention (blocks past Hkv x n_splits skip it), rows
+// [o0, o1) of W_o and W_down and SwiGLU units [f0, f1).  Phases, each ending in
+// a grid barrier:
+//   A  z = RMSNorm(x); the block's q/k/v pairs of W~_qkv [s; z]; RoPE; k, v to
+//      the page
+//   B  attention partial of the block's key range; the last range of a KV head
+//      merges the ranges
+//   C  x += W_o attn (own rows)
+//   D  n = RMSNorm(x); h = silu(W_g n) * (W_u n) (own units)
+//   E  x += W_down h (own rows)
+// Shared memory regions:
+//   A  QKV pair rows (requested before griddepcontrol.wait), then the gate/up
+//      rows (requested when phase A is done), then the down rows (requested
+//      when phase D is done)
+//   B  W_o rows (requested before griddepcontrol.wait)
+//   C  [s; z], then the attention pages, then the activation of C-E
+// Values written by other blocks are read through L2 (ld.global.cg), or by
+// bulk copies after proxy fences on both sides of the barrier.
+constexpr int LY_THREADS = 256;
+constexpr int LY_WARPS = LY_THREADS / 32;
+constexpr int LY_NSPW = 1;   // attention pages in flight per warp
+
+struct LayerPlan {
+    int nu, up, ro, rf;   // pair units (all), per block at most; O/down rows, SwiGLU units per block at most
+    size_t a_bytes, b_bytes, c_bytes, smem;
+};
+
+static __host__ __device__ size_t ly_round(size_t x) { return (x + 127) / 128 * 128; }
+
+static __host__ __device__ LayerPlan layer_plan(const Dims &D, int grid) {
+    LayerPlan p{};
+    p.nu = (D.Hq + 2 * D.Hkv) * (D.hd / 2);
+    p.up = (p.nu + grid - 1) / grid;
+    p.ro = (D.d + grid - 1) / grid;
+    p.rf = (D.F + grid - 1) / grid;
+    const int Ko = D.Hq * D.hd;
+    const size_t qkv = (size_t)2 * p.up * 2 * D.d * 2, gu = (size_t)2 * p.rf * D.d * 2;
+    const size_t dn = (size_t)p.ro * D.F * 2;
+    size_t a = qkv > gu ? qkv : gu;
+    a = a > dn ? a : dn;
+    const size_t ring = (size_t)LY_WARPS * LY_NSPW * 2 * 16 * D.hd * 2;
+    int act = 2 * D.d > Ko ? 2 * D.d : Ko;
+    act = act > D.F ? act : D.F;
+    p.a_bytes = ly_round(a);
+    p.b_bytes = ly_round((size_t)p.ro * Ko * 2);
+    p.c_bytes = ly_round(ring > (size_t)act * 4 ? ring : (size_t)act * 4);
+    p.smem = p.a_bytes + p.b_bytes + p.c_bytes;
+    return p;
+}
+
+// Dot of one bf16 weight row with a float32 row, both in shared memory: lane l
+// takes elements base + 8l .. base + 8l + 7 of every 256-wide chunk in
+// ascending order, then a butterfly sum.  Kd is a multiple of 256.
+__device__ __forceinline__ float ly_dot(const uint16_t *w, const float *xs, int Kd) {
+    const int lane = threadIdx.x & 31;
+    float acc = 0.f;
+#pragma unroll 4
+    for (int base = 0; base < Kd; base += 256) {
+        const uint4 wv = *(const uint4 *)(w + base + lane * 8);
+        float wf[8];
+        unpack8(wv, wf);
+        const float4 x0 = *(const float4 *)(xs + base + lane * 8);
+        const float4 x1 = *(const float4 *)(xs + base + lane * 8 + 4);
+        const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], xf[e], acc);
+    }
+    return warp_sum(acc);
+}
+
+// v[0, d) <- RMSNorm(v) * gain, in place, by the whole block.
+__device__ __forceinline__ void ly_rmsnorm(float *v, const uint16_t *gain, int d, float eps, float *red) {
+    __syncthreads();   // v was written by other threads
+    float ss = 0.f;
+    for (int i = threadIdx.x; i < d; i += LY_THREADS) ss = fmaf(v[i], v[i], ss);
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < LY_WARPS; ++w) t += red[w];
+    const float inv = rsqrtf(t / (float)d + eps);
+    for (int i = threadIdx.x; i < d; i += LY_THREADS) v[i] = v[i] * inv * bf_to_f(gain[i]);
+    __syncthreads();
+}
+
+__device__ __forceinline__ void fence_proxy_async_global() {
+    asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
+template <int HD, int G>
+__global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerArgs a) {
+    constexpr int NW = LY_WARPS;
+    extern __shared__ __align__(128) uint8_t smem[];
+    __shared__ __align__(8) uint64_t bar[4];   // QKV rows, W_o rows, gate/up rows, down rows
+    __shared__ __align__(8) uint64_t full[NW][LY_NSPW];
+    __shared__ float sm_m[NW][G], sm_l[NW][G];
+    __shared__ float sm_acc[NW][G][HD];
+    __shared__ float red[NW];
+    const Dims &D = a.dim;
+    const int d = D.d, F = D.F, Ko = D.Hq * HD, half = HD / 2;
+    const int nb = gridDim.x, c = blockIdx.x;
+    const LayerPlan p = layer_plan(D, nb);
+    uint8_t *regA = smem, *regB = smem + p.a_bytes, *regC = regB + p.b_bytes;
+    const int u0 = (int)((long long)p.nu * c / nb), u1 = (int)((long long)p.nu * (c + 1) / nb), nu = u1 - u0;
+    const int o0 = (int)((long long)d * c / nb), o1 = (int)((long long)d * (c + 1) / nb), no = o1 - o0;
+    const int f0 = (int)((long long)F * c / nb), f1 = (int)((long long)F * (c + 1) / nb), nf = f1 - f0;
+    uint16_t *wq_lo = (uint16_t *)regA;                    // [up][2d]: row i of the unit's head
+    uint16_t *wq_hi = wq_lo + (size_t)p.up * 2 * d;         // [up][2d]: row i + hd/2
+    uint16_t *wg = (uint16_t *)regA;                        // [rf][d]
+    uint16_t *wu = wg + (size_t)p.rf * d;                   // [rf][d]
+    uint16_t *wd = (uint16_t *)regA;                        // [ro][F]
+    uint16_t *wo = (uint16_t *)regB;                        // [ro][Ko]
+    float *act = (float *)regC;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int issued = 0;   // thread 0: barriers 0 .. issued-1 have copies requested
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < 4; ++i) mbar_init(&bar[i], 1);
+        mbar_fence_init();
+        // the weights do not depend on earlier kernels: request them now
+        const uint32_t row_b = (uint32_t)4 * d;   // one expanded QKV row: 2d bf16
+        mbar_arrive_expect_tx(&bar[0], (uint32_t)nu * 2 * row_b);
+        for (int u = u0; u < u1;) {   // the units of one head at a time: two row ranges each
+            const int h = u / half, i = u - h * half;
+            const int n = min(u1 - u, half - i);
+            const size_t lo = (size_t)h * HD + i;
+            bulk_g2s(wq_lo + (size_t)(u - u0) * 2 * d, a.W_qkv + lo * 2 * d, (uint32_t)n * row_b, &bar[0]);
+            bulk_g2s(wq_hi + (size_t)(u - u0) * 2 * d, a.W_qkv + (lo + half) * 2 * d, (uint32_t)n * row_b, &bar[0]);
+            u += n;
+        }
+        const uint32_t bo = (uint32_t)no * Ko * 2;
+        mbar_arrive_expect_tx(&bar[1], bo);
+        if (bo) bulk_g2s(wo, a.W_o + (size_t)o0 * Ko, bo, &bar[1]);
+        issued = 2;
+    }
+    pdl_trigger();
+    int b = 0, pos = 0;
+    const bool live = a.map.row(0, b, pos);   // the row map was written before the chain
+    __syncthreads();
+    pdl_wait();   // the residual, the context slot and this call's K/V rows come from earlier kernels
+    bool ok = true;
+
+    // ---- A. [s; RMSNorm(x) gamma] -> the block's q/k/v pairs, RoPE, K/V rows
+    float *u_s = act;   // [2d]
+    if (live) {
+        for (int i = threadIdx.x * 4; i < d; i += LY_THREADS * 4) {
+            *(float4 *)(u_s + i) = __ldcg((const float4 *)(a.s + i));
+            *(float4 *)(u_s + d + i) = __ldcg((const float4 *)(a.x + i));
+        }
+        ly_rmsnorm(u_s + d, a.attn_norm, d, D.eps, red);
+    }
+    ok = ok && __syncthreads_and(mbar_wait(&bar[0], 0));
+    if (ok && live)
+        for (int k = warp; k < nu; k += NW) {
+            const float y1 = ly_dot(wq_lo + (size_t)k * 2 * d, u_s, 2 * d);
+            const float y2 = ly_dot(wq_hi + (size_t)k * 2 * d, u_s, 2 * d);
+            if (lane == 0) {
+                const int unit = u0 + k, h = unit / half, i = unit - h * half;
+                float x1 = y1, x2 = y2;
+                if (h < D.Hq + D.Hkv) {   // rotate-half RoPE on q and k
+                    float cs, sn;
+                    rope_cs2(a.inv_freq[i], pos, cs, sn);
+                    x1 = y1 * cs - y2 * sn;
+                    x2 = y2 * cs + y1 * sn;
+                }
+                if (h < D.Hq) {
+                    a.q[(size_t)h * HD + i] = x1;
+                    a.q[(size_t)h * HD + i + half] = x2;
+                } else {
+                    const bool is_k = h < D.Hq + D.Hkv;
+                    const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
+                    const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
+                    uint16_t *dst = (is_k ? a.k_pages : a.v_pages) +
+                                    (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * HD;
+                    dst[i] = f_to_bf(x1);
+                    dst[i + half] = f_to_bf(x2);
+                }
+            }
+        }
+    fence_proxy_async_global();   // the K/V rows are read by other blocks' bulk copies
+    grid_sync(a.bar_count, a.bar_gen, a.status);
+
+    // ---- B. attention partial of the block's key range; gate/up rows requested
+    fence_proxy_async_global();
+    fence_proxy_async_smem();     // regions A and C are refilled by bulk copies
+    __syncthreads();
+    if (threadIdx.x == 0 && ok) {
+        const uint32_t bf = (uint32_t)nf * d * 2;
+        mbar_arrive_expect_tx(&bar[2], 2 * bf);
+        if (bf) {
+            bulk_g2s(wg, a.W_gate + (size_t)f0 * d, bf, &bar[2]);
+            bulk_g2s(wu, a.W_up + (size_t)f0 * d, bf, &bar[2]);
+        }
+        issued = 3;
+    }
+    const int units = D.Hkv * a.n_splits;
+    if (live && c < units) {
+        const int kvh = c / a.n_splits, split = c - kvh * a.n_splits;
+        const int n_keys = pos + 1, pos0 = a.map.pos0[b];
+        const int k_begin = split * a.split_len;   // a multiple of the page size
+        const int k_end = min(n_keys, k_begin + a.split_len);
+        AttnArgs at{};
+        at.dim = D;
+        at.q = a.q;
+        at.k_pages = a.k_pages;
+        at.v_pages = a.v_pages;
+        at.page_table = a.page_table;
+        at.max_pages = a.max_pages;
+        at.status = a.status;
+        attn_warp_pages<HD, G, NW, LY_NSPW, true>(at, b, 0, kvh, kvh * G, k_begin, k_end, pos0, regC, full, sm_m,
+                                                  sm_l, sm_acc);
+        __syncthreads();
+        for (int idx = threadIdx.x; idx < G * HD; idx += LY_THREADS) {
+            const int g = idx / HD, dim = idx - g * HD;
+            float M = -INFINITY;
+#pragma unroll
+            for (int w = 0; w < NW; ++w) M = fmaxf(M, sm_m[w][g]);
+            float num = 0.f, den = 0.f;
+            if (M != -INFINITY)
+#pragma unroll
+                for (int w = 0; w < NW; ++w) {
+                    const float f = sm_m[w][g] == -INFINITY ? 0.f : __expf(sm_m[w][g] - M);
+                    num = fmaf(f, sm_acc[w][g][dim], num);
+                    den = fmaf(f, sm_l[w][g], den);
+                }
+            float *pp = a.attn_part + ((size_t)(kvh * G + g) * a.n_splits + split) * (HD + 2);
+            pp[2 + dim] = num;
+            if (dim == 0) { pp[0] = M; pp[1] = den; }
+        }
+        if (arrive_last(a.attn_ticket + kvh, a.n_splits)) {
+            // the last key range of this KV head merges the ranges
+            for (int idx = threadIdx.x; idx < G * HD; idx += LY_THREADS) {
+                const int g = idx / HD, dim = idx - g * HD;
+                const float *base = a.attn_part + (size_t)(kvh * G + g) * a.n_splits * (HD + 2);
+                float M = -INFINITY;
+                for (int sp = 0; sp < a.n_splits; ++sp) M = fmaxf(M, __ldcg(base + (size_t)sp * (HD + 2)));
+                float num = 0.f, den = 0.f;
+                for (int sp = 0; sp < a.n_splits; ++sp) {
+                    const float *pp = base + (size_t)sp * (HD + 2);
+                    const float ms = __ldcg(pp);
+                    const float f = ms == -INFINITY ? 0.f : __expf(ms - M);
+                    num = fmaf(f, __ldcg(pp + 2 + dim), num);
+                    den = fmaf(f, __ldcg(pp + 1), den);
+                }
+                a.attn_out[(size_t)(kvh * G + g) * HD + dim] = num / den;
+            }
+        }
+    }
+    grid_sync(a.bar_count, a.bar_gen, a.status);
+
+    // ---- C. O-proj and residual
+    if (live)
+        for (int i = threadIdx.x * 4; i < Ko; i += LY_THREADS * 4)
+            *(float4 *)(act + i) = __ldcg((const float4 *)(a.attn_out + i));
+    __syncthreads();
+    ok = ok && __syncthreads_and(mbar_wait(&bar[1], 0));
+    if (ok && live)
+        for (int j = warp; j < no; j += NW) {
+            const float acc = ly_dot(wo + (size_t)j * Ko, act, Ko);
+            if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
+        }
+    grid_sync(a.bar_count, a.bar_gen, a.status);
+
+    // ---- D. RMSNorm of the whole residual, gate/up and SwiGLU
+    if (live) {
+        for (int i = threadIdx.x * 4; i < d; i += LY_THREADS * 4)
+            *(float4 *)(act + i) = __ldcg((const float4 *)(a.x + i));
+        ly_rmsnorm(act, a.ffn_norm, d, D.eps, red);
+    }
+    __syncthreads();
+    ok = ok && __syncthreads_and(mbar_wait(&bar[2], 0));
+    if (ok && live)
+        for (int j = warp; j < nf; j += NW) {
+            const float g = ly_dot(wg + (size_t)j * d, act, d);
+            const float u = ly_dot(wu + (size_t)j * d, act, d);
+            if (lane == 0) a.h[f0 + j] = g / (1.f + expf(-g)) * u;
+        }
+    fence_proxy_async_smem();   // region A takes the down rows next
+    __syncthreads();
+    if (threadIdx.x == 0 && ok) {
+        const uint32_t bd = (uint32_t)no * F * 2;
+        mbar_arrive_expect_tx(&bar[3], bd);
+        if (bd) bulk_g2s(wd, a.W_down + (size_t)o0 * F, bd, &bar[3]);
+        issued = 4;
+    }
+    grid_sync(a.bar_count, a.bar_gen, a.status);
+
+    // ---- E. down and residual
+    if (live)
+        for (int i = threadIdx.x * 4; i < F; i += LY_THREADS * 4)
+            *(float4 *)(act + i) = __ldcg((const float4 *)(a.h + i));
+    __syncthreads();
+    ok = ok && __syncthreads_and(mbar_wait(&bar[3], 0));
+    if (ok && live)
+        for (int j = warp; j < no; j += NW) {
+            const float acc = ly_dot(wd + (size_t)j * F, act, F);
+            if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
+        }
+    if (!ok) {
+        if (threadIdx.x == 0) {
+            set_status(a.status, OSPREY_ERR_TIMEOUT);
+            for (int i = 0; i < issued; ++i) mbar_wait(&bar[i], 0, 200000000LL);   // copies land before exit
+        }
+        __syncthreads();
+    }
+}
+
+int layer_fused_splits(const Dims &D, int max_ctx, int sms) {
+    int ns = sms / D.Hkv;
+    const int cap = attn_splits(1, D.Hkv, max_ctx, sms);
+    if (ns > cap) ns = cap;
+    return ns < 1 ? 1 : ns;
+}
+
+template <int HD, int G>
+static bool layer_fits(const LayerPlan &p) {
+    int dev = 0, optin = 0;
+    cudaFuncAttributes fa{};
+    if (cudaGetDevice(&dev) != cudaSuccess ||
+        cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess ||
+        cudaFuncGetAttributes(&fa, layer_fused_kernel<HD, G>) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return p.smem + fa.sharedSizeBytes <= (size_t)optin;
+}
+
+bool layer_fused_supported(const Dims &D, int sms) {
+    const int G = D.Hq / D.Hkv;
+    if ((D.hd != 64 && D.hd != 128) || (G != 1 && G != 2 && G != 4 && G != 8) || D.P != 16) return false;
+    if (D.d % 256 || D.F % 256 || (D.Hq * D.hd) % 256 || D.Hkv > sms) return false;
+    const LayerPlan p = layer_plan(D, sms);
+    // each mbarrier phase counts fewer than 2^20 bytes
+    if ((size_t)p.up * 2 * 4 * D.d >= (1u << 20) || (size_t)p.ro * D.Hq * D.hd * 2 >= (1u << 20) ||
+        (size_t)2 * p.rf * D.d * 2 >= (1u << 20) || (size_t)p.ro * D.F * 2 >= (1u << 20))
+        return false;
+#define OSP_LY_FITS(hd_, g_) \
+    if (D.hd == hd_ && G == g_) return layer_fits<hd_, g_>(p);
+    OSP_LY_FITS(64, 1) OSP_LY_FITS(64, 2) OSP_LY_FITS(64, 4) OSP_LY_FITS(64, 8)
+    OSP_LY_FITS(128, 1) OSP_LY_FITS(128, 2) OSP_LY_FITS(128, 4) OSP_LY_FITS(128, 8)
+#undef OSP_LY_FITS
+    return false;
+}
+
+template <int HD, int G>
+static cudaError_t launch_layer_t(const LayerArgs &a, int sms, cudaStream_t s) {
+    const LayerPlan p = layer_plan(a.dim, sms);
+    static int attr_dev = -1;
+    static size_t attr_smem = 0;   // the opt-in grows with the largest shape launched so far
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    if (attr_dev != dev || p.smem > attr_smem) {
+        e = cudaFuncSetAttribute(layer_fused_kernel<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
+        if (e != cudaSuccess) return e;
+        attr_dev = dev;
+        attr_smem = p.smem;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(sms);
+    cfg.blockDim = dim3(LY_THREADS);
+    cfg.dynamicSmemBytes = p.smem;
+    cfg.stream = s;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    e = cudaLaunchKernelEx(&cfg, layer_fused_kernel<HD, G>, a);
+    count_launch();
+    return e;
+}
+
+cudaError_t launch_layer_fused(const LayerArgs &a, int sms, cudaStream_t s) {
+    const int G = a.dim.Hq / a.dim.Hkv;
+    if (a.n_splits < 1 || a.dim.Hkv * a.n_splits > sms || a.split_len % 16) return cudaErrorInvalidValue;
+#define OSP_LY_LAUNCH(hd_, g_) \
+    if (a.dim.hd == hd_ && G == g_) return launch_layer_t<hd_, g_>(a, sms, s);
+    OSP_LY_LAUNCH(64, 1) OSP_LY_LAUNCH(64, 2) OSP_LY_LAUNCH(64, 4) OSP_LY_LAUNCH(64, 8)
+    OSP_LY_LAUNCH(128, 1) OSP_LY_LAUNCH(128, 2) OSP_LY_LAUNCH(128, 4) OSP_LY_LAUNCH(128, 8)
+#undef OSP_LY_LAUNCH
+    return cudaErrorInvalidValue;
 }
 
 }  // namespace osp

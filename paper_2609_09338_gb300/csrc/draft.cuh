@@ -183,6 +183,33 @@ struct MlpArgs {
 bool mlp_fused_supported(const Dims &D, int sms);
 cudaError_t launch_mlp_fused(const MlpArgs &a, int sms, cudaStream_t s);
 
+// Batch-1 chain steps: a whole drafter layer in one launch (one block per SM):
+// RMSNorm + expanded QKV + RoPE + K/V write | split-KV attention (the last
+// split of a KV head merges) | O-proj + residual | RMSNorm + gate/up + SwiGLU |
+// down + residual, each '|' a grid barrier.
+struct LayerArgs {
+    Dims dim;
+    RowMap map;                       // row 0 of the step
+    const uint16_t *W_qkv, *attn_norm, *W_o, *W_gate, *W_up, *W_down, *ffn_norm;
+    float *x;                         // [d] residual stream of the row
+    const float *s;                   // [d] context slot of the row
+    float *q;                         // [Hq hd] rotated queries (scratch)
+    uint16_t *k_pages, *v_pages;      // this layer's pages
+    const int32_t *page_table;
+    int max_pages;
+    int n_splits, split_len;          // attention: key ranges per KV head (Hkv x n_splits <= grid)
+    float *attn_part;                 // [Hq][n_splits][hd + 2]
+    float *attn_out;                  // [Hq hd]
+    int *attn_ticket;                 // [Hkv], zero between uses
+    float *h;                         // [F] SwiGLU hidden (scratch)
+    unsigned *bar_count, *bar_gen;    // grid barrier words; count zero between uses
+    int32_t *status;
+    double inv_freq[64];
+};
+bool layer_fused_supported(const Dims &D, int sms);
+int layer_fused_splits(const Dims &D, int max_ctx, int sms);
+cudaError_t launch_layer_fused(const LayerArgs &a, int sms, cudaStream_t s);
+
 StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms);
 bool stream_supported(GemvMode mode, const Dims &D, int rg, int sms);
 cudaError_t launch_stream(GemvMode mode, const StreamArgs &a, int rg, cudaStream_t s);

@@ -246,6 +246,23 @@ def test_fused_layer_tail_matches_oracle(T, monkeypatch):
     check_case(case)
 
 
+@pytest.mark.skipif(os.environ.get("OSPREY_TEST_FUSED_LAYER") != "1",
+                    reason="the fused layer (OSPREY_FUSED_LAYER) is off by default; set OSPREY_TEST_FUSED_LAYER=1")
+@pytest.mark.parametrize("which", ["qwen3-8b-greedy", "qwen3-8b-sampled", "tiny-2-layers"])
+def test_fused_layer_matches_oracle(which, monkeypatch):
+    """Batch-1 chain steps with each whole layer (QKV + RoPE + K/V write,
+    attention, O-proj, gate/up, down) in one launch, grid barriers between the
+    phases."""
+    monkeypatch.setenv("OSPREY_FUSED_LAYER", "1")
+    if which.startswith("qwen3"):
+        wl = WORKLOADS["qwen3-8b-d1024-v151936-b1-k7"]
+        case = run_case(wl.shape, syn.make_contexts(wl), wl.K, 0.0 if which.endswith("greedy") else 1.0, wl.seed)
+    else:
+        shape = replace(TINY, n_layers=2)
+        case = run_case(shape, [77], 5, 1.0, 57)
+    check_case(case)
+
+
 def test_paper_shaped_body_extend_rows():
     """The paper's drafter body (two blocks, d 2560, 32/8 heads of 128, FFN 9728,
     12288 feature columns) at a reduced vocabulary and context: 3 extend rows
