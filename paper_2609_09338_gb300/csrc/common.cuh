@@ -184,6 +184,26 @@ __device__ __forceinline__ void rope_cs2(double inv_freq, int pos, float &c, flo
     sincosf((float)(frac * 6.283185307179586), &s, &c);
 }
 
+// One warp: dot of a bf16 weight row with a float32 row, both in shared
+// memory.  Lane l takes elements base + 8l .. base + 8l + 7 of every 256-wide
+// chunk in ascending order, then a butterfly sum.  Kd is a multiple of 256.
+__device__ __forceinline__ float warp_smem_dot(const uint16_t *w, const float *xs, int Kd) {
+    const int lane = threadIdx.x & 31;
+    float acc = 0.f;
+#pragma unroll 4
+    for (int base = 0; base < Kd; base += 256) {
+        const uint4 wv = *(const uint4 *)(w + base + lane * 8);
+        float wf[8];
+        unpack8(wv, wf);
+        const float4 x0 = *(const float4 *)(xs + base + lane * 8);
+        const float4 x1 = *(const float4 *)(xs + base + lane * 8 + 4);
+        const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+        for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], xf[e], acc);
+    }
+    return warp_sum(acc);
+}
+
 __device__ __forceinline__ void set_status(int32_t *status, int code) {
     if (status) atomicCAS((int *)status, 0, code);
 }

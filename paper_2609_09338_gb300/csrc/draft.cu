@@ -1287,26 +1287,6 @@ static __host__ __device__ LayerPlan layer_plan(const Dims &D, int grid) {
     return p;
 }
 
-// Dot of one bf16 weight row with a float32 row, both in shared memory: lane l
-// takes elements base + 8l .. base + 8l + 7 of every 256-wide chunk in
-// ascending order, then a butterfly sum.  Kd is a multiple of 256.
-__device__ __forceinline__ float ly_dot(const uint16_t *w, const float *xs, int Kd) {
-    const int lane = threadIdx.x & 31;
-    float acc = 0.f;
-#pragma unroll 4
-    for (int base = 0; base < Kd; base += 256) {
-        const uint4 wv = *(const uint4 *)(w + base + lane * 8);
-        float wf[8];
-        unpack8(wv, wf);
-        const float4 x0 = *(const float4 *)(xs + base + lane * 8);
-        const float4 x1 = *(const float4 *)(xs + base + lane * 8 + 4);
-        const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], xf[e], acc);
-    }
-    return warp_sum(acc);
-}
-
 // v[0, d) <- RMSNorm(v) * gain, in place, by the whole block.
 __device__ __forceinline__ void ly_rmsnorm(float *v, const uint16_t *gain, int d, float eps, float *red) {
     __syncthreads();   // v was written by other threads
@@ -1392,8 +1372,8 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
     ok = ok && __syncthreads_and(mbar_wait(&bar[0], 0));
     if (ok && live)
         for (int k = warp; k < nu; k += NW) {
-            const float y1 = ly_dot(wq_lo + (size_t)k * 2 * d, u_s, 2 * d);
-            const float y2 = ly_dot(wq_hi + (size_t)k * 2 * d, u_s, 2 * d);
+            const float y1 = warp_smem_dot(wq_lo + (size_t)k * 2 * d, u_s, 2 * d);
+            const float y2 = warp_smem_dot(wq_hi + (size_t)k * 2 * d, u_s, 2 * d);
             if (lane == 0) {
                 const int unit = u0 + k, h = unit / half, i = unit - h * half;
                 float x1 = y1, x2 = y2;
@@ -1496,7 +1476,7 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
     ok = ok && __syncthreads_and(mbar_wait(&bar[1], 0));
     if (ok && live)
         for (int j = warp; j < no; j += NW) {
-            const float acc = ly_dot(wo + (size_t)j * Ko, act, Ko);
+            const float acc = warp_smem_dot(wo + (size_t)j * Ko, act, Ko);
             if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
         }
     grid_sync(a.bar_count, a.bar_gen, a.status);
@@ -1511,8 +1491,8 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
     ok = ok && __syncthreads_and(mbar_wait(&bar[2], 0));
     if (ok && live)
         for (int j = warp; j < nf; j += NW) {
-            const float g = ly_dot(wg + (size_t)j * d, act, d);
-            const float u = ly_dot(wu + (size_t)j * d, act, d);
+            const float g = warp_smem_dot(wg + (size_t)j * d, act, d);
+            const float u = warp_smem_dot(wu + (size_t)j * d, act, d);
             if (lane == 0) a.h[f0 + j] = g / (1.f + expf(-g)) * u;
         }
     fence_proxy_async_smem();   // region A takes the down rows next
@@ -1533,7 +1513,7 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
     ok = ok && __syncthreads_and(mbar_wait(&bar[3], 0));
     if (ok && live)
         for (int j = warp; j < no; j += NW) {
-            const float acc = ly_dot(wd + (size_t)j * F, act, F);
+            const float acc = warp_smem_dot(wd + (size_t)j * F, act, F);
             if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
         }
     if (!ok) {

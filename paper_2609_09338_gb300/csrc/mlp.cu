@@ -9,26 +9,6 @@
 
 namespace osp {
 
-// Dot of one bf16 weight row in shared memory with a float32 row in shared
-// memory: lane l takes elements base + 8l .. base + 8l + 7 of every 256-wide
-// chunk in ascending order, then a butterfly sum (the streamed GEMV's order).
-__device__ __forceinline__ float mlp_dot(const uint16_t *w, const float *xs, int Kd) {
-    const int lane = threadIdx.x & 31;
-    float acc = 0.f;
-#pragma unroll 4
-    for (int base = 0; base < Kd; base += 256) {
-        const uint4 wv = *(const uint4 *)(w + base + lane * 8);
-        float wf[8];
-        unpack8(wv, wf);
-        const float4 x0 = *(const float4 *)(xs + base + lane * 8);
-        const float4 x1 = *(const float4 *)(xs + base + lane * 8 + 4);
-        const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
-#pragma unroll
-        for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], xf[e], acc);
-    }
-    return warp_sum(acc);
-}
-
 // Fused O-proj / gate-up / down of one layer for one activation row (batch-1
 // chain steps).  Block c owns output rows [o0, o1) of W_o and W_down and
 // SwiGLU units [f0, f1) of W_gate / W_up; all four slices are contiguous in
@@ -105,7 +85,7 @@ __global__ void __launch_bounds__(MLP_THREADS, 1) mlp_fused_kernel(const MlpArgs
     ok = ok && __syncthreads_and(mbar_wait(&bar[0], 0));
     if (ok && live)
         for (int j = warp; j < no; j += NW) {
-            const float acc = mlp_dot(wo + (size_t)j * Ko, act, Ko);
+            const float acc = warp_smem_dot(wo + (size_t)j * Ko, act, Ko);
             if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
         }
     grid_sync(a.bar_count, a.bar_gen, a.status);
@@ -131,8 +111,8 @@ __global__ void __launch_bounds__(MLP_THREADS, 1) mlp_fused_kernel(const MlpArgs
     ok = ok && __syncthreads_and(mbar_wait(&bar[1], 0));
     if (ok && live)
         for (int j = warp; j < nf; j += NW) {
-            const float g = mlp_dot(wg + (size_t)j * d, act, d);
-            const float u = mlp_dot(wu + (size_t)j * d, act, d);
+            const float g = warp_smem_dot(wg + (size_t)j * d, act, d);
+            const float u = warp_smem_dot(wu + (size_t)j * d, act, d);
             if (lane == 0) a.h[f0 + j] = g / (1.f + expf(-g)) * u;
         }
     grid_sync(a.bar_count, a.bar_gen, a.status);
@@ -145,7 +125,7 @@ __global__ void __launch_bounds__(MLP_THREADS, 1) mlp_fused_kernel(const MlpArgs
     ok = ok && __syncthreads_and(mbar_wait(&bar[2], 0));
     if (ok && live)
         for (int j = warp; j < no; j += NW) {
-            const float acc = mlp_dot(wd + (size_t)j * F, act, F);
+            const float acc = warp_smem_dot(wd + (size_t)j * F, act, F);
             if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
         }
     if (!ok) {
