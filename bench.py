@@ -219,6 +219,16 @@ def run_reference(args):
     }))
 
 
+def lm_head_label(B):
+    """The LM-head launches the probes bracket, by the number of rows (the draft
+    step's kernel selection)."""
+    if B <= 2:
+        return "stream_kernel<LM> (final RMSNorm + TMA-streamed LM-head GEMV + on-chip sampling)"
+    if B <= 80:
+        return "planes_kernel + tc_kernel<STORE> + row_sample_kernel (tcgen05 LM head, then sampling)"
+    return "lm_head_kernel (CUDA-core LM head + on-chip sampling)"
+
+
 def config_of(wl, ctx):
     sh = wl.shape
     return {"workload": wl.name, "batch": wl.batch, "K": wl.K, "ctx": [int(ctx.min()), int(ctx.max())],
@@ -529,7 +539,7 @@ def main():
             "draft_step_bytes": nb["draft"],
             "step_hbm_frac": (nb["draft"] + nb["verify"]) / (ms * 1e-3) / 1e9 / peak,
             "synthetic_al": acc_len,
-            "roofline": {"kernel": "stream_kernel<LM> (final RMSNorm + TMA-streamed LM-head GEMV + on-chip sampling)",
+            "roofline": {"kernel": lm_head_label(B),
                          "bound": "hbm", "achieved": lm_gbs, "peak": peak, "unit": "GB/s",
                          "frac": lm_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
                          "bytes_per_launch": nb["lm_head_launch"], "mean_launch_us": lm_mean_ms * 1e3,
