@@ -113,7 +113,11 @@ const char *osprey_last_error(void);
  *     partials.
  * Two environment variables, read here, select the alternatives for testing:
  * OSPREY_TC=0 (CUDA-core GEMVs for batched rows) and OSPREY_ATTN_CLUSTER=0
- * (global-partials attention).
+ * (global-partials attention).  Two more select fused batch-1 chain steps,
+ * off by default: OSPREY_FUSED_MLP=1 (O-proj, gate/up and down of a layer as
+ * one launch) and OSPREY_FUSED_LAYER=1 (the whole layer as one launch, for
+ * shapes whose per-SM weight slices fit shared memory); both use one block per
+ * SM and bounded grid barriers.
  * Errors: INVALID_ARG (null), SHAPE (unsupported dimension). */
 int osprey_create(const osprey_config *cfg, const osprey_weights *w, osprey_ctx **out);
 void osprey_destroy(osprey_ctx *ctx);
