@@ -53,7 +53,7 @@ enum {
     OSPREY_ERR_DTYPE = -3,       /* unknown logits dtype */
     OSPREY_ERR_CAPACITY = -4,    /* pages or workspace too small */
     OSPREY_ERR_CUDA = -5,        /* a CUDA runtime call failed */
-    OSPREY_ERR_TIMEOUT = -6      /* reserved for bounded device waits */
+    OSPREY_ERR_TIMEOUT = -6      /* a bounded device wait ran out (dev_status) */
 };
 
 enum { OSPREY_F32 = 0, OSPREY_BF16 = 1 };
