@@ -56,16 +56,26 @@ def parse():
     p.add_argument("--temperature", type=float, default=None, help="override the workload's temperature")
     p.add_argument("--verify-sweep", action="store_true",
                    help="time verify alone over batch x K at V=200064 (fp32 and bf16 logits)")
+    p.add_argument("--weights", default=None,
+                   help="drafter weight file: read it if it exists (it must hold the workload's shape), "
+                        "else write the seeded weights there")
     p.add_argument("--verify-hidden", action="store_true",
                    help="compare draft (logits written) + verify against draft (states kept) + logits-free verify")
     return p.parse_args()
 
 
-def make_inputs(wl, rank=0):
+def make_inputs(wl, rank=0, weights_path=None):
     sh = wl.shape
     seed = wl.seed + 1000 * rank
     ctx = syn.make_contexts(wl, seed + 17)
-    w = syn.make_weights(sh, seed)
+    if weights_path and os.path.exists(weights_path):
+        from paper_2609_09338_gb300 import checkpoint
+        _, w = checkpoint.load_weights(weights_path, sh)
+    else:
+        w = syn.make_weights(sh, seed)
+        if weights_path and rank == 0:
+            from paper_2609_09338_gb300 import checkpoint
+            checkpoint.save_weights(weights_path, sh, w)
     kv = syn.make_kv_prefix(sh, ctx, wl.n_new + wl.K, seed + 1)
     di = syn.make_draft_inputs(sh, wl.batch, wl.n_new, wl.K, seed + 2)
     vi = syn.make_verify_inputs(sh.vocab, wl.batch, wl.K, wl.temperature, wl.sigma_p, seed + 3)
@@ -189,7 +199,7 @@ def run_reference(args):
     if rank != 0:
         return
     wl = WORKLOADS[args.workload]
-    ctx, w, kv, di, vi = make_inputs(wl)
+    ctx, w, kv, di, vi = make_inputs(wl, 0, args.weights)
     from oracle import drafter as od
     from oracle import verify as ov
     import torch
@@ -309,7 +319,7 @@ def verify_hidden_compare(args):
     if wl.temperature <= 0:
         raise SystemExit("--verify-hidden needs a sampled workload (temperature > 0)")
     sh, B, K, T = wl.shape, wl.batch, wl.K, wl.temperature
-    ctx, w, kv, di, vi = make_inputs(wl)
+    ctx, w, kv, di, vi = make_inputs(wl, 0, args.weights)
     dev = "cuda"
     T_ = lambda a: torch.from_numpy(np.ascontiguousarray(a)).to(dev)
     target = T_(vi["target_logits"]) if wl.logits_dtype == "f32" else \
@@ -400,7 +410,7 @@ def main():
     if args.temperature is not None:
         wl = wl.with_(temperature=args.temperature)
     sh, B, K, T = wl.shape, wl.batch, wl.K, wl.temperature
-    ctx, w, kv, di, vi = make_inputs(wl, rank)
+    ctx, w, kv, di, vi = make_inputs(wl, rank, args.weights)
     dev = "cuda"
     sess = DraftSession(sh, w, kv["page_table"], kv["n_pages"], K, wl.n_new)
     sess.append(ctx, kv["k_rows"], kv["v_rows"])
@@ -464,9 +474,11 @@ def main():
         with torch.cuda.stream(stream):
             for i in range(args.steps):
                 flush()
+                torch.cuda.nvtx.range_push(f"step {i}")
                 starts[i].record(stream)
                 graph.replay()
                 ends[i].record(stream)
+                torch.cuda.nvtx.range_pop()
                 ends[i].synchronize()
                 lm_ms.extend(ob.osprey_probe_read(sess.ctx, K))
         torch.cuda.synchronize()
