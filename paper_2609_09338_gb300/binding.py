@@ -22,6 +22,14 @@ OSPREY_F32, OSPREY_BF16 = 0, 1
 ERRORS = {0: "OK", -1: "INVALID_ARG", -2: "SHAPE", -3: "DTYPE", -4: "CAPACITY", -5: "CUDA", -6: "TIMEOUT"}
 
 
+def status_name(code: int) -> str:
+    """Name of a status code; a bounds-checked build (-DOSP_BOUNDS=1) reports a
+    failed check as -(1000 + source line)."""
+    if code <= -1000:
+        return f"BOUNDS(line {-code - 1000})"
+    return ERRORS.get(code, f"UNKNOWN({code})")
+
+
 class OspreyError(RuntimeError):
     def __init__(self, code: int, msg: str):
         super().__init__(f"osprey error {code} ({ERRORS.get(code, '?')}): {msg}")

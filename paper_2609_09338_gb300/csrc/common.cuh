@@ -208,6 +208,28 @@ __device__ __forceinline__ void set_status(int32_t *status, int code) {
     if (status) atomicCAS((int *)status, 0, code);
 }
 
+// Bounds-checked debug build (nvcc -DOSP_BOUNDS=1, e.g. through
+// OSPREY_NVCC_DEFINES): OSP_BOUNDS_OK(cond, status) is false when cond fails,
+// after writing -(1000 + source line) to the status word (first error wins), and
+// the caller skips the access it guards.  A skipped copy leaves its barrier
+// short, so the bounded wait on it runs out and the kernel returns.  In the
+// default build the macro is the constant true.
+#ifndef OSP_BOUNDS
+#define OSP_BOUNDS 0
+#endif
+#if OSP_BOUNDS
+#define OSP_BOUNDS_OK(cond, status) ((cond) || (::osp::set_status((status), -1000 - __LINE__), false))
+#else
+#define OSP_BOUNDS_OK(cond, status) true
+#endif
+
+// Bytes of dynamic shared memory the running block was launched with.
+__device__ __forceinline__ unsigned dynamic_smem_bytes() {
+    unsigned v;
+    asm("mov.u32 %0, %%dynamic_smem_size;" : "=r"(v));
+    return v;
+}
+
 __device__ __forceinline__ unsigned ld_acquire_gpu(const unsigned *p) {
     unsigned v;
     asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");

@@ -1344,13 +1344,18 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
             const int h = u / half, i = u - h * half;
             const int n = min(u1 - u, half - i);
             const size_t lo = (size_t)h * HD + i;
-            bulk_g2s(wq_lo + (size_t)(u - u0) * 2 * d, a.W_qkv + lo * 2 * d, (uint32_t)n * row_b, &bar[0]);
-            bulk_g2s(wq_hi + (size_t)(u - u0) * 2 * d, a.W_qkv + (lo + half) * 2 * d, (uint32_t)n * row_b, &bar[0]);
+            if (OSP_BOUNDS_OK(u - u0 + n <= p.up && lo + half + n <= (size_t)(D.Hq + 2 * D.Hkv) * HD &&
+                                  p.smem <= dynamic_smem_bytes(),
+                              a.status)) {
+                bulk_g2s(wq_lo + (size_t)(u - u0) * 2 * d, a.W_qkv + lo * 2 * d, (uint32_t)n * row_b, &bar[0]);
+                bulk_g2s(wq_hi + (size_t)(u - u0) * 2 * d, a.W_qkv + (lo + half) * 2 * d, (uint32_t)n * row_b,
+                         &bar[0]);
+            }
             u += n;
         }
         const uint32_t bo = (uint32_t)no * Ko * 2;
         mbar_arrive_expect_tx(&bar[1], bo);
-        if (bo) bulk_g2s(wo, a.W_o + (size_t)o0 * Ko, bo, &bar[1]);
+        if (bo && OSP_BOUNDS_OK(no <= p.ro && o1 <= d, a.status)) bulk_g2s(wo, a.W_o + (size_t)o0 * Ko, bo, &bar[1]);
         issued = 2;
     }
     pdl_trigger();
@@ -1389,11 +1394,13 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
                 } else {
                     const bool is_k = h < D.Hq + D.Hkv;
                     const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
-                    const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
-                    uint16_t *dst = (is_k ? a.k_pages : a.v_pages) +
-                                    (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * HD;
-                    dst[i] = f_to_bf(x1);
-                    dst[i + half] = f_to_bf(x2);
+                    if (OSP_BOUNDS_OK(pos / D.P < a.max_pages, a.status)) {
+                        const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
+                        uint16_t *dst = (is_k ? a.k_pages : a.v_pages) +
+                                        (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * HD;
+                        dst[i] = f_to_bf(x1);
+                        dst[i + half] = f_to_bf(x2);
+                    }
                 }
             }
         }
@@ -1407,7 +1414,7 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
     if (threadIdx.x == 0 && ok) {
         const uint32_t bf = (uint32_t)nf * d * 2;
         mbar_arrive_expect_tx(&bar[2], 2 * bf);
-        if (bf) {
+        if (bf && OSP_BOUNDS_OK(nf <= p.rf && f1 <= F, a.status)) {
             bulk_g2s(wg, a.W_gate + (size_t)f0 * d, bf, &bar[2]);
             bulk_g2s(wu, a.W_up + (size_t)f0 * d, bf, &bar[2]);
         }
@@ -1500,7 +1507,8 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
     if (threadIdx.x == 0 && ok) {
         const uint32_t bd = (uint32_t)no * F * 2;
         mbar_arrive_expect_tx(&bar[3], bd);
-        if (bd) bulk_g2s(wd, a.W_down + (size_t)o0 * F, bd, &bar[3]);
+        if (bd && OSP_BOUNDS_OK((size_t)bd <= p.a_bytes && o1 <= d, a.status))
+            bulk_g2s(wd, a.W_down + (size_t)o0 * F, bd, &bar[3]);
         issued = 4;
     }
     grid_sync(a.bar_count, a.bar_gen, a.status);

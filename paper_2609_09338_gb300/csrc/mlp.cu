@@ -60,15 +60,16 @@ __global__ void __launch_bounds__(MLP_THREADS, 1) mlp_fused_kernel(const MlpArgs
         mbar_fence_init();
         // the weights do not depend on earlier kernels: request them now
         const uint32_t bo = (uint32_t)no * Ko * 2, bf = (uint32_t)nf * d * 2, bd = (uint32_t)no * F * 2;
+        const bool fits = OSP_BOUNDS_OK(p.smem <= dynamic_smem_bytes() && no <= p.ro && nf <= p.rf, a.status);
         mbar_arrive_expect_tx(&bar[0], bo);
-        if (bo) bulk_g2s(wo, a.W_o + (size_t)o0 * Ko, bo, &bar[0]);
+        if (bo && fits) bulk_g2s(wo, a.W_o + (size_t)o0 * Ko, bo, &bar[0]);
         mbar_arrive_expect_tx(&bar[1], 2 * bf);
-        if (bf) {
+        if (bf && fits) {
             bulk_g2s(wg, a.W_gate + (size_t)f0 * d, bf, &bar[1]);
             bulk_g2s(wu, a.W_up + (size_t)f0 * d, bf, &bar[1]);
         }
         mbar_arrive_expect_tx(&bar[2], bd);
-        if (bd) bulk_g2s(wd, a.W_down + (size_t)o0 * F, bd, &bar[2]);
+        if (bd && fits) bulk_g2s(wd, a.W_down + (size_t)o0 * F, bd, &bar[2]);
     }
     pdl_trigger();
     int b, pos;

@@ -103,3 +103,10 @@ def test_logits_free_entry_points_validate_on_host(lib):
     f = ob._c_verify_hidden
     assert f(None, 1, 2, 0, p, p, p, p, p, 1.0, p, p, p, p, p, None, p, 1 << 20, None, None) == -1
     assert ob._c_verify_hidden_ws(None, 1, 2) == 0
+
+
+def test_status_names_cover_bounds_checked_builds(lib):
+    from paper_2609_09338_gb300 import binding as ob
+    assert ob.status_name(0) == "OK" and ob.status_name(-6) == "TIMEOUT"
+    assert ob.status_name(-1342) == "BOUNDS(line 342)"
+    assert ob.status_name(-77).startswith("UNKNOWN")
