@@ -229,6 +229,23 @@ def run_reference(args):
     }))
 
 
+def nvtx_push(name):
+    """An NVTX range for a profiler's timeline; nothing when this torch build has no NVTX."""
+    try:
+        import torch
+        torch.cuda.nvtx.range_push(name)
+    except (RuntimeError, AttributeError):
+        pass
+
+
+def nvtx_pop():
+    try:
+        import torch
+        torch.cuda.nvtx.range_pop()
+    except (RuntimeError, AttributeError):
+        pass
+
+
 def lm_head_label(B):
     """The LM-head launches the probes bracket, by the number of rows (the draft
     step's kernel selection)."""
@@ -474,11 +491,11 @@ def main():
         with torch.cuda.stream(stream):
             for i in range(args.steps):
                 flush()
-                torch.cuda.nvtx.range_push(f"step {i}")
+                nvtx_push(f"step {i}")
                 starts[i].record(stream)
                 graph.replay()
                 ends[i].record(stream)
-                torch.cuda.nvtx.range_pop()
+                nvtx_pop()
                 ends[i].synchronize()
                 lm_ms.extend(ob.osprey_probe_read(sess.ctx, K))
         torch.cuda.synchronize()
