@@ -103,6 +103,8 @@ def emulate(sh, W, pages_k, pages_v, ptab, x, s, pos, grid=152):
 
 
 def run(sh, ctx_len, seed):
+    """Token 3 at position ctx_len after a ctx_len-position paged prefix: the
+    block-by-block model and the oracle's forward_row give the same residual."""
     sh = replace(sh, n_layers=1)
     wb = syn.make_weights(sh, seed)
     W = od.widen_weights(wb)
