@@ -53,12 +53,14 @@ class DraftSession:
 
 
 class VerifyBuffers:
-    def __init__(self, B: int, K: int, V: int, device: str = "cuda"):
+    def __init__(self, B: int, K: int, V: int, device: str = "cuda", workspace_bytes: int | None = None):
         self.out_tokens = torch.zeros((B, K + 1), dtype=torch.int32, device=device)
         self.n_accepted = torch.zeros(B, dtype=torch.int32, device=device)
         self.flags = torch.zeros((B, K + 1), dtype=torch.uint8, device=device)
         self.probs = torch.zeros((B, K, 2), dtype=torch.float32, device=device)
-        self.workspace = torch.zeros(ob.osprey_verify_workspace_bytes(B, K, V), dtype=torch.uint8, device=device)
+        if workspace_bytes is None:
+            workspace_bytes = ob.osprey_verify_workspace_bytes(B, K, V)
+        self.workspace = torch.zeros(workspace_bytes, dtype=torch.uint8, device=device)
         self.status = torch.zeros(1, dtype=torch.int32, device=device)
 
     def run(self, target, draft, tokens, temperature, u_accept, u_sample, stream=None):
@@ -70,10 +72,8 @@ class VerifyHiddenBuffers(VerifyBuffers):
     """Outputs and workspace of the logits-free verify for one drafter context."""
 
     def __init__(self, ctx: "ob.Ctx", B: int, K: int, device: str = "cuda"):
-        super().__init__(B, K, ctx.shape.vocab, device)
+        super().__init__(B, K, ctx.shape.vocab, device, ob.osprey_verify_hidden_workspace_bytes(ctx, B, K))
         self.ctx = ctx
-        self.workspace = torch.zeros(ob.osprey_verify_hidden_workspace_bytes(ctx, B, K), dtype=torch.uint8,
-                                     device=device)
 
     def run_hidden(self, target, hidden, qx, stats, tokens, temperature, u_accept, u_sample, stream=None):
         ob.osprey_verify_hidden(self.ctx, target, hidden, qx, stats, tokens, temperature, u_accept, u_sample,
