@@ -5,11 +5,15 @@ drafter, LM head sampled on chip) + one osprey_verify over the workload's
 synthetic target/draft logits, captured in one CUDA graph.  Inputs are seeded
 synthetic data shaped like the workload (weights bf16 ~ N(0, 0.02^2)).
 
-Default workload: Qwen3-8B-shaped drafter (d=1024, 1 layer, 16/8 heads, hd 128,
-FFN 3072, vocab 151936), batch 1, K=7, context 2048, temperature 1.
+Default workload: the large-vocabulary drafter (d=1024, 1 layer, 16/8 heads of
+128, FFN 3072, vocab 200064, 3 x 3072 feature columns), batch 64, K=8, ragged
+paged contexts U[1024, 16384], temperature 1, float32 logits: the largest
+single-GPU workload.  The other workloads are measured after it under
+"other_workloads" (--no-extra skips them).
 
 Prints ONE JSON line (rank 0).  ``--impl reference`` times the CPU oracle on
-the same workload instead (a deliberately slow float64 program).
+the same workload instead (a deliberately slow float64 program), on a bounded
+sample of sequences per step.
 """
 from __future__ import annotations
 
@@ -61,7 +65,13 @@ def parse():
                         "else write the seeded weights there")
     p.add_argument("--verify-hidden", action="store_true",
                    help="compare draft (logits written) + verify against draft (states kept) + logits-free verify")
+    p.add_argument("--no-extra", action="store_true", help="measure the headline workload only")
     return p.parse_args()
+
+
+# measured after the headline workload, each with its own dominant kernel
+EXTRA_WORKLOADS = ["qwen3-8b-d1024-v151936-b1-k7", "qwen3-8b-d1024-v151936-b32-k7",
+                   "llama70b-d2048-v128256-b16-k7", "osprey-d2560-v151936-b1-k7-ext3"]
 
 
 def make_inputs(wl, rank=0, weights_path=None):
@@ -83,7 +93,11 @@ def make_inputs(wl, rank=0, weights_path=None):
 
 
 def algorithmic_bytes(wl, ctx):
-    """Bytes the method must touch per step (no L2 reuse credited)."""
+    """Bytes the method must touch per step (no L2 reuse credited).
+
+    attn_call: the K/V bytes of every attention launch of one draft call (chain
+    step k of sequence b reads its ctx_b + n_new + k cached positions, K and V,
+    bf16, for each of the L layers), over the K * L launches of the call."""
     sh = wl.shape
     B, K = wl.batch, wl.K
     w_step = sh.weight_bytes_per_step()
@@ -94,7 +108,14 @@ def algorithmic_bytes(wl, ctx):
     s = 4 if wl.logits_dtype == "f32" else 2
     verify = B * (K + 1) * sh.vocab * s + B * K * sh.vocab * s
     lm_launch = sh.vocab * sh.d_model * 2 * 1 + 2 * sh.d_model
-    return {"draft": draft, "verify": verify, "lm_head_launch": lm_launch}
+    return {"draft": draft, "verify": verify, "lm_head_launch": lm_launch, "attn_call": kv,
+            "attn_launches": K * sh.n_layers, "lm_launches": K,
+            "verify_f32": B * (2 * K + 1) * sh.vocab * 4, "verify_bf16": B * (2 * K + 1) * sh.vocab * 2}
+
+
+def dominant_kernel(nb):
+    """The kernel class with the most algorithmic bytes per draft call."""
+    return "attention" if nb["attn_call"] > nb["lm_head_launch"] * nb["lm_launches"] else "lm_head"
 
 
 class ClockSampler:
@@ -158,29 +179,82 @@ def peaks():
         return 6800.0, "fallback"
 
 
-def cpu_baseline(wl, ctx, w, kv, di, vi, budget_s=10.0):
-    """The oracle as it stands on the host cores: whole steps of the same workload."""
-    import torch
+def _blas():
+    """numpy's OpenBLAS (get, set) thread-count functions, or None."""
+    import ctypes
+    np.ones((64, 64)) @ np.ones((64, 64))   # make sure the library is loaded
+    try:
+        with open("/proc/self/maps") as f:
+            libs = sorted({ln.split()[-1] for ln in f if "openblas" in ln.lower() and ".so" in ln.split()[-1]})
+    except OSError:
+        return None
+    for path in libs:
+        try:
+            lib = ctypes.CDLL(path)
+        except OSError:
+            continue
+        for suffix in ("64_", "", "_64"):
+            for pre in ("scipy_openblas", "openblas"):
+                try:
+                    get = getattr(lib, f"{pre}_get_num_threads{suffix}")
+                    put = getattr(lib, f"{pre}_set_num_threads{suffix}")
+                except AttributeError:
+                    continue
+                get.restype = ctypes.c_int
+                put.argtypes = [ctypes.c_int]
+                return get, put
+    return None
+
+
+def oracle_sequence_step(wl, ctx, w, W, kv, di, vi, b):
+    """One sequence's share of a step, run by the oracle: its draft call (extend
+    rows + K-token chain) and its verification."""
     from oracle import drafter as od
     from oracle import verify as ov
+    offs = np.concatenate([[0], np.cumsum(ctx)]).astype(np.int64)
+    sl = slice(int(offs[b]), int(offs[b + 1]))
+    od.draft_step(w, wl.shape, kv["k_rows"][:, sl], kv["v_rows"][:, sl], ctx[b:b + 1], di["tokens"][b:b + 1],
+                  di["feats"][b:b + 1], di["n_new"][b:b + 1], wl.K, wl.temperature, di["u_draft"][b:b + 1],
+                  widened=W)
+    ov.verify(vi["target_logits"][b:b + 1], vi["draft_logits"][b:b + 1], vi["draft_tokens"][b:b + 1],
+              wl.temperature, vi["u_accept"][b:b + 1], vi["u_sample"][b:b + 1])
+
+
+def cpu_baseline(wl, ctx, w, kv, di, vi, budget_s=8.0):
+    """The oracle as it stands on the host cores, on a bounded sample: whole
+    sequences of the workload (draft call + verify of one sequence), scaled to
+    steps/s as 1 / (B x mean seconds per sequence).  Timed with numpy's BLAS at
+    its own thread count and again at one thread."""
+    from oracle import drafter as od
     t0 = time.perf_counter()
     W = od.widen_weights(w)
     setup = time.perf_counter() - t0
-    n, t_run = 0, 0.0
-    while True:
-        t1 = time.perf_counter()
-        od.draft_step(w, wl.shape, kv["k_rows"], kv["v_rows"], ctx, di["tokens"], di["feats"], di["n_new"], wl.K,
-                      wl.temperature, di["u_draft"], widened=W)
-        ov.verify(vi["target_logits"], vi["draft_logits"], vi["draft_tokens"], wl.temperature, vi["u_accept"],
-                  vi["u_sample"])
-        t_run += time.perf_counter() - t1
-        n += 1
-        if t_run > budget_s or n >= 50:
-            break
-    cores = torch.get_num_threads()
-    return {"value": n / t_run, "unit": "steps/s", "cores": cores, "kind": "oracle",
-            "sample": f"{n} full step(s) (draft K={wl.K} + verify) of {wl.name}, float64 numpy; "
-                      f"weights widened once ({setup:.1f}s, untimed); {os.cpu_count()} host cores visible"}
+    blas = _blas()
+    threads = blas[0]() if blas else None
+
+    def sample(budget):
+        n, t_run = 0, 0.0
+        while True:
+            b = n % wl.batch
+            t1 = time.perf_counter()
+            oracle_sequence_step(wl, ctx, w, W, kv, di, vi, b)
+            t_run += time.perf_counter() - t1
+            n += 1
+            if t_run > budget or n >= 4 * wl.batch:
+                return n, t_run
+    n, t_run = sample(budget_s)
+    res = {"value": n / t_run / wl.batch, "unit": "steps/s", "cores": threads, "kind": "oracle",
+           "sample": f"{n} sequence(s) of {wl.name} (draft call K={wl.K} + verify each, float64 numpy), "
+                     f"scaled to steps of {wl.batch} sequences; weights widened once ({setup:.1f}s, untimed); "
+                     f"cores = numpy BLAS threads; {os.cpu_count()} host cores visible"}
+    if blas and threads and threads > 1:
+        blas[1](1)
+        try:
+            n1, t1 = sample(budget_s / 2)
+        finally:
+            blas[1](threads)
+        res["one_core"] = {"value": n1 / t1 / wl.batch, "cores": 1, "sample": f"{n1} sequence(s)"}
+    return res
 
 
 def max_over_ranks(x: float, world: int, device="cpu") -> float:
@@ -201,30 +275,31 @@ def run_reference(args):
     wl = WORKLOADS[args.workload]
     ctx, w, kv, di, vi = make_inputs(wl, 0, args.weights)
     from oracle import drafter as od
-    from oracle import verify as ov
-    import torch
     W = od.widen_weights(w)
+    blas = _blas()
+    cores = blas[0]() if blas else None
+    # one step of the reference arm is a bounded sample of the workload: up to
+    # ``per`` of its sequences (draft call + verify each), scaled to whole steps
+    per = max(1, min(wl.batch, 2))
 
-    def step():
-        od.draft_step(w, wl.shape, kv["k_rows"], kv["v_rows"], ctx, di["tokens"], di["feats"], di["n_new"], wl.K,
-                      wl.temperature, di["u_draft"], widened=W)
-        ov.verify(vi["target_logits"], vi["draft_logits"], vi["draft_tokens"], wl.temperature, vi["u_accept"],
-                  vi["u_sample"])
-    for _ in range(args.warmup):
-        step()
+    def step(i):
+        for j in range(per):
+            oracle_sequence_step(wl, ctx, w, W, kv, di, vi, (i * per + j) % wl.batch)
+    for i in range(args.warmup):
+        step(i)
     t0 = time.perf_counter()
-    for _ in range(args.steps):
-        step()
+    for i in range(args.steps):
+        step(args.warmup + i)
     dt = time.perf_counter() - t0
-    v = args.steps / dt
-    cores = torch.get_num_threads()
+    v = args.steps * per / wl.batch / dt
+    sample = (f"each step: {per} of the {wl.batch} sequences of {wl.name} (draft call K={wl.K} + verify), "
+              f"scaled to steps/s as sequences / {wl.batch}; float64 numpy; cores = numpy BLAS threads")
     print(json.dumps({
         "impl": "reference", "metric": "draft+verify steps/s", "value": v, "unit": "steps/s", "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * dt / args.steps, "higher_is_better": True,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 / v, "higher_is_better": True,
         "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
         "config": config_of(wl, ctx),
-        "cpu_baseline": {"value": v, "unit": "steps/s", "cores": cores, "kind": "oracle",
-                         "sample": f"whole steps of {wl.name} on the host cores"},
+        "cpu_baseline": {"value": v, "unit": "steps/s", "cores": cores, "kind": "oracle", "sample": sample},
         "e2e": {"value": v, "unit": "steps/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }))
 
@@ -402,32 +477,19 @@ def verify_hidden_compare(args):
                       "decision_row_lm_bytes": -(-B // 80) * sh.vocab * sh.d_model * 2 + B * sh.vocab * s_}))
 
 
-def main():
-    args = parse()
-    if args.impl == "reference":
-        return run_reference(args)
-    if args.verify_sweep:
-        return verify_sweep(args)
-    if args.verify_hidden:
-        return verify_hidden_compare(args)
+def measure(wl, args, rank, world, local, full):
+    """Time `args.steps` draft+verify steps of one workload (graph replays, L2
+    flushed before each).  With ``full``: also verify alone (float32 and bf16
+    logits), the end-to-end form from pinned host memory, clocks and the CPU
+    baseline."""
     import torch
-    import torch.distributed as dist
-    world = int(os.environ.get("WORLD_SIZE", "1"))
-    rank = int(os.environ.get("RANK", "0"))
-    local = int(os.environ.get("LOCAL_RANK", "0"))
-    torch.cuda.set_device(local)
-    if world > 1:
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
-    import __graft_entry__
-    __graft_entry__.build()
     from paper_2609_09338_gb300 import binding as ob
     from paper_2609_09338_gb300.session import DraftSession, VerifyBuffers
 
-    wl = WORKLOADS[args.workload]
-    if args.temperature is not None:
-        wl = wl.with_(temperature=args.temperature)
     sh, B, K, T = wl.shape, wl.batch, wl.K, wl.temperature
-    ctx, w, kv, di, vi = make_inputs(wl, rank, args.weights)
+    ctx, w, kv, di, vi = make_inputs(wl, rank, args.weights if full else None)
+    nb = algorithmic_bytes(wl, ctx)
+    dom = dominant_kernel(nb)
     dev = "cuda"
     sess = DraftSession(sh, w, kv["page_table"], kv["n_pages"], K, wl.n_new)
     sess.append(ctx, kv["k_rows"], kv["v_rows"])
@@ -445,9 +507,11 @@ def main():
     v_in.update({"tokens": T_(vi["draft_tokens"]), "u_accept": T_(vi["u_accept"]), "u_sample": T_(vi["u_sample"])})
     out = sess.draft_buffers()
     vb = VerifyBuffers(B, K, sh.vocab)
-    ob.osprey_probe_enable(sess.ctx, K)
+    n_probe = nb["attn_launches"] if dom == "attention" else nb["lm_launches"]
+    ob.osprey_probe_select(sess.ctx, ob.PROBE_ATTENTION if dom == "attention" else ob.PROBE_LM_HEAD)
+    ob.osprey_probe_enable(sess.ctx, n_probe)
     stream = torch.cuda.Stream()
-    stream.wait_stream(torch.cuda.current_stream())   # inputs, buffers and zeroed workspaces first
+    stream.wait_stream(torch.cuda.current_stream())   # inputs and buffers first
 
     def step():
         sess.kv.seq_len.copy_(seq0)
@@ -481,8 +545,9 @@ def main():
 
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    lm_ms = []
+    probe_ms = []
     if world > 1:
+        import torch.distributed as dist
         dist.barrier()
     torch.cuda.synchronize()
     clk_file = tempfile.NamedTemporaryFile(prefix=f"osprey_clocks_{rank}_", suffix=".csv", delete=False)
@@ -497,7 +562,7 @@ def main():
                 ends[i].record(stream)
                 nvtx_pop()
                 ends[i].synchronize()
-                lm_ms.extend(ob.osprey_probe_read(sess.ctx, K))
+                probe_ms.append(ob.osprey_probe_read(sess.ctx, n_probe))
         torch.cuda.synchronize()
     clocks = clk.summary()
     try:
@@ -506,23 +571,65 @@ def main():
         pass
     if world > 1:
         dist.barrier()
-    step_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    assert int(sess.status.item()) == 0 and int(vb.status.item()) == 0
+    step_ms = [s_.elapsed_time(e_) for s_, e_ in zip(starts, ends)]
     ms = max_over_ranks(sum(step_ms) / len(step_ms), world, dev)
+    peak, peak_kind = peaks()
+    acc = vb.n_accepted.float()
+    if dom == "attention":
+        # bytes of all the call's attention launches / their summed duration
+        call_ms = sum(sum(p) for p in probe_ms) / len(probe_ms)
+        achieved = nb["attn_call"] / (call_ms * 1e-3) / 1e9
+        roof = {"kernel": "split-KV GQA decode attention (attn_kernel / attn_cluster_kernel), all launches of a call",
+                "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
+                "traffic": None, "peak_kind": peak_kind,
+                "bytes_per_launch": nb["attn_call"] / nb["attn_launches"],
+                "mean_launch_us": 1e3 * call_ms / nb["attn_launches"], "launches_timed": len(probe_ms) * n_probe}
+    else:
+        lm = [x for p in probe_ms for x in p]
+        lm_mean_ms = sum(lm) / len(lm)
+        achieved = nb["lm_head_launch"] / (lm_mean_ms * 1e-3) / 1e9
+        sha = _sha(os.path.join(ROOT, LM_TRAFFIC["source"]))
+        roof = {"kernel": lm_head_label(B), "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                "frac": achieved / peak,
+                "traffic": LM_TRAFFIC["bytes_per_launch"] if LM_TRAFFIC["sha256"] == sha and B <= 2 else None,
+                "peak_kind": peak_kind, "bytes_per_launch": nb["lm_head_launch"], "mean_launch_us": lm_mean_ms * 1e3,
+                "launches_timed": len(lm)}
+    res = {"ms_per_step": ms, "steps_per_s": world * 1e3 / ms, "drafted_tokens_per_s": world * B * K * 1e3 / ms,
+           "draft_step_bytes": nb["draft"], "verify_bytes": nb["verify"],
+           "step_hbm_frac": (nb["draft"] + nb["verify"]) / (ms * 1e-3) / 1e9 / peak,
+           "synthetic_al": float(acc.mean().item()) + 1.0, "synthetic_al_sequences": B,
+           "roofline": roof, "launches_per_step": launches_per_step, "clocks": clocks, "config": config_of(wl, ctx)}
+    if not full:
+        del sess, vb, graph
+        return res
 
-    # verify alone (same inputs, L2 flushed): verify GB/s
-    vgraph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(vgraph, stream=stream):
-        vb.run(v_in["target"], v_in["draft"] if T > 0 else None, v_in["tokens"], T, v_in["u_accept"], v_in["u_sample"])
-    vs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    ve = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
-    with torch.cuda.stream(stream):
-        for i in range(args.steps):
-            flush()
-            vs[i].record(stream)
-            vgraph.replay()
-            ve[i].record(stream)
-    torch.cuda.synchronize()
-    v_ms = sum(s.elapsed_time(e) for s, e in zip(vs, ve)) / args.steps
+    # verify alone (same inputs, L2 flushed): verify GB/s in the workload's dtype and in bf16
+    def time_verify(tgt, drf):
+        vgraph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(vgraph, stream=stream):
+            vb.run(tgt, drf if T > 0 else None, v_in["tokens"], T, v_in["u_accept"], v_in["u_sample"])
+        vs = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 3)]
+        ve = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps + 3)]
+        with torch.cuda.stream(stream):
+            for i in range(args.steps + 3):
+                flush()
+                vs[i].record(stream)
+                vgraph.replay()
+                ve[i].record(stream)
+        torch.cuda.synchronize()
+        assert int(vb.status.item()) == 0
+        return sum(s_.elapsed_time(e_) for s_, e_ in zip(vs[3:], ve[3:])) / args.steps
+    v_ms = time_verify(v_in["target"], v_in["draft"])
+    tb, db = v_in["target"].to(torch.bfloat16), v_in["draft"].to(torch.bfloat16)
+    vbf_ms = time_verify(tb, db)
+    del tb, db
+    res["verify_us"] = v_ms * 1e3
+    res["verify_gbs"] = nb["verify"] / (v_ms * 1e-3) / 1e9
+    res["verify_frac"] = res["verify_gbs"] / peak
+    res["verify_bf16_us"] = vbf_ms * 1e3
+    res["verify_bf16_gbs"] = nb["verify_bf16"] / (vbf_ms * 1e-3) / 1e9
+    res["verify_bf16_frac"] = res["verify_bf16_gbs"] / peak
 
     # end to end: inputs from pinned host memory, results back to the host
     h_in = {k: v.cpu().pin_memory() for k, v in {**d_in, **v_in}.items()}
@@ -544,42 +651,68 @@ def main():
             h_out["n_accepted"].copy_(vb.n_accepted, non_blocking=True)
             ee[i].record(stream)
     torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(sum(s.elapsed_time(e) for s, e in zip(es, ee)) / args.steps, world, dev)
-    h2d = sum(v.numel() * v.element_size() for v in h_in.values())
-    d2h = sum(v.numel() * v.element_size() for v in h_out.values())
+    e2e_ms = max_over_ranks(sum(s_.elapsed_time(e_) for s_, e_ in zip(es, ee)) / args.steps, world, dev)
+    res["e2e"] = {"value": world * 1e3 / e2e_ms, "unit": "steps/s",
+                  "h2d_bytes_per_step": sum(v.numel() * v.element_size() for v in h_in.values()),
+                  "d2h_bytes_per_step": sum(v.numel() * v.element_size() for v in h_out.values())}
+    res["gpu_launches"] = launches_per_step * args.steps
+    if rank == 0 and not args.no_cpu_baseline:
+        res["cpu_baseline"] = cpu_baseline(wl, ctx, w, kv, di, vi)
+    del sess, vb, graph, h_in
+    return res
 
-    nb = algorithmic_bytes(wl, ctx)
-    peak, peak_kind = peaks()
-    lm_mean_ms = sum(lm_ms) / len(lm_ms)
-    lm_gbs = nb["lm_head_launch"] / (lm_mean_ms * 1e-3) / 1e9
-    sha = _sha(os.path.join(ROOT, LM_TRAFFIC["source"]))
-    traffic = LM_TRAFFIC["bytes_per_launch"] if LM_TRAFFIC["sha256"] == sha else None
-    acc_len = float(vb.n_accepted.float().mean().item()) + 1.0
 
+def main():
+    args = parse()
+    if args.impl == "reference":
+        return run_reference(args)
+    if args.verify_sweep:
+        return verify_sweep(args)
+    if args.verify_hidden:
+        return verify_hidden_compare(args)
+    import torch
+    import torch.distributed as dist
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    import __graft_entry__
+    __graft_entry__.build()
+
+    wl = WORKLOADS[args.workload]
+    if args.temperature is not None:
+        wl = wl.with_(temperature=args.temperature)
+    r = measure(wl, args, rank, world, local, full=True)
+    torch.cuda.empty_cache()
+    others = {}
+    if not args.no_extra and world == 1:
+        for name in EXTRA_WORKLOADS:
+            if name == wl.name:
+                continue
+            o = measure(WORKLOADS[name], args, rank, world, local, full=False)
+            torch.cuda.empty_cache()
+            others[name] = {k: o[k] for k in ("ms_per_step", "steps_per_s", "step_hbm_frac", "synthetic_al",
+                                              "launches_per_step")}
+            others[name]["roofline"] = {k: o["roofline"][k] for k in ("kernel", "achieved", "frac",
+                                                                      "mean_launch_us")}
+            others[name]["clocks"] = o["clocks"]
     if rank == 0:
         res = {
-            "metric": "draft+verify steps/s", "value": world * 1e3 / ms, "unit": "steps/s", "n_gpus": world,
-            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "metric": "draft+verify steps/s", "value": r["steps_per_s"], "unit": "steps/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": r["ms_per_step"], "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
-            "config": config_of(wl, ctx),
-            "drafted_tokens_per_s": world * B * K * 1e3 / ms,
-            "verify_gbs": nb["verify"] / (v_ms * 1e-3) / 1e9,
-            "verify_us": v_ms * 1e3,
-            "draft_step_bytes": nb["draft"],
-            "step_hbm_frac": (nb["draft"] + nb["verify"]) / (ms * 1e-3) / 1e9 / peak,
-            "synthetic_al": acc_len,
-            "roofline": {"kernel": lm_head_label(B),
-                         "bound": "hbm", "achieved": lm_gbs, "peak": peak, "unit": "GB/s",
-                         "frac": lm_gbs / peak, "traffic": traffic, "peak_kind": peak_kind,
-                         "bytes_per_launch": nb["lm_head_launch"], "mean_launch_us": lm_mean_ms * 1e3,
-                         "launches_timed": len(lm_ms)},
-            "e2e": {"value": world * 1e3 / e2e_ms, "unit": "steps/s", "h2d_bytes_per_step": h2d,
-                    "d2h_bytes_per_step": d2h},
-            "gpu_launches": launches_per_step * args.steps,
-            "clocks": clocks,
+            "config": r["config"],
+            **{k: r[k] for k in ("drafted_tokens_per_s", "verify_gbs", "verify_us", "verify_frac", "verify_bf16_gbs",
+                                 "verify_bf16_us", "verify_bf16_frac", "draft_step_bytes", "step_hbm_frac",
+                                 "synthetic_al", "synthetic_al_sequences", "roofline", "e2e", "gpu_launches",
+                                 "clocks")},
         }
-        if not args.no_cpu_baseline:
-            res["cpu_baseline"] = cpu_baseline(wl, ctx, w, kv, di, vi)
+        if "cpu_baseline" in r:
+            res["cpu_baseline"] = r["cpu_baseline"]
+        if others:
+            res["other_workloads"] = others
         print(json.dumps(res))
     if world > 1:
         dist.destroy_process_group()

@@ -28,9 +28,11 @@
  *     `dev_status` word (first error wins; it is never cleared by the library:
  *     the caller zeroes it).  The affected sequence's outputs are filled with
  *     -1 / 0 and the other sequences are unaffected.
- *   - A workspace must be zero-filled once before its first use (the kernels
- *     leave their counters at zero again when they finish).  A workspace must
- *     not be shared by calls that can run at the same time.
+ *   - A workspace needs no initialisation: every call clears the arrival
+ *     counters it uses, on its stream, before the kernels that count (the
+ *     draft step in its first kernel, verification with a memset), so a call
+ *     that ran out of a bounded wait leaves nothing stale for the next one.  A
+ *     workspace must not be shared by calls that can run at the same time.
  *   - bf16 is IEEE-754 binary32 truncated to its top 16 bits (round to nearest
  *     even by the producer); all row-major, no padding.
  */
@@ -199,8 +201,7 @@ size_t osprey_verify_hidden_workspace_bytes(const osprey_ctx *ctx, int B, int K)
  *          float: as written by osprey_draft_step_hidden at the same T
  *   draft_tokens, u_accept, u_sample, out_tokens, n_accepted, flags, probs:
  *          as osprey_verify (probs' q column is draft_qx)
- *   workspace: osprey_verify_hidden_workspace_bytes(ctx, B, K) bytes, zeroed
- *          before the first call (its arrival counters return to zero)
+ *   workspace: osprey_verify_hidden_workspace_bytes(ctx, B, K) bytes
  * Host errors: INVALID_ARG (null pointer, T <= 0), SHAPE (the context has no
  * tensor-core path: OSPREY_TC=0 or a device without tcgen05), CAPACITY. */
 int osprey_verify_hidden(osprey_ctx *ctx, int B, int K, int logits_dtype, const void *target_logits,
@@ -250,15 +251,17 @@ int osprey_verify(int B, int K, int V, int logits_dtype, const void *target_logi
  * that the library keeps in device global memory (every GPU that loads the
  * library holds it until the process exits).
  *   - It allocates nothing: no cudaMalloc/cudaFree, no allocating library call.
- *   - The first call on a device looks up the array's device address (a one-time
- *     set-up per device, done with that device current); make that first call
+ *   - The first call on a device may load the library's device code into the
+ *     current context (the runtime does this lazily); make that first call
  *     before any stream capture.
  *   - Requests whose scratch would exceed the array (see
  *     osprey_verify_workspace_bytes) return OSPREY_ERR_CAPACITY with a message.
  *   - All calls share the one array: calls whose work can overlap on the GPU
  *     (different streams, or different host threads) race and must be
  *     serialised by the caller.  The counters that must start at zero are
- *     cleared on the call's stream before its kernels run. */
+ *     cleared on the call's stream before its kernels run.
+ *   - The array's device address is looked up (cudaGetSymbolAddress, which
+ *     allocates nothing) with the caller's device current on every call. */
 #define OSPREY_VERIFY_STATIC_SCRATCH_BYTES (4u << 20)
 int osprey_verify_static(int B, int K, int V, int logits_dtype, const void *target_logits,
                          const void *draft_logits, const int32_t *draft_tokens, float temperature,
@@ -269,11 +272,17 @@ int osprey_verify_static(int B, int K, int V, int logits_dtype, const void *targ
 /* ---- measurement hooks (not part of the method) ------------------------------
  * osprey_probe_enable: make n_slots pairs of timing events in the context (n = 0
  * releases them).  While enabled, osprey_draft_step records pair k around its
- * k-th LM-head launch (k < n_slots), also under stream capture (as external
- * event nodes).  osprey_probe_read writes the elapsed milliseconds of the first
- * n pairs after the caller has synchronised.  osprey_launch_count: kernels the
- * library has launched (or captured) in this process. */
+ * k-th launch of the selected kernel (k < n_slots), also under stream capture
+ * (as external event nodes).  osprey_probe_select picks that kernel:
+ * OSPREY_PROBE_LM_HEAD (the default; pair k = chain step k's LM head) or
+ * OSPREY_PROBE_ATTENTION (pair step * n_layers + layer = that attention launch;
+ * none where a fused layer kernel runs the attention).  osprey_probe_read
+ * writes the elapsed milliseconds of the first n pairs after the caller has
+ * synchronised.  osprey_launch_count: kernels the library has launched (or
+ * captured) in this process. */
+enum { OSPREY_PROBE_LM_HEAD = 0, OSPREY_PROBE_ATTENTION = 1 };
 int osprey_probe_enable(osprey_ctx *ctx, int n_slots);
+int osprey_probe_select(osprey_ctx *ctx, int kind);
 int osprey_probe_read(osprey_ctx *ctx, float *ms, int n);
 int64_t osprey_launch_count(void);
 

@@ -127,13 +127,16 @@ class _SeqCache:
 
 
 def forward_row(W: dict, shape, cache: _SeqCache, token: int, s: np.ndarray, pos: int,
-                new_k: list, new_v: list, forced=None) -> np.ndarray:
+                new_k: list, new_v: list, forced=None, new_mag: list | None = None) -> np.ndarray:
     """One drafter position through every layer; returns x_L (pre final norm).
 
     new_k/new_v receive the rows this computation produces.  With ``forced`` =
     (k [L, Hkv, hd], v [L, Hkv, hd]) the cache holds those rows instead (another
     run's cached values at this position), so attention reads the same cache
-    state as that run."""
+    state as that run.  ``new_mag`` (optional, per layer a list) receives for
+    each new row the pair (k_mag, v_mag): sum_j |W~_ij| |u_j| of the projection
+    that made each element (for a rotated key, summed over the two elements
+    of its rotation pair), the scale of a rounding error in that element."""
     Hq, Hkv, hd = shape.n_q_heads, shape.n_kv_heads, shape.head_dim
     eps, theta = shape.rms_eps, shape.rope_theta
     x = W["embed"][token].copy()
@@ -143,6 +146,11 @@ def forward_row(W: dict, shape, cache: _SeqCache, token: int, s: np.ndarray, pos
         q = qkv[: Hq * hd].reshape(Hq, hd)
         k = qkv[Hq * hd: (Hq + Hkv) * hd].reshape(Hkv, hd)
         v = qkv[(Hq + Hkv) * hd:].reshape(Hkv, hd)
+        if new_mag is not None:
+            mag = np.abs(W["W_qkv"][l]) @ np.abs(np.concatenate([s, z]))
+            km = mag[Hq * hd: (Hq + Hkv) * hd].reshape(Hkv, hd)
+            pair = km[:, : hd // 2] + km[:, hd // 2:]
+            new_mag[l].append((np.concatenate([pair, pair], axis=-1), mag[(Hq + Hkv) * hd:].reshape(Hkv, hd)))
         q, k = rope(q, pos, theta), round_to_bf16(rope(k, pos, theta))
         v = round_to_bf16(v)
         assert cache.length(l) == pos, "positions must be contiguous"
@@ -215,8 +223,9 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
     chain.)
 
     Returns logits [B, K, V], tokens/qx [B, K], stats [B, K, 2], margins [B, K],
-    new_k/new_v: per sequence [L, n_new + K - 1, Hkv, hd], and g [B, d] (the
-    last row's x_L).
+    new_k/new_v: per sequence [L, n_new + K - 1, Hkv, hd] (with new_k_mag /
+    new_v_mag of the same shape: the error scale of each element, see
+    forward_row), and g [B, d] (the last row's x_L).
     """
     W = widened if widened is not None else widen_weights(weights)
     B, V, L = len(ctx_lens), shape.vocab, shape.n_layers
@@ -224,7 +233,7 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
     out = {
         "logits": np.zeros((B, K, V)), "tokens": np.zeros((B, K), np.int64),
         "qx": np.zeros((B, K)), "stats": np.zeros((B, K, 2)), "margins": np.zeros((B, K)),
-        "new_k": [], "new_v": [], "g": np.zeros((B, shape.d_model)),
+        "new_k": [], "new_v": [], "new_k_mag": [], "new_v_mag": [], "g": np.zeros((B, shape.d_model)),
     }
     for b in range(B):
         L0 = int(ctx_lens[b])
@@ -232,6 +241,7 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
                           [widen(prefix_v[l, offs[b]:offs[b + 1]]) for l in range(L)])
         new_k = [[] for _ in range(L)]
         new_v = [[] for _ in range(L)]
+        new_mag = [[] for _ in range(L)]
         nb = int(n_new[b])
         fk = None if forced_kv is None else forced_kv[b]
 
@@ -240,7 +250,7 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
 
         for j in range(nb):
             c = feature_projection(W["W_c"], widen(feats[b, j]))
-            g = forward_row(W, shape, cache, int(tokens[b, j]), c, L0 + j, new_k, new_v, fr(j))
+            g = forward_row(W, shape, cache, int(tokens[b, j]), c, L0 + j, new_k, new_v, fr(j), new_mag)
         for k in range(K):
             h = rmsnorm(g, W["final_norm"], shape.rms_eps)
             z = W["lm_head"] @ h
@@ -253,8 +263,10 @@ def draft_step(weights: dict, shape, prefix_k: np.ndarray, prefix_v: np.ndarray,
             if k == K - 1:
                 break
             nxt = int(forced_tokens[b, k]) if forced_tokens is not None else smp["token"]
-            g = forward_row(W, shape, cache, nxt, g, L0 + nb + k, new_k, new_v, fr(nb + k))
+            g = forward_row(W, shape, cache, nxt, g, L0 + nb + k, new_k, new_v, fr(nb + k), new_mag)
         out["g"][b] = g
         out["new_k"].append(np.asarray(new_k))
         out["new_v"].append(np.asarray(new_v))
+        out["new_k_mag"].append(np.asarray([[m[0] for m in ml] for ml in new_mag]))
+        out["new_v_mag"].append(np.asarray([[m[1] for m in ml] for ml in new_mag]))
     return out

@@ -93,6 +93,7 @@ _c_verify_static = _sig("osprey_verify_static", ctypes.c_int,
                         [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
                          _vp, _vp, _vp, _vp, _vp])
 _c_probe_enable = _sig("osprey_probe_enable", ctypes.c_int, [_vp, ctypes.c_int])
+_c_probe_select = _sig("osprey_probe_select", ctypes.c_int, [_vp, ctypes.c_int])
 _c_probe_read = _sig("osprey_probe_read", ctypes.c_int, [_vp, ctypes.POINTER(_f32), ctypes.c_int])
 _c_launch_count = _sig("osprey_launch_count", _i64, [])
 _c_selftest_wait = _sig("osprey_selftest_wait_timeout", ctypes.c_int, [_i64, _vp, _vp])
@@ -100,7 +101,7 @@ _c_selftest_wait = _sig("osprey_selftest_wait_timeout", ctypes.c_int, [_i64, _vp
 EXPORTED = ["osprey_last_error", "osprey_create", "osprey_destroy", "osprey_draft_workspace_bytes",
             "osprey_kv_append", "osprey_draft_step", "osprey_draft_step_hidden", "osprey_verify_workspace_bytes",
             "osprey_verify", "osprey_verify_static", "osprey_verify_hidden_workspace_bytes", "osprey_verify_hidden",
-            "osprey_probe_enable", "osprey_probe_read", "osprey_launch_count", "osprey_selftest_wait_timeout"]
+            "osprey_probe_enable", "osprey_probe_select", "osprey_probe_read", "osprey_launch_count", "osprey_selftest_wait_timeout"]
 
 
 def osprey_last_error() -> str:
@@ -408,6 +409,13 @@ def osprey_verify_static(target_logits: torch.Tensor, draft_logits, draft_tokens
 
 def osprey_probe_enable(ctx: Ctx, n_slots: int):
     _check(_c_probe_enable(ctx.handle, n_slots))
+
+
+PROBE_LM_HEAD, PROBE_ATTENTION = 0, 1
+
+
+def osprey_probe_select(ctx: Ctx, kind: int):
+    _check(_c_probe_select(ctx.handle, kind))
 
 
 def osprey_probe_read(ctx: Ctx, n: int) -> list:

@@ -54,6 +54,7 @@ struct osprey_ctx {
         tm_up[OSPREY_MAX_LAYERS], tm_down[OSPREY_MAX_LAYERS];
     double inv_freq[64];
     int n_probe;
+    int probe_kind;   // OSPREY_PROBE_LM_HEAD or OSPREY_PROBE_ATTENTION
     cudaEvent_t *probe_begin, *probe_end;
 };
 
@@ -204,6 +205,13 @@ extern "C" int osprey_probe_enable(osprey_ctx *ctx, int n) {
     return OSPREY_OK;
 }
 
+extern "C" int osprey_probe_select(osprey_ctx *ctx, int kind) {
+    if (!ctx || (kind != OSPREY_PROBE_LM_HEAD && kind != OSPREY_PROBE_ATTENTION))
+        return fail(OSPREY_ERR_INVALID_ARG, "bad probe kind");
+    ctx->probe_kind = kind;
+    return OSPREY_OK;
+}
+
 extern "C" int osprey_probe_read(osprey_ctx *ctx, float *ms, int n) {
     if (!ctx || !ms || n < 0 || n > ctx->n_probe) return fail(OSPREY_ERR_INVALID_ARG, "bad probe read");
     for (int i = 0; i < n; ++i) {
@@ -233,8 +241,12 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t off = 0;
     auto take = [&](size_t bytes) { size_t o = off; off = align256(off + bytes); return o; };
     size_t o_valid = take(4ull * B), o_pos0 = take(4ull * B), o_nn = take(4ull * B);
-    size_t o_at = take(4ull * R_ext * D.Hkv), o_lt = take(4ull * B);
-    size_t o_gb = take(2 * sizeof(unsigned));   // grid barrier of the fused layer tail
+    // arrival counters and the grid barrier, one contiguous block of int32
+    // words that the call's first kernel zeroes
+    const size_t o_at = off, n_at = (size_t)R_ext * D.Hkv;
+    const size_t o_lt = o_at + 4 * n_at, o_gb = o_lt + 4ull * B, o_rt = o_gb + 8;
+    const size_t n_counters = n_at + B + 2 + B;
+    take(4 * n_counters);
     size_t o_xe = take(4ull * R_ext * D.d), o_se = take(4ull * R_ext * D.d);
     size_t o_xc = take(4ull * B * D.d), o_sc = take(4ull * B * D.d);
     size_t o_q = take(4ull * R_ext * D.Hq * D.hd);
@@ -253,7 +265,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_xq = take(tcw ? 2ull * TC_PLANES * np * 2 * D.d : 0), o_yq = take(tcw ? 4ull * np * nqkv : 0);
     size_t o_xo = take(tcw ? 2ull * TC_PLANES * np * D.Hq * D.hd : 0), o_xg = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
-    size_t o_rp = take(tcw ? 16ull * B * row_sample_chunks(D.V) : 0), o_rt = take(tcw ? 4ull * B : 0);
+    size_t o_rp = take(tcw ? 16ull * B * row_sample_chunks(D.V) : 0);
     size_t o_tg = take(tcw ? 4ull * np * D.F : 0);
     // split-K partials: the largest nsplit x rows x outputs of the call's projections
     long long part = 0;
@@ -298,6 +310,8 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->tc_xl = (uint16_t *)(p + o_xl);
         ws->rs_part = (float4 *)(p + o_rp);
         ws->rs_ticket = (int *)(p + o_rt);
+        ws->counters = (int *)(p + o_at);
+        ws->n_counters = (int)n_counters;
         ws->tc_g = (float *)(p + o_tg);
         ws->tc_part = (float *)(p + o_tp);
         ws->tc_part_cap = part;
@@ -389,7 +403,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
 
     PrepArgs pa{B, K, max_new, kv->max_pages_per_seq, kv->n_pages, D.P, D.V,
                 kv->seq_len, n_new, tokens, kv->page_table,
-                ws.seq_valid, ws.seq_pos0, ws.seq_nnew, draft_tokens, dev_status};
+                ws.seq_valid, ws.seq_pos0, ws.seq_nnew, draft_tokens, dev_status, ws.counters, ws.n_counters};
     if ((e = launch_prepare(pa, s)) != cudaSuccess) return cuda_fail(e, "prepare launch");
 
     GemvArgs g{};
@@ -464,6 +478,11 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         return cuda_fail(e, "feature projection launch");
     }
 
+    // measurement hook: events around the attention launch of (step, layer)
+    auto attn_probe = [&](int slot, bool begin) -> cudaError_t {
+        if (ctx->probe_kind != OSPREY_PROBE_ATTENTION || slot >= ctx->n_probe) return cudaSuccess;
+        return probe_record(begin ? ctx->probe_begin[slot] : ctx->probe_end[slot], s);
+    };
     for (int step = 0; step < K; ++step) {
         const bool ext = step == 0;
         const int rows_per_seq = ext ? max_new : 1;
@@ -561,8 +580,10 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
             at.status = dev_status;
+            if ((e = attn_probe(step * D.L + l, true)) != cudaSuccess) return cuda_fail(e, "probe record");
             e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+            if ((e = attn_probe(step * D.L + l, false)) != cudaSuccess) return cuda_fail(e, "probe record");
             // x += W_o attn;  x += W_down (silu(W_g n) * W_u n),  n = RMSNorm(x)
             const int ha = D.Hq * D.hd;
             if ((rc = planes(ws.attn_out, nullptr, ha, R, ha, 0, ws.tc_xo, rows_per_seq, false, "o-proj operand")) !=
@@ -638,8 +659,10 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             at.out = ws.attn_out;
             at.ticket = ws.attn_ticket;
             at.status = dev_status;
+            if ((e = attn_probe(step * D.L + l, true)) != cudaSuccess) return cuda_fail(e, "probe record");
             e = clu ? launch_attn_cluster(at, ctx->attn_cs, s) : launch_attn(at, s);
             if (e != cudaSuccess) return cuda_fail(e, "attention launch");
+            if ((e = attn_probe(step * D.L + l, false)) != cudaSuccess) return cuda_fail(e, "probe record");
             if (streamed && R == 1 && ctx->fused_mlp) {
                 MlpArgs ma{};
                 ma.dim = D;
@@ -675,7 +698,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             (e = launch_keep_hidden(x, ext, B, K, step, max_new, D.d, ws.seq_valid, ws.seq_nnew, draft_hidden, s)) !=
                 cudaSuccess)
             return cuda_fail(e, "keep-hidden launch");
-        const bool probe = step < ctx->n_probe;
+        const bool probe = ctx->probe_kind == OSPREY_PROBE_LM_HEAD && step < ctx->n_probe;
         if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
         if (B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
@@ -834,7 +857,11 @@ extern "C" int osprey_verify(int B, int K, int V, int logits_dtype, const void *
     a.flags = flags;
     a.probs = probs;
     a.status = dev_status;
-    cudaError_t e = launch_verify(a, (cudaStream_t)stream);
+    // the arrival counters start at zero on every call, so a call that ran out
+    // of a bounded wait leaves nothing stale for the next one
+    cudaError_t e = cudaMemsetAsync(a.ticket1, 0, a.counter_bytes, (cudaStream_t)stream);
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the verify counters");
+    e = launch_verify(a, (cudaStream_t)stream);
     return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "verify launch");
 }
 
@@ -937,7 +964,8 @@ extern "C" int osprey_verify_hidden(osprey_ctx *ctx, int B, int K, int logits_dt
     a.stats_in = draft_stats;
     a.zrec = hw.z;
     cudaStream_t s = (cudaStream_t)stream;
-    cudaError_t e;
+    cudaError_t e = cudaMemsetAsync(a.ticket1, 0, a.counter_bytes, s);   // counters start at zero on every call
+    if (e != cudaSuccess) return cuda_fail(e, "clearing the verify counters");
     // 1. target row statistics, the acceptance chain and the decision row r
     if ((e = launch_verify_hidden_stats(a, s)) != cudaSuccess) return cuda_fail(e, "verify launch");
     for (int b0 = 0; b0 < B; b0 += hw.group) {

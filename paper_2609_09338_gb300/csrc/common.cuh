@@ -243,10 +243,15 @@ __device__ __forceinline__ void st_release_gpu(unsigned *p, unsigned v) {
 // `count` is zero between uses (the last block to arrive resets it) and `gen`
 // advances once per use; a block reads `gen` before arriving, so the release
 // cannot be missed.  The wait is bounded (about a second of SM clocks): on
-// expiry the status word gets OSPREY_ERR_TIMEOUT and the block goes on.
-__device__ __forceinline__ void grid_sync(unsigned *count, unsigned *gen, int32_t *status) {
+// expiry the status word gets OSPREY_ERR_TIMEOUT and the call returns false in
+// every thread of the block, which then stops (after draining its own copies).
+// The count may then stay short; the draft call's first kernel zeroes both
+// words, so the next call starts clean.
+__device__ __forceinline__ bool grid_sync(unsigned *count, unsigned *gen, int32_t *status) {
+    __shared__ int s_ok;
     __syncthreads();
     if (threadIdx.x == 0) {
+        int ok = 1;
         const unsigned g = ld_acquire_gpu(gen);
         __threadfence();   // this block's writes, ordered before the arrival
         if (atomicAdd(count, 1u) == gridDim.x - 1) {
@@ -258,14 +263,17 @@ __device__ __forceinline__ void grid_sync(unsigned *count, unsigned *gen, int32_
             while (ld_acquire_gpu(gen) == g) {
                 if (clock64() - t0 > 2000000000LL) {
                     set_status(status, OSPREY_ERR_TIMEOUT);
+                    ok = 0;
                     break;
                 }
                 __nanosleep(64);
             }
         }
         __threadfence();
+        s_ok = ok;
     }
     __syncthreads();
+    return s_ok != 0;
 }
 
 }  // namespace osp

@@ -897,6 +897,9 @@ __global__ void __launch_bounds__(GT) lm_head_kernel(const LmArgs a) {
 __global__ void __launch_bounds__(128) prepare_kernel(const PrepArgs a) {
     __shared__ int ok, code;
     const int b = blockIdx.x;
+    // every kernel of the call starts after this one has finished (it is
+    // launched without early dependents), so the counters read zero for all
+    for (int i = b * blockDim.x + threadIdx.x; i < a.n_counters; i += gridDim.x * blockDim.x) a.counters[i] = 0;
     const int L0 = a.seq_len[b], nn = a.n_new[b];
     if (threadIdx.x == 0) {
         const bool n_ok = nn >= 1 && nn <= a.max_new;
@@ -1009,15 +1012,12 @@ cudaError_t launch_gemv(GemvMode mode, const GemvArgs &a, int rg, int sms, cudaS
 
 template <int HD, int G>
 static cudaError_t launch_attn_t(const AttnArgs &a, cudaStream_t s) {
-    static int attr_dev = -1;   // the ring's dynamic shared memory, opted into once per device
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
+    static std::atomic<int> done[kMaxDevices];   // the ring's dynamic shared memory, opted into once per device
+    cudaError_t e = once_per_device(done, [] {
+        return cudaFuncSetAttribute(attn_kernel<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    AttnSplit<HD>::RING);
+    });
     if (e != cudaSuccess) return e;
-    if (attr_dev != dev) {
-        e = cudaFuncSetAttribute(attn_kernel<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, AttnSplit<HD>::RING);
-        if (e != cudaSuccess) return e;
-        attr_dev = dev;
-    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(a.n_splits, a.dim.Hkv, a.R);
     cfg.blockDim = dim3(AT);
@@ -1194,20 +1194,6 @@ cudaError_t launch_prepare(const PrepArgs &a, cudaStream_t s) {
     prepare_kernel<<<a.B, 128, 0, s>>>(a);
     count_launch();
     return cudaGetLastError();
-}
-
-// Let a kernel use all the opt-in shared memory left after its static part.
-template <typename F>
-static cudaError_t allow_smem(F *kernel) {
-    int dev = 0, optin = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
-    cudaFuncAttributes fa{};
-    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, kernel);
-    if (e == cudaSuccess)
-        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 optin - (int)fa.sharedSizeBytes);
-    return e;
 }
 
 template <int MODE>
@@ -1405,7 +1391,7 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
             }
         }
     fence_proxy_async_global();   // the K/V rows are read by other blocks' bulk copies
-    grid_sync(a.bar_count, a.bar_gen, a.status);
+    ok = ok && grid_sync(a.bar_count, a.bar_gen, a.status);   // a block that timed out stops
 
     // ---- B. attention partial of the block's key range; gate/up rows requested
     fence_proxy_async_global();
@@ -1421,7 +1407,7 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
         issued = 3;
     }
     const int units = D.Hkv * a.n_splits;
-    if (live && c < units) {
+    if (ok && live && c < units) {
         const int kvh = c / a.n_splits, split = c - kvh * a.n_splits;
         const int n_keys = pos + 1, pos0 = a.map.pos0[b];
         const int k_begin = split * a.split_len;   // a multiple of the page size
@@ -1473,10 +1459,10 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
             }
         }
     }
-    grid_sync(a.bar_count, a.bar_gen, a.status);
+    ok = ok && grid_sync(a.bar_count, a.bar_gen, a.status);   // a block that timed out stops
 
     // ---- C. O-proj and residual
-    if (live)
+    if (ok && live)
         for (int i = threadIdx.x * 4; i < Ko; i += LY_THREADS * 4)
             *(float4 *)(act + i) = __ldcg((const float4 *)(a.attn_out + i));
     __syncthreads();
@@ -1486,10 +1472,10 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
             const float acc = warp_smem_dot(wo + (size_t)j * Ko, act, Ko);
             if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
         }
-    grid_sync(a.bar_count, a.bar_gen, a.status);
+    ok = ok && grid_sync(a.bar_count, a.bar_gen, a.status);   // a block that timed out stops
 
     // ---- D. RMSNorm of the whole residual, gate/up and SwiGLU
-    if (live) {
+    if (ok && live) {
         for (int i = threadIdx.x * 4; i < d; i += LY_THREADS * 4)
             *(float4 *)(act + i) = __ldcg((const float4 *)(a.x + i));
         ly_rmsnorm(act, a.ffn_norm, d, D.eps, red);
@@ -1511,10 +1497,10 @@ __global__ void __launch_bounds__(LY_THREADS, 1) layer_fused_kernel(const LayerA
             bulk_g2s(wd, a.W_down + (size_t)o0 * F, bd, &bar[3]);
         issued = 4;
     }
-    grid_sync(a.bar_count, a.bar_gen, a.status);
+    ok = ok && grid_sync(a.bar_count, a.bar_gen, a.status);   // a block that timed out stops
 
     // ---- E. down and residual
-    if (live)
+    if (ok && live)
         for (int i = threadIdx.x * 4; i < F; i += LY_THREADS * 4)
             *(float4 *)(act + i) = __ldcg((const float4 *)(a.h + i));
     __syncthreads();
@@ -1541,7 +1527,7 @@ int layer_fused_splits(const Dims &D, int max_ctx, int sms) {
 }
 
 template <int HD, int G>
-static bool layer_fits(const LayerPlan &p) {
+static bool layer_fits(const LayerPlan &p, int sms) {
     int dev = 0, optin = 0;
     cudaFuncAttributes fa{};
     if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -1550,7 +1536,13 @@ static bool layer_fits(const LayerPlan &p) {
         cudaGetLastError();
         return false;
     }
-    return p.smem + fa.sharedSizeBytes <= (size_t)optin;
+    if (p.smem + fa.sharedSizeBytes > (size_t)optin) return false;
+    // the grid barriers need every block resident at once: one per SM
+    if (allow_smem(layer_fused_kernel<HD, G>) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return grid_fits_resident(layer_fused_kernel<HD, G>, LY_THREADS, p.smem, sms, sms);
 }
 
 bool layer_fused_supported(const Dims &D, int sms) {
@@ -1563,7 +1555,7 @@ bool layer_fused_supported(const Dims &D, int sms) {
         (size_t)2 * p.rf * D.d * 2 >= (1u << 20) || (size_t)p.ro * D.F * 2 >= (1u << 20))
         return false;
 #define OSP_LY_FITS(hd_, g_) \
-    if (D.hd == hd_ && G == g_) return layer_fits<hd_, g_>(p);
+    if (D.hd == hd_ && G == g_) return layer_fits<hd_, g_>(p, sms);
     OSP_LY_FITS(64, 1) OSP_LY_FITS(64, 2) OSP_LY_FITS(64, 4) OSP_LY_FITS(64, 8)
     OSP_LY_FITS(128, 1) OSP_LY_FITS(128, 2) OSP_LY_FITS(128, 4) OSP_LY_FITS(128, 8)
 #undef OSP_LY_FITS
@@ -1572,18 +1564,10 @@ bool layer_fused_supported(const Dims &D, int sms) {
 
 template <int HD, int G>
 static cudaError_t launch_layer_t(const LayerArgs &a, int sms, cudaStream_t s) {
+    // the shared-memory opt-in and the residency check ran when the context chose
+    // this path (layer_fused_supported, with the same grid)
     const LayerPlan p = layer_plan(a.dim, sms);
-    static int attr_dev = -1;
-    static size_t attr_smem = 0;   // the opt-in grows with the largest shape launched so far
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (attr_dev != dev || p.smem > attr_smem) {
-        e = cudaFuncSetAttribute(layer_fused_kernel<HD, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
-        if (e != cudaSuccess) return e;
-        attr_dev = dev;
-        attr_smem = p.smem;
-    }
+    cudaError_t e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(sms);
     cfg.blockDim = dim3(LY_THREADS);

@@ -43,6 +43,8 @@ struct DraftWs {
     uint16_t *tc_xl;                       // [P][np][d]     final RMSNorm rows for the LM head
     float4 *rs_part;                       // [B][V/4096]    row-sampler chunk partials
     int *rs_ticket;                        // [B]
+    int *counters;                         // attn_ticket .. rs_ticket: one contiguous block
+    int n_counters;
     int n_splits_max, lm_warps_max;
 };
 
@@ -127,6 +129,10 @@ struct PrepArgs {
     int *valid, *pos0, *nnew;
     int32_t *draft_tokens;
     int32_t *status;
+    // the call's arrival counters and grid-barrier words, zeroed here so that a
+    // call that ran out of a bounded wait leaves no stale count to the next one
+    int *counters;
+    int n_counters;
 };
 
 enum GemvMode { G_FEAT = 0, G_QKV = 1, G_OPROJ = 2, G_GATEUP = 3, G_DOWN = 4, G_LM = 5 };

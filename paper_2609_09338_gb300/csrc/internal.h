@@ -3,6 +3,8 @@
 
 #include <cuda_runtime.h>
 #include <stddef.h>
+
+#include <atomic>
 #include <stdint.h>
 
 #include "osprey.h"
@@ -14,6 +16,49 @@ void count_launch(int n = 1);
 
 // Sets the message osprey_last_error() returns on this thread.
 void set_last_error(const char *msg);
+
+// Runs set() (a cudaFuncSetAttribute call) the first time it is reached with a
+// device current, per flag array.  set() must be idempotent: host threads that
+// race here may both run it, but no thread reads a flag torn by another.
+constexpr int kMaxDevices = 256;
+template <typename F>
+cudaError_t once_per_device(std::atomic<int> (&done)[kMaxDevices], F set) {
+    int dev = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e != cudaSuccess) return e;
+    const bool tracked = dev >= 0 && dev < kMaxDevices;
+    if (tracked && done[dev].load(std::memory_order_acquire)) return cudaSuccess;
+    e = set();
+    if (e == cudaSuccess && tracked) done[dev].store(1, std::memory_order_release);
+    return e;
+}
+
+// Lets a kernel use all the opt-in shared memory left after its static part
+// (the same value every time, so a repeated call is harmless).
+template <typename F>
+cudaError_t allow_smem(F *kernel) {
+    int dev = 0, optin = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    cudaFuncAttributes fa{};
+    if (e == cudaSuccess) e = cudaFuncGetAttributes(&fa, kernel);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, optin - (int)fa.sharedSizeBytes);
+    return e;
+}
+
+// True when `grid` blocks of `threads` threads and `smem` bytes of dynamic
+// shared memory can all be resident at once on `sms` SMs of the current
+// device (what a grid-wide barrier needs).  Call after allow_smem(kernel).
+template <typename F>
+bool grid_fits_resident(F *kernel, int threads, size_t smem, int grid, int sms) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kernel, threads, smem) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return per_sm >= 1 && (long long)per_sm * sms >= grid;
+}
 
 // ---------------------------------------------------------------- verify
 struct Decision {

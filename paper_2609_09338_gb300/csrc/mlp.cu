@@ -89,10 +89,10 @@ __global__ void __launch_bounds__(MLP_THREADS, 1) mlp_fused_kernel(const MlpArgs
             const float acc = warp_smem_dot(wo + (size_t)j * Ko, act, Ko);
             if (lane == 0) a.x[o0 + j] = __ldcg(a.x + o0 + j) + acc;
         }
-    grid_sync(a.bar_count, a.bar_gen, a.status);
+    ok = ok && grid_sync(a.bar_count, a.bar_gen, a.status);   // a block that timed out stops
 
     // 2. RMSNorm of the whole residual, gate/up and SwiGLU
-    if (live) {
+    if (ok && live) {
         float ss = 0.f;
         for (int i = threadIdx.x * 4; i < d; i += MLP_THREADS * 4) {
             const float4 v = __ldcg((const float4 *)(a.x + i));
@@ -116,10 +116,10 @@ __global__ void __launch_bounds__(MLP_THREADS, 1) mlp_fused_kernel(const MlpArgs
             const float u = warp_smem_dot(wu + (size_t)j * d, act, d);
             if (lane == 0) a.h[f0 + j] = g / (1.f + expf(-g)) * u;
         }
-    grid_sync(a.bar_count, a.bar_gen, a.status);
+    ok = ok && grid_sync(a.bar_count, a.bar_gen, a.status);   // a block that timed out stops
 
     // 3. down and residual
-    if (live)
+    if (ok && live)
         for (int i = threadIdx.x * 4; i < F; i += MLP_THREADS * 4)
             *(float4 *)(act + i) = __ldcg((const float4 *)(a.h + i));
     __syncthreads();
@@ -148,24 +148,23 @@ bool mlp_fused_supported(const Dims &D, int sms) {
     }
     // whole 16-byte vectors everywhere; one block per SM fits
     // (each mbarrier phase counts fewer than 2^20 bytes)
-    return D.d % 256 == 0 && D.F % 256 == 0 && (D.Hq * D.hd) % 256 == 0 && p.smem + 1024 <= (size_t)optin &&
-           (size_t)p.ro * D.Hq * D.hd * 2 < (1u << 20) && (size_t)p.rf * D.d * 2 * 2 < (1u << 20) &&
-           (size_t)p.ro * D.F * 2 < (1u << 20);
+    if (!(D.d % 256 == 0 && D.F % 256 == 0 && (D.Hq * D.hd) % 256 == 0 && p.smem + 1024 <= (size_t)optin &&
+          (size_t)p.ro * D.Hq * D.hd * 2 < (1u << 20) && (size_t)p.rf * D.d * 2 * 2 < (1u << 20) &&
+          (size_t)p.ro * D.F * 2 < (1u << 20)))
+        return false;
+    // the grid barriers need every block resident at once: one per SM
+    if (allow_smem(mlp_fused_kernel) != cudaSuccess) {
+        cudaGetLastError();
+        return false;
+    }
+    return grid_fits_resident(mlp_fused_kernel, MLP_THREADS, p.smem, sms, sms);
 }
 
 cudaError_t launch_mlp_fused(const MlpArgs &a, int sms, cudaStream_t s) {
+    // the shared-memory opt-in and the residency check ran when the context chose
+    // this path (mlp_fused_supported, with the same grid)
     const MlpPlan p = mlp_plan(a.dim, sms);
-    static int attr_dev = -1;
-    static size_t attr_smem = 0;   // the opt-in grows with the largest shape launched so far
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (attr_dev != dev || p.smem > attr_smem) {
-        e = cudaFuncSetAttribute(mlp_fused_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)p.smem);
-        if (e != cudaSuccess) return e;
-        attr_dev = dev;
-        attr_smem = p.smem;
-    }
+    cudaError_t e;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(sms);
     cfg.blockDim = dim3(MLP_THREADS);

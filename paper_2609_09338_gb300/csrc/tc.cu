@@ -559,10 +559,12 @@ __global__ void __launch_bounds__(256) embed_rows_kernel(const EmbedArgs a) {
 
 // ---------------------------------------------------------------- host side
 static PFN_cuTensorMapEncodeTiled_v12000 g_encode = nullptr;
-static int g_encode_state = 0;   // 0 unknown, 1 ok, -1 unavailable
 
+// The driver's tensor-map encoder and a device with tcgen05 (compute
+// capability 10 or above); looked up once, thread-safely (a function-local
+// static is initialised exactly once).
 bool tc_available() {
-    if (g_encode_state == 0) {
+    static const bool ok = [] {
         cudaDriverEntryPointQueryResult q;
         void *fn = nullptr;
         const cudaError_t e = cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q);
@@ -573,9 +575,9 @@ bool tc_available() {
             cudaGetLastError();
             major = 0;
         }
-        g_encode_state = g_encode && major >= 10 ? 1 : -1;
-    }
-    return g_encode_state == 1;
+        return g_encode != nullptr && major >= 10;
+    }();
+    return ok;
 }
 
 static bool encode2d(CUtensorMap *m, const void *base, uint64_t inner, uint64_t rows, uint32_t box_rows) {

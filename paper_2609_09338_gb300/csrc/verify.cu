@@ -19,7 +19,6 @@
 #include <math.h>
 
 #include <cstdio>
-#include <mutex>
 
 #include "common.cuh"
 #include "internal.h"
@@ -505,16 +504,12 @@ cudaError_t launch_verify(const VerifyArgs &a, cudaStream_t s) {
 // Allocation-free verify: the scratch lives in this file-scope device array
 // instead of a caller workspace.  Host code may not use the array's name as a
 // device address (on the host it names a stand-in), so its device address is
-// looked up once per device with cudaGetSymbolAddress, with that device current.
+// looked up with cudaGetSymbolAddress, with the caller's device current, on
+// every call: the address belongs to the current context (a context torn down
+// and made again loads the module again), and the lookup allocates nothing.
 namespace osp {
 
 static __device__ __align__(256) unsigned char g_verify_scratch[OSPREY_VERIFY_STATIC_SCRATCH_BYTES];
-
-namespace {
-std::mutex g_scratch_mu;
-constexpr int kMaxDevices = 256;
-void *g_scratch_addr[kMaxDevices] = {};
-}  // namespace
 
 }  // namespace osp
 
@@ -538,35 +533,15 @@ extern "C" int osprey_verify_static(int B, int K, int V, int logits_dtype, const
         set_last_error(msg);
         return OSPREY_ERR_CAPACITY;
     }
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess || dev < 0 || dev >= kMaxDevices) {
-        set_last_error("osprey_verify_static: no usable current device");
-        return OSPREY_ERR_CUDA;
-    }
     void *base = nullptr;
-    {
-        std::lock_guard<std::mutex> lock(g_scratch_mu);
-        if (!g_scratch_addr[dev]) {
-            void *p = nullptr;
-            e = cudaGetSymbolAddress(&p, g_verify_scratch);
-            if (e != cudaSuccess || !p) {
-                cudaGetLastError();
-                set_last_error("osprey_verify_static: cudaGetSymbolAddress of the scratch array failed");
-                return OSPREY_ERR_CUDA;
-            }
-            g_scratch_addr[dev] = p;
-        }
-        base = g_scratch_addr[dev];
-    }
-    // the arrival counters must start at zero; everything else is written before it is read
-    VerifyArgs view{};
-    verify_workspace_layout(B, K, V, &view, base);
-    cudaStream_t s = (cudaStream_t)stream;
-    if ((e = cudaMemsetAsync(view.ticket1, 0, view.counter_bytes, s)) != cudaSuccess) {
-        set_last_error("osprey_verify_static: clearing the scratch counters failed");
+    const cudaError_t e = cudaGetSymbolAddress(&base, g_verify_scratch);
+    if (e != cudaSuccess || !base) {
+        cudaGetLastError();
+        set_last_error("osprey_verify_static: cudaGetSymbolAddress of the scratch array failed");
         return OSPREY_ERR_CUDA;
     }
+    // osprey_verify clears the arrival counters on the stream before its
+    // kernels; everything else is written before it is read
     return osprey_verify(B, K, V, logits_dtype, target_logits, draft_logits, draft_tokens, temperature, u_accept,
                          u_sample, out_tokens, n_accepted, flags, probs, base, OSPREY_VERIFY_STATIC_SCRATCH_BYTES,
                          dev_status, stream);

@@ -779,14 +779,10 @@ bool verify_stream_ok(const VerifyArgs &a) {
 // lives in a per-kernel template (the kernels share one function type).
 template <auto Kernel>
 static cudaError_t vs_allow_smem() {
-    static int done[256] = {0};
-    int dev = 0;
-    cudaError_t e = cudaGetDevice(&dev);
-    if (e != cudaSuccess) return e;
-    if (dev >= 0 && dev < 256 && done[dev]) return cudaSuccess;
-    e = cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, VS_NST * VS_SLOT);
-    if (e == cudaSuccess && dev >= 0 && dev < 256) done[dev] = 1;
-    return e;
+    static std::atomic<int> done[kMaxDevices];
+    return once_per_device(done, [] {
+        return cudaFuncSetAttribute(Kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, VS_NST * VS_SLOT);
+    });
 }
 
 template <auto Kernel>

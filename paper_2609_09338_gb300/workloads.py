@@ -114,4 +114,4 @@ WORKLOADS = {
                                                  sigma_p=0.7, seed=1004),
 }
 
-BENCH_WORKLOAD = "qwen3-8b-d1024-v151936-b1-k7"
+BENCH_WORKLOAD = "large-vocab-d1024-v200064-b64-k8"

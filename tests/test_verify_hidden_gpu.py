@@ -1,19 +1,13 @@
 """Logits-free sampled verification (the Sec. 3.1 rule with the draft rows
 defined by the drafter's final norm and LM head over its kept states,
-Sec. 3.3-3.4) through the C ABI, against the oracle.
-
-Held back until the kernels have run on a GB300: set
-OSPREY_TEST_VERIFY_HIDDEN=1 to run these."""
-import os
+Sec. 3.3-3.4) through the C ABI, against the oracle."""
 from dataclasses import replace
 
 import numpy as np
 import pytest
 
 torch = pytest.importorskip("torch")
-pytestmark = [pytest.mark.gpu,
-              pytest.mark.skipif(os.environ.get("OSPREY_TEST_VERIFY_HIDDEN") != "1",
-                                 reason="logits-free verify not yet run on a GB300 (OSPREY_TEST_VERIFY_HIDDEN=1)")]
+pytestmark = pytest.mark.gpu
 
 from oracle import verify as ov  # noqa: E402
 from oracle.drafter import inverse_cdf  # noqa: E402

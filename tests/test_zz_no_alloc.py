@@ -5,8 +5,9 @@ all HBM for its weights and KV cache, or code on a latency-critical path where
 cudaMalloc/cudaFree may block or synchronise the device.  For them the library
 keeps verify's scratch in a fixed device array of its own.  This file checks,
 through the C ABI, that two calls in a row give what the workspace entry point
-gives, and that requests too large for the array are refused with a message.
-Kept in a file that pytest collects last."""
+gives, that a call changes neither the device's free memory nor torch's
+allocations, and that requests too large for the array are refused with a
+message.  Kept in a file that pytest collects last."""
 import numpy as np
 import pytest
 
@@ -43,11 +44,16 @@ def test_static_scratch_matches_workspace_entry_point(V, B, K, T):
     ref = _outputs(B, K)
     ws = torch.zeros(ob.osprey_verify_workspace_bytes(B, K, V), dtype=torch.uint8, device="cuda")
     ob.osprey_verify(*args, ref["out_tokens"], ref["n_accepted"], ref["flags"], ref["probs"], ws, ref["status"])
-    for _ in range(2):                          # two calls in a row share the static array
-        got = _outputs(B, K)
+    outs = [_outputs(B, K) for _ in range(2)]   # allocated before the calls are measured
+    torch.cuda.synchronize()
+    for i, got in enumerate(outs):              # two calls in a row share the static array
+        free0, alloc0 = torch.cuda.mem_get_info()[0], torch.cuda.memory_allocated()
         ob.osprey_verify_static(*args, got["out_tokens"], got["n_accepted"], got["flags"], got["probs"],
                                 got["status"])
         torch.cuda.synchronize()
+        if i == 1:   # the first call may load the library's device code; the second allocates nothing
+            assert torch.cuda.mem_get_info()[0] == free0
+            assert torch.cuda.memory_allocated() == alloc0
         assert int(got["status"].item()) == 0
         for k in ("out_tokens", "n_accepted", "flags"):
             np.testing.assert_array_equal(got[k].cpu().numpy(), ref[k].cpu().numpy())
