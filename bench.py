@@ -66,12 +66,15 @@ def parse():
     p.add_argument("--verify-hidden", action="store_true",
                    help="compare draft (logits written) + verify against draft (states kept) + logits-free verify")
     p.add_argument("--no-extra", action="store_true", help="measure the headline workload only")
+    p.add_argument("--sweep", default=None,
+                   help="verify sweep points as dtype:B:K[,dtype:B:K...] (default: all of f32/bf16 x B x K)")
     return p.parse_args()
 
 
 # measured after the headline workload, each with its own dominant kernel
 EXTRA_WORKLOADS = ["qwen3-8b-d1024-v151936-b1-k7", "qwen3-8b-d1024-v151936-b32-k7",
-                   "llama70b-d2048-v128256-b16-k7", "osprey-d2560-v151936-b1-k7-ext3"]
+                   "llama70b-d2048-v128256-b16-k7", "osprey-d2560-v151936-b1-k7-ext3",
+                   "dflash-d4096-l4-v151936-b1-blk16"]
 
 
 def make_inputs(wl, rank=0, weights_path=None):
@@ -86,7 +89,7 @@ def make_inputs(wl, rank=0, weights_path=None):
         if weights_path and rank == 0:
             from paper_2609_09338_gb300 import checkpoint
             checkpoint.save_weights(weights_path, sh, w)
-    kv = syn.make_kv_prefix(sh, ctx, wl.n_new + wl.K, seed + 1)
+    kv = syn.make_kv_prefix(sh, ctx, wl.extra.get("block", wl.n_new + wl.K), seed + 1)
     di = syn.make_draft_inputs(sh, wl.batch, wl.n_new, wl.K, seed + 2)
     vi = syn.make_verify_inputs(sh.vocab, wl.batch, wl.K, wl.temperature, wl.sigma_p, seed + 3)
     return ctx, w, kv, di, vi
@@ -102,6 +105,17 @@ def algorithmic_bytes(wl, ctx):
     B, K = wl.batch, wl.K
     w_step = sh.weight_bytes_per_step()
     kv_row = 2 * sh.n_layers * sh.n_kv_heads * sh.head_dim * 2           # K and V, bf16, all layers
+    if wl.extra.get("block"):
+        # block drafting: one forward over the block (weights once), every
+        # sequence's cached positions read once, its block rows written
+        blk = wl.extra["block"]
+        kv = sum(kv_row * (int(c) + blk - 1) for c in ctx)
+        draft = w_step + 2 * sh.d_model * sh.feat_dim + kv + B * sh.feat_dim * 2
+        s = 4 if wl.logits_dtype == "f32" else 2
+        return {"draft": draft, "verify": B * (2 * K + 1) * sh.vocab * s,
+                "lm_head_launch": sh.vocab * sh.d_model * 2 + 2 * sh.d_model, "attn_call": kv,
+                "attn_launches": sh.n_layers, "lm_launches": 1,
+                "verify_f32": B * (2 * K + 1) * sh.vocab * 4, "verify_bf16": B * (2 * K + 1) * sh.vocab * 2}
     # chain step k attends over ctx + n_new + k positions (extend row: ctx + 1 with n_new = 1)
     kv = sum(kv_row * (int(c) + wl.n_new + k) for c in ctx for k in range(K))
     draft = K * w_step + 2 * sh.d_model * sh.feat_dim + kv + B * wl.n_new * sh.feat_dim * 2
@@ -321,9 +335,11 @@ def nvtx_pop():
         pass
 
 
-def lm_head_label(B):
+def lm_head_label(B, block=False):
     """The LM-head launches the probes bracket, by the number of rows (the draft
     step's kernel selection)."""
+    if block:
+        return "planes_kernel + tc_kernel<STORE> + row_sample_kernel over every block row (tcgen05 LM head)"
     if B <= 2:
         return "stream_kernel<LM> (final RMSNorm + TMA-streamed LM-head GEMV + on-chip sampling)"
     if B <= 80:
@@ -353,42 +369,44 @@ def verify_sweep(args):
     flush_r = torch.ones(256 * 1024 * 1024 // 4, dtype=torch.float32, device="cuda")
     gen = torch.Generator(device="cuda").manual_seed(1234)
     points = []
-    for dtype in (torch.float32, torch.bfloat16):
-        for B in (1, 8, 64, 256):
-            for K in (1, 4, 8):
-                zp = torch.randn((B, K + 1, V), generator=gen, device="cuda").to(dtype)
-                zq = torch.randn((B, K, V), generator=gen, device="cuda").to(dtype)
-                x = torch.randint(0, V, (B, K), generator=gen, device="cuda", dtype=torch.int32)
-                ua = torch.rand((B, K), generator=gen, device="cuda")
-                us = torch.rand((B, K + 1), generator=gen, device="cuda")
-                vb = VerifyBuffers(B, K, V)
-                st = torch.cuda.Stream()
-                st.wait_stream(torch.cuda.current_stream())   # inputs and zeroed workspace first
-                with torch.cuda.stream(st):
-                    vb.run(zp, zq, x, T, ua, us)
-                torch.cuda.synchronize()
-                g = torch.cuda.CUDAGraph()   # replayed, so host marshalling stays out of the timing
-                with torch.cuda.graph(g, stream=st):
-                    vb.run(zp, zq, x, T, ua, us)
-                ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                      for _ in range(args.steps + 3)]
-                with torch.cuda.stream(st):
-                    for s_, e_ in ev:
-                        flush_w.zero_()
-                        flush_r.sum()
-                        s_.record(st)
-                        g.replay()
-                        e_.record(st)
-                torch.cuda.synchronize()
-                assert int(vb.status.item()) == 0
-                ev = ev[3:]
-                us_ = 1e3 * sum(s_.elapsed_time(e_) for s_, e_ in ev) / len(ev)
-                nbytes = (B * (K + 1) * V + B * K * V) * zp.element_size()
-                gbs = nbytes / (us_ * 1e-6) / 1e9
-                points.append({"dtype": "f32" if dtype == torch.float32 else "bf16", "B": B, "K": K,
-                               "bytes": nbytes, "us": round(us_, 2), "GBps": round(gbs, 1),
-                               "frac": round(gbs / peak, 3), "roofline_us": round(nbytes / peak / 1e3, 2)})
-                del zp, zq
+    grid = [(dt, B, K) for dt in ("f32", "bf16") for B in (1, 8, 64, 256) for K in (1, 4, 8)]
+    if args.sweep:
+        grid = [(p.split(":")[0], int(p.split(":")[1]), int(p.split(":")[2])) for p in args.sweep.split(",")]
+    for dname, B, K in grid:
+        dtype = torch.float32 if dname == "f32" else torch.bfloat16
+        zp = torch.randn((B, K + 1, V), generator=gen, device="cuda").to(dtype)
+        zq = torch.randn((B, K, V), generator=gen, device="cuda").to(dtype)
+        x = torch.randint(0, V, (B, K), generator=gen, device="cuda", dtype=torch.int32)
+        ua = torch.rand((B, K), generator=gen, device="cuda")
+        us = torch.rand((B, K + 1), generator=gen, device="cuda")
+        vb = VerifyBuffers(B, K, V)
+        st = torch.cuda.Stream()
+        st.wait_stream(torch.cuda.current_stream())   # inputs and zeroed workspace first
+        with torch.cuda.stream(st):
+            vb.run(zp, zq, x, T, ua, us)
+        torch.cuda.synchronize()
+        g = torch.cuda.CUDAGraph()   # replayed, so host marshalling stays out of the timing
+        with torch.cuda.graph(g, stream=st):
+            vb.run(zp, zq, x, T, ua, us)
+        ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+              for _ in range(args.steps + 3)]
+        with torch.cuda.stream(st):
+            for s_, e_ in ev:
+                flush_w.zero_()
+                flush_r.sum()
+                s_.record(st)
+                g.replay()
+                e_.record(st)
+        torch.cuda.synchronize()
+        assert int(vb.status.item()) == 0
+        ev = ev[3:]
+        us_ = 1e3 * sum(s_.elapsed_time(e_) for s_, e_ in ev) / len(ev)
+        nbytes = (B * (K + 1) * V + B * K * V) * zp.element_size()
+        gbs = nbytes / (us_ * 1e-6) / 1e9
+        points.append({"dtype": "f32" if dtype == torch.float32 else "bf16", "B": B, "K": K,
+                       "bytes": nbytes, "us": round(us_, 2), "GBps": round(gbs, 1),
+                       "frac": round(gbs / peak, 3), "roofline_us": round(nbytes / peak / 1e3, 2)})
+        del zp, zq
     print(json.dumps({"metric": "verify GB/s sweep", "peak": peak, "peak_kind": peak_kind, "V": V,
                       "temperature": T, "steps": args.steps, "l2": "flushed before every call",
                       "verify_sweep": points}))
@@ -491,7 +509,12 @@ def measure(wl, args, rank, world, local, full):
     nb = algorithmic_bytes(wl, ctx)
     dom = dominant_kernel(nb)
     dev = "cuda"
-    sess = DraftSession(sh, w, kv["page_table"], kv["n_pages"], K, wl.n_new)
+    blk = wl.extra.get("block")
+    if blk:
+        from paper_2609_09338_gb300.session import DflashSession
+        sess = DflashSession(sh, w, kv["page_table"], kv["n_pages"], blk)
+    else:
+        sess = DraftSession(sh, w, kv["page_table"], kv["n_pages"], K, wl.n_new)
     sess.append(ctx, kv["k_rows"], kv["v_rows"])
     torch.cuda.synchronize()
     assert int(sess.status.item()) == 0
@@ -513,9 +536,16 @@ def measure(wl, args, rank, world, local, full):
     stream = torch.cuda.Stream()
     stream.wait_stream(torch.cuda.current_stream())   # inputs and buffers first
 
+    if blk:   # the block's anchor and feature: the first extend row's token and feature
+        d_in["anchors"] = d_in["tokens"][:, 0].contiguous()
+        d_in["feats1"] = d_in["feats"][:, 0].contiguous()
+
     def step():
         sess.kv.seq_len.copy_(seq0)
-        sess.draft(d_in["n_new"], d_in["tokens"], d_in["feats"], T, d_in["u_draft"], out)
+        if blk:
+            sess.propose(d_in["anchors"], 0, d_in["feats1"], T, d_in["u_draft"], out)
+        else:
+            sess.draft(d_in["n_new"], d_in["tokens"], d_in["feats"], T, d_in["u_draft"], out)
         vb.run(v_in["target"], v_in["draft"] if T > 0 else None, v_in["tokens"], T, v_in["u_accept"],
                v_in["u_sample"])
 
@@ -590,7 +620,7 @@ def measure(wl, args, rank, world, local, full):
         lm_mean_ms = sum(lm) / len(lm)
         achieved = nb["lm_head_launch"] / (lm_mean_ms * 1e-3) / 1e9
         sha = _sha(os.path.join(ROOT, LM_TRAFFIC["source"]))
-        roof = {"kernel": lm_head_label(B), "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
+        roof = {"kernel": lm_head_label(B, bool(blk)), "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak,
                 "traffic": LM_TRAFFIC["bytes_per_launch"] if LM_TRAFFIC["sha256"] == sha and B <= 2 else None,
                 "peak_kind": peak_kind, "bytes_per_launch": nb["lm_head_launch"], "mean_launch_us": lm_mean_ms * 1e3,

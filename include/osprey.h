@@ -184,6 +184,42 @@ int osprey_draft_step_hidden(osprey_ctx *ctx, const osprey_kv *kv, int B, int K,
                              float *draft_qx, float *draft_stats, float *draft_hidden,
                              void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
 
+/* Bytes of workspace osprey_dflash_step needs.  0 on bad arguments. */
+size_t osprey_dflash_workspace_bytes(const osprey_ctx *ctx, int B, int block, int max_pages_per_seq);
+
+/* Block drafting with the EAGLE-style DFlash interface (Appendix, "EAGLE-Style
+ * Target Interface for DFlash"): one drafter forward over a block of `block`
+ * positions per sequence - the verified anchor token at position seq_len[b],
+ * then the mask placeholder token at the next block - 1 positions - with causal
+ * attention inside the block, and with the target feature gathered at the
+ * anchor fed to every position through the expanded QKV projection (its
+ * target-side columns are Eq. 2's context columns, zero at initialisation).
+ * Labels are shifted by one: the output at block position j proposes the
+ * token at j + 1, so positions 0..block-2 give block - 1 proposals, each drawn
+ * from its own q_j = softmax(logits_j / T) by the inverse CDF at u_draft[b][j]
+ * (argmax at T = 0).  The proposals are verified like a chain of block - 1
+ * draft tokens (osprey_verify with K = block - 1).
+ *   block  4 .. 81 (3 .. 80 proposals); sequences are processed in groups of
+ *          floor(80 / (block - 1)), each group one tensor-core pass over the
+ *          weights (SHAPE if the context has no tensor-core path)
+ *   anchors [B] int32 (device), mask_token in [0, vocab)
+ *   feats  [B][feat_dim] bf16: the concatenated target hidden states gathered
+ *          at the anchor (c = W_c feats, Eq. 1, broadcast over the block)
+ *   u_draft [B][block-1] float in [0,1) (may be NULL when T == 0)
+ * Outputs (device): draft_tokens [B][block-1] int32, draft_qx [B][block-1],
+ *   draft_stats [B][block-1][2] (as osprey_draft_step; qx and stats may be
+ *   NULL), draft_logits [B][block-1][vocab] float (NULL to keep them in the
+ *   workspace)
+ * Effects: the anchor's K/V row is committed (seq_len[b] += 1); the mask rows'
+ * K/V are written speculatively after it (the next call overwrites them).  The
+ * pages must hold seq_len[b] + block - 1 positions (else dev_status = CAPACITY
+ * and the sequence is skipped: tokens -1, seq_len unchanged).
+ * Host errors: INVALID_ARG, SHAPE, CAPACITY (workspace_bytes too small). */
+int osprey_dflash_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int block, const int32_t *anchors,
+                       int32_t mask_token, const void *feats, float temperature, const float *u_draft,
+                       int32_t *draft_tokens, float *draft_qx, float *draft_stats, float *draft_logits,
+                       void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
+
 /* Bytes of workspace osprey_verify_hidden needs.  0 on bad arguments. */
 size_t osprey_verify_hidden_workspace_bytes(const osprey_ctx *ctx, int B, int K);
 

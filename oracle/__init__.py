@@ -13,9 +13,12 @@ Everything is plain numpy in float64, written from the paper:
 * ``oracle.verify`` - speculative-sampling verification (Sec. 3.1, the
   unmodified acceptance rule of Leviathan et al.), its greedy form, and the
   exact emission distribution obtained by integrating the rule over its
-  uniforms.
+  uniforms;
+* ``oracle.dflash`` - the EAGLE-style DFlash block drafter (Appendix, "EAGLE-
+  Style Target Interface for DFlash"): one causal forward over an anchor and
+  mask placeholders, the target feature broadcast through the expanded QKV.
 
 Every function below is pinned by a ``-m "not gpu"`` test against something
 other than itself (closed forms, library routines, invariants, brute force).
 """
-from . import bf16, drafter, verify  # noqa: F401
+from . import bf16, dflash, drafter, verify  # noqa: F401

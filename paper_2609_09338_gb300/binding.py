@@ -81,6 +81,10 @@ _c_draft = _sig("osprey_draft_step", ctypes.c_int,
 _c_draft_hidden = _sig("osprey_draft_step_hidden", ctypes.c_int,
                        [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32,
                         _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp])
+_c_dflash_ws = _sig("osprey_dflash_workspace_bytes", _sz, [_vp, ctypes.c_int, ctypes.c_int, ctypes.c_int])
+_c_dflash = _sig("osprey_dflash_step", ctypes.c_int,
+                 [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, _vp, ctypes.c_int32, _vp,
+                  ctypes.c_float, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp])
 _c_verify_hidden_ws = _sig("osprey_verify_hidden_workspace_bytes", _sz, [_vp, ctypes.c_int, ctypes.c_int])
 _c_verify_hidden = _sig("osprey_verify_hidden", ctypes.c_int,
                         [_vp, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _vp, _vp, _f32, _vp, _vp, _vp,
@@ -99,7 +103,8 @@ _c_launch_count = _sig("osprey_launch_count", _i64, [])
 _c_selftest_wait = _sig("osprey_selftest_wait_timeout", ctypes.c_int, [_i64, _vp, _vp])
 
 EXPORTED = ["osprey_last_error", "osprey_create", "osprey_destroy", "osprey_draft_workspace_bytes",
-            "osprey_kv_append", "osprey_draft_step", "osprey_draft_step_hidden", "osprey_verify_workspace_bytes",
+            "osprey_kv_append", "osprey_draft_step", "osprey_draft_step_hidden", "osprey_dflash_workspace_bytes",
+            "osprey_dflash_step", "osprey_verify_workspace_bytes",
             "osprey_verify", "osprey_verify_static", "osprey_verify_hidden_workspace_bytes", "osprey_verify_hidden",
             "osprey_probe_enable", "osprey_probe_select", "osprey_probe_read", "osprey_launch_count", "osprey_selftest_wait_timeout"]
 
@@ -306,6 +311,39 @@ def osprey_draft_step_hidden(ctx: Ctx, kv: KvCache, n_new: torch.Tensor, tokens:
     _check(_c_draft_hidden(ctx.handle, ctypes.byref(kvs), B, K, max_new, _ptr(n_new), _ptr(tokens), _ptr(feats),
                            float(temperature), _ptr(u_draft), _ptr(draft_tokens), _ptr(draft_qx), _ptr(draft_stats),
                            _ptr(draft_hidden), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+
+
+def osprey_dflash_workspace_bytes(ctx: Ctx, B: int, block: int, max_pages: int) -> int:
+    return int(_c_dflash_ws(ctx.handle, B, block, max_pages))
+
+
+def osprey_dflash_step(ctx: Ctx, kv: KvCache, anchors: torch.Tensor, mask_token: int, feats: torch.Tensor,
+                       temperature: float, u_draft, draft_tokens: torch.Tensor, draft_qx=None, draft_stats=None,
+                       draft_logits=None, workspace: torch.Tensor = None, status: torch.Tensor = None, stream=None):
+    """Block drafting (EAGLE-style DFlash): one forward over anchor + block-1
+    mask positions per sequence; draft_tokens [B, block-1] are its proposals."""
+    s = ctx.shape
+    B = anchors.shape[0]
+    P = draft_tokens.shape[1]
+    _need(anchors, torch.int32, (B,), "anchors")
+    _need(feats, torch.bfloat16, (B, s.feat_dim), "feats")
+    _need(draft_tokens, torch.int32, (B, P), "draft_tokens")
+    if u_draft is not None:
+        _need(u_draft, torch.float32, (B, P), "u_draft")
+    if draft_qx is not None:
+        _need(draft_qx, torch.float32, (B, P), "draft_qx")
+    if draft_stats is not None:
+        _need(draft_stats, torch.float32, (B, P, 2), "draft_stats")
+    if draft_logits is not None:
+        _need(draft_logits, torch.float32, (B, P, s.vocab), "draft_logits")
+    _need(workspace, torch.uint8, None, "workspace")
+    _need(status, torch.int32, (1,), "status")
+    if kv.page_table.shape[0] != B:
+        raise ValueError("page table rows must equal the batch")
+    kvs = kv.c_struct()
+    _check(_c_dflash(ctx.handle, ctypes.byref(kvs), B, P + 1, _ptr(anchors), int(mask_token), _ptr(feats),
+                     float(temperature), _ptr(u_draft), _ptr(draft_tokens), _ptr(draft_qx), _ptr(draft_stats),
+                     _ptr(draft_logits), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
 
 
 def osprey_verify_hidden_workspace_bytes(ctx: Ctx, B: int, K: int) -> int:

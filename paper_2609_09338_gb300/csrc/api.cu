@@ -230,10 +230,13 @@ static cudaError_t probe_record(cudaEvent_t ev, cudaStream_t s) {
 }
 
 // ------------------------------------------------------------------ workspace
+// block: the layout of a block-drafting call (every extend row is sampled, so
+// the logits and sampler buffers hold B * max_new rows instead of B)
 static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int max_pages,
-                           DraftWs *ws, void *base) {
+                           DraftWs *ws, void *base, bool block = false) {
     const Dims &D = ctx->dim;
     const long long R_ext = (long long)B * max_new;
+    const long long R_lm = block ? R_ext : B;
     const int max_ctx = max_pages * D.P;
     const int ns = std::max(attn_splits((int)R_ext, D.Hkv, max_ctx, ctx->sms),
                             attn_splits(B, D.Hkv, max_ctx, ctx->sms));
@@ -245,7 +248,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     // words that the call's first kernel zeroes
     const size_t o_at = off, n_at = (size_t)R_ext * D.Hkv;
     const size_t o_lt = o_at + 4 * n_at, o_gb = o_lt + 4ull * B, o_rt = o_gb + 8;
-    const size_t n_counters = n_at + B + 2 + B;
+    const size_t n_counters = n_at + B + 2 + R_lm;
     take(4 * n_counters);
     size_t o_xe = take(4ull * R_ext * D.d), o_se = take(4ull * R_ext * D.d);
     size_t o_xc = take(4ull * B * D.d), o_sc = take(4ull * B * D.d);
@@ -255,7 +258,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
     const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
-    size_t o_lz = take(4ull * B * D.V);
+    size_t o_lz = take(4ull * R_lm * D.V);
     size_t o_lc = take(16ull * B * lmp.blocks);
     // tensor-core path: bf16 operand planes, QKV output, row-sampler partials
     const long long tc_rows = std::min<long long>(std::max<long long>(R_ext, B), TC_MAX_ROWS);
@@ -265,7 +268,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_xq = take(tcw ? 2ull * TC_PLANES * np * 2 * D.d : 0), o_yq = take(tcw ? 4ull * np * nqkv : 0);
     size_t o_xo = take(tcw ? 2ull * TC_PLANES * np * D.Hq * D.hd : 0), o_xg = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
-    size_t o_rp = take(tcw ? 16ull * B * row_sample_chunks(D.V) : 0);
+    size_t o_rp = take(tcw ? 16ull * R_lm * row_sample_chunks(D.V) : 0);
     size_t o_tg = take(tcw ? 4ull * np * D.F : 0);
     // split-K partials: the largest nsplit x rows x outputs of the call's projections
     long long part = 0;
@@ -370,11 +373,15 @@ extern "C" int osprey_kv_append(const osprey_ctx *ctx, const osprey_kv *kv, int 
 }
 
 // ------------------------------------------------------------------ draft step
+// block: a block-drafting call (EAGLE-style DFlash): K = 1, every one of the
+// max_new extend rows of a sequence is sampled (row j's output proposes the
+// token at j + 1) into draft_* [B][max_new], and only the first row (the
+// anchor) is committed.
 static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int max_new,
                            const int32_t *n_new, const int32_t *tokens, const void *feats, float temperature,
                            const float *u_draft, int32_t *draft_tokens, float *draft_qx, float *draft_stats,
                            float *draft_logits, float *draft_hidden, void *workspace, size_t workspace_bytes,
-                           int32_t *dev_status, void *stream) {
+                           int32_t *dev_status, void *stream, bool block = false) {
     g_err[0] = 0;
     if (!ctx || !kv) return fail(OSPREY_ERR_INVALID_ARG, "null context or kv");
     if (B == 0) return OSPREY_OK;
@@ -390,9 +397,11 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
     if (((uintptr_t)feats | (uintptr_t)workspace | (uintptr_t)draft_hidden) % 16)
         return fail(OSPREY_ERR_INVALID_ARG, "feats, workspace and draft_hidden must be 16-byte aligned");
     DraftWs ws{};
-    const size_t need = draft_layout(ctx, B, K, max_new, kv->max_pages_per_seq, &ws, workspace);
+    const size_t need = draft_layout(ctx, B, K, max_new, kv->max_pages_per_seq, &ws, workspace, block);
     if (workspace_bytes < need)
         return fail(OSPREY_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
+    if (block && (K != 1 || !ctx->tc || B * max_new < 3 || B * max_new > TC_MAX_ROWS))
+        return fail(OSPREY_ERR_SHAPE, "block drafting runs 3..%d rows per group on the tensor cores", TC_MAX_ROWS);
 
     cudaStream_t s = (cudaStream_t)stream;
     const Dims &D = ctx->dim;
@@ -403,7 +412,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
 
     PrepArgs pa{B, K, max_new, kv->max_pages_per_seq, kv->n_pages, D.P, D.V,
                 kv->seq_len, n_new, tokens, kv->page_table,
-                ws.seq_valid, ws.seq_pos0, ws.seq_nnew, draft_tokens, dev_status, ws.counters, ws.n_counters};
+                ws.seq_valid, ws.seq_pos0, ws.seq_nnew, draft_tokens, dev_status, ws.counters, ws.n_counters,
+                block ? 1 : 0, block ? max_new : 0};
     if ((e = launch_prepare(pa, s)) != cudaSuccess) return cuda_fail(e, "prepare launch");
 
     GemvArgs g{};
@@ -701,7 +711,39 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         const bool probe = ctx->probe_kind == OSPREY_PROBE_LM_HEAD && step < ctx->n_probe;
         if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
-        if (B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
+        if (block) {
+            // every extend row: final RMSNorm -> logits -> its own draw (row r of
+            // sequence r / max_new proposes the token after it)
+            const int rows = B * max_new;
+            float *zb = draft_logits ? draft_logits : ws.lm_z;
+            int rc;
+            if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, rows, D.d, 0, ws.tc_xl, max_new, false,
+                             "lm operand")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_STORE, rows, D.d, D.V, TC_PLANES, ctx->tm_lm, ws.tc_xl, false, zb, D.V, nullptr,
+                              "lm head launch")) != OSPREY_OK)
+                return rc;
+            RowSampleArgs rs{};
+            rs.dim = D;
+            rs.B = rows;
+            rs.K = 1;
+            rs.step = 0;
+            rs.max_new = max_new;
+            rs.valid = ws.seq_valid;
+            rs.nnew = ws.seq_nnew;
+            rs.rows_per_valid = max_new;
+            rs.z = zb;
+            rs.ldz = D.V;
+            rs.temperature = temperature;
+            rs.u_draft = u_draft;
+            rs.tokens = draft_tokens;
+            rs.qx = draft_qx;
+            rs.stats = draft_stats;
+            rs.embed = (const uint16_t *)W.embed;
+            rs.part = ws.rs_part;
+            rs.ticket = ws.rs_ticket;
+            rs.nch = row_sample_chunks(D.V);
+            if ((e = launch_row_sample(rs, s)) != cudaSuccess) return cuda_fail(e, "sampler launch");
+        } else if (B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
             plan_into(G_LM);
             sa.W = (const uint16_t *)W.lm_head;
             sa.gain = (const uint16_t *)W.final_norm;
@@ -810,6 +852,95 @@ extern "C" int osprey_draft_step_hidden(osprey_ctx *ctx, const osprey_kv *kv, in
     }
     return draft_step_impl(ctx, kv, B, K, max_new, n_new, tokens, feats, temperature, u_draft, draft_tokens, draft_qx,
                            draft_stats, nullptr, draft_hidden, workspace, workspace_bytes, dev_status, stream);
+}
+
+// ------------------------------------------------------------------ block drafting
+// Sequences are drafted in groups whose block rows fit one tensor-core tile
+// (TC_MAX_ROWS rows); each group's call re-reads the weights once.  Workspace:
+// the block-mode draft layout of one group, then the group's token array
+// [n][P], n_new [n] and broadcast features [n][P][feat_dim] bf16.
+static int block_group(int B, int P) {
+    const int g = TC_MAX_ROWS / P;
+    return g < 1 ? 1 : (g < B ? g : B);
+}
+
+static size_t block_layout(const osprey_ctx *ctx, int n, int P, int max_pages, DraftWs *ws, void *base,
+                           int32_t **tok, int32_t **nnew, uint16_t **feats) {
+    size_t off = align256(draft_layout(ctx, n, 1, P, max_pages, ws, base, true));
+    const size_t o_t = off;
+    off = align256(off + 4ull * n * P);
+    const size_t o_n = off;
+    off = align256(off + 4ull * n);
+    const size_t o_f = off;
+    off = align256(off + 2ull * n * P * ctx->dim.feat);
+    if (base) {
+        *tok = (int32_t *)((char *)base + o_t);
+        *nnew = (int32_t *)((char *)base + o_n);
+        *feats = (uint16_t *)((char *)base + o_f);
+    }
+    return off;
+}
+
+static bool block_args_ok(const osprey_ctx *ctx, int B, int block, int max_pages) {
+    return ctx && B >= 1 && B <= 65535 && block >= 4 && block <= TC_MAX_ROWS + 1 && max_pages >= 1 &&
+           (long long)max_pages * ctx->dim.P < (1LL << 30);
+}
+
+extern "C" size_t osprey_dflash_workspace_bytes(const osprey_ctx *ctx, int B, int block, int max_pages_per_seq) {
+    if (!block_args_ok(ctx, B, block, max_pages_per_seq)) return 0;
+    const int P = block - 1;
+    return block_layout(ctx, block_group(B, P), P, max_pages_per_seq, nullptr, nullptr, nullptr, nullptr, nullptr);
+}
+
+extern "C" int osprey_dflash_step(osprey_ctx *ctx, const osprey_kv *kv, int B, int block, const int32_t *anchors,
+                                  int32_t mask_token, const void *feats, float temperature, const float *u_draft,
+                                  int32_t *draft_tokens, float *draft_qx, float *draft_stats, float *draft_logits,
+                                  void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    g_err[0] = 0;
+    if (!ctx || !kv) return fail(OSPREY_ERR_INVALID_ARG, "null context or kv");
+    if (B == 0) return OSPREY_OK;
+    if (!block_args_ok(ctx, B, block, kv->max_pages_per_seq))
+        return fail(OSPREY_ERR_INVALID_ARG, "B in 1..65535, block in 4..%d and max_pages_per_seq >= 1 required",
+                    TC_MAX_ROWS + 1);
+    if (!ctx->tc)
+        return fail(OSPREY_ERR_SHAPE, "block drafting runs on the tensor cores; this context has none "
+                                      "(OSPREY_TC=0 or no tcgen05)");
+    if (mask_token < 0 || mask_token >= ctx->dim.V) return fail(OSPREY_ERR_INVALID_ARG, "mask_token out of range");
+    if (!(temperature >= 0.f) || !std::isfinite(temperature))
+        return fail(OSPREY_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+    if (!anchors || !feats || !draft_tokens || !workspace || !kv->k_pages || !kv->v_pages || !kv->page_table ||
+        !kv->seq_len)
+        return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
+    if (temperature > 0.f && !u_draft) return fail(OSPREY_ERR_INVALID_ARG, "u_draft is required when temperature > 0");
+    if (((uintptr_t)feats | (uintptr_t)workspace) % 16)
+        return fail(OSPREY_ERR_INVALID_ARG, "feats and workspace must be 16-byte aligned");
+    const int P = block - 1, G = block_group(B, P);
+    const Dims &D = ctx->dim;
+    DraftWs ws{};
+    int32_t *tok = nullptr, *nnew = nullptr;
+    uint16_t *frep = nullptr;
+    const size_t need = block_layout(ctx, G, P, kv->max_pages_per_seq, &ws, workspace, &tok, &nnew, &frep);
+    if (workspace_bytes < need)
+        return fail(OSPREY_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
+    cudaStream_t s = (cudaStream_t)stream;
+    for (int b0 = 0; b0 < B; b0 += G) {
+        const int n = B - b0 < G ? B - b0 : G;
+        BlockInArgs bi{n, P, D.feat, anchors + b0, mask_token, (const uint16_t *)feats + (size_t)b0 * D.feat,
+                       tok, nnew, frep};
+        cudaError_t e = launch_block_inputs(bi, s);
+        if (e != cudaSuccess) return cuda_fail(e, "block inputs launch");
+        osprey_kv kg = *kv;
+        kg.page_table = kv->page_table + (size_t)b0 * kv->max_pages_per_seq;
+        kg.seq_len = kv->seq_len + b0;
+        const size_t o = (size_t)b0 * P;
+        const int rc = draft_step_impl(ctx, &kg, n, 1, P, nnew, tok, frep, temperature, u_draft ? u_draft + o : nullptr,
+                                       draft_tokens + o, draft_qx ? draft_qx + o : nullptr,
+                                       draft_stats ? draft_stats + 2 * o : nullptr,
+                                       draft_logits ? draft_logits + o * D.V : nullptr, nullptr, workspace,
+                                       workspace_bytes, dev_status, stream, true);
+        if (rc != OSPREY_OK) return rc;
+    }
+    return OSPREY_OK;
 }
 
 // ------------------------------------------------------------------ verify

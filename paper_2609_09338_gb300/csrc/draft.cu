@@ -924,11 +924,12 @@ __global__ void __launch_bounds__(128) prepare_kernel(const PrepArgs a) {
         a.valid[b] = ok;
         a.pos0[b] = L0;
         a.nnew[b] = nn;
-        if (ok) a.seq_len[b] = L0 + nn;
+        if (ok) a.seq_len[b] = L0 + (a.commit > 0 ? a.commit : nn);
         else set_status(a.status, code);
     }
+    const int n_out = a.n_out > 0 ? a.n_out : a.K;
     if (!ok)
-        for (int k = threadIdx.x; k < a.K; k += blockDim.x) a.draft_tokens[(size_t)b * a.K + k] = -1;
+        for (int k = threadIdx.x; k < n_out; k += blockDim.x) a.draft_tokens[(size_t)b * n_out + k] = -1;
 }
 
 // ---------------------------------------------------------------------------

@@ -133,6 +133,8 @@ struct PrepArgs {
     // call that ran out of a bounded wait leaves no stale count to the next one
     int *counters;
     int n_counters;
+    int commit;    // rows committed per sequence (0: all n_new rows)
+    int n_out;     // draft tokens per sequence set to -1 for a skipped sequence (0: K)
 };
 
 enum GemvMode { G_FEAT = 0, G_QKV = 1, G_OPROJ = 2, G_GATEUP = 3, G_DOWN = 4, G_LM = 5 };

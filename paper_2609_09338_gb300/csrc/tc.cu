@@ -451,7 +451,7 @@ __global__ void __launch_bounds__(RS_THREADS) row_sample_kernel(const RowSampleA
     const int c = blockIdx.x, b = blockIdx.y, t = threadIdx.x;
     pdl_trigger();
     pdl_wait();
-    if (!a.valid[b]) return;   // every block of the row leaves here
+    if (!a.valid[a.rows_per_valid > 1 ? b / a.rows_per_valid : b]) return;   // every block of the row leaves here
     const bool greedy = a.temperature == 0.f;
     const float invT = greedy ? 1.f : 1.f / a.temperature;
     const float *z = a.z + (size_t)b * a.ldz;
@@ -555,6 +555,25 @@ __global__ void __launch_bounds__(256) embed_rows_kernel(const EmbedArgs a) {
     if (!a.valid[b] || j >= a.nnew[b]) return;
     const uint16_t *e = a.embed + (size_t)a.tokens[r] * a.d;   // ids checked by the prepare kernel
     for (int k = threadIdx.x; k < a.d; k += blockDim.x) a.x[(size_t)r * a.d + k] = bf_to_f(e[k]);
+}
+
+// ---------------------------------------------------------------- block inputs
+__global__ void __launch_bounds__(256) block_inputs_kernel(const BlockInArgs a) {
+    const int r = blockIdx.x, b = r / a.P, j = r - b * a.P;
+    if (threadIdx.x == 0) {
+        a.tokens[r] = j == 0 ? a.anchors[b] : a.mask;
+        if (j == 0) a.nnew[b] = a.P;
+    }
+    const uint4 *src = (const uint4 *)(a.feats + (size_t)b * a.feat);
+    uint4 *dst = (uint4 *)(a.feats_rep + (size_t)r * a.feat);
+    for (int k = threadIdx.x; k < a.feat / 8; k += blockDim.x) dst[k] = src[k];
+}
+
+cudaError_t launch_block_inputs(const BlockInArgs &a, cudaStream_t s) {
+    // a normal launch: the draft call's prepare kernel reads these arrays
+    block_inputs_kernel<<<a.n * a.P, 256, 0, s>>>(a);
+    count_launch();
+    return cudaGetLastError();
 }
 
 // ---------------------------------------------------------------- host side

@@ -114,8 +114,21 @@ struct RowSampleArgs {
     float4 *part;              // [B][nch] chunk partials
     int *ticket;               // [B]
     int nch;
+    int rows_per_valid;        // row b belongs to sequence b / rows_per_valid (0 or 1: itself)
 };
 int row_sample_chunks(int V);
+// Block drafting inputs (EAGLE-style DFlash): for row r = b*P + j of n
+// sequences, tokens[r] = anchor[b] (j = 0) or mask (j > 0); feats_rep[r] =
+// feats[b] (feat_dim bf16, broadcast over the block); nnew[b] = P.
+struct BlockInArgs {
+    int n, P, feat;
+    const int32_t *anchors;
+    int32_t mask;
+    const uint16_t *feats;
+    int32_t *tokens, *nnew;
+    uint16_t *feats_rep;
+};
+cudaError_t launch_block_inputs(const BlockInArgs &a, cudaStream_t s);
 // x[r] = E[tokens[r]] (float32) for the active extend rows r = b*max_new + j, j < n_new[b].
 struct EmbedArgs {
     int d, R, max_new;

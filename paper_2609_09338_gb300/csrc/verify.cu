@@ -19,6 +19,7 @@
 #include <math.h>
 
 #include <cstdio>
+#include <type_traits>
 
 #include "common.cuh"
 #include "internal.h"
@@ -87,6 +88,32 @@ __device__ __forceinline__ void load_chunk(const T *row, int start, int V, float
 template <typename T, bool VEC>
 __device__ __forceinline__ int elem_index(int start, int j) {
     return VEC ? start + chunk_index<T, true>(j) : start + j * VT + threadIdx.x;
+}
+
+// Load this thread's VPER values of a float32 row in the element order that
+// load_chunk<T, VEC> gives a row of T (so that value j of both loads is the
+// same id): the logits-free draw pairs bf16 target rows with float32 draft rows.
+template <typename T, bool VEC>
+__device__ __forceinline__ void load_chunk_f32_as(const float *row, int start, int V, float (&f)[VPER]) {
+    if (!VEC || Vec<T>::W == 4) {
+        load_chunk<float, VEC>(row, start, V, f);
+        return;
+    }
+    constexpr int NV = VPER / 8;   // T has 8 values per 16-byte vector: two float4 loads each
+    uint4 lo[NV], hi[NV];
+#pragma unroll
+    for (int it = 0; it < NV; ++it) {
+        const int e = start + (it * VT + threadIdx.x) * 8;
+        lo[it] = e < V ? ld_stream(row + e) : make_uint4(0, 0, 0, 0);
+        hi[it] = e < V ? ld_stream(row + e + 4) : make_uint4(0, 0, 0, 0);
+    }
+#pragma unroll
+    for (int it = 0; it < NV; ++it) {
+        const int e = start + (it * VT + threadIdx.x) * 8;
+        const uint32_t w[8] = {lo[it].x, lo[it].y, lo[it].z, lo[it].w, hi[it].x, hi[it].y, hi[it].z, hi[it].w};
+#pragma unroll
+        for (int j = 0; j < 8; ++j) f[it * 8 + j] = e < V ? __uint_as_float(w[j]) : -INFINITY;
+    }
 }
 
 __device__ __forceinline__ MS thread_ms(const float (&f)[VPER], float invT) {
@@ -262,7 +289,10 @@ __global__ void __launch_bounds__(VT) verify_sample(VerifyArgs a) {
     if (valid) {
         float f[VPER], g[VPER];
         load_chunk<T, VEC>(zp, start, V, f);
-        if (residual) load_chunk<TQ, VEC>(zq, start, V, g);
+        if (residual) {
+            if constexpr (std::is_same<T, TQ>::value) load_chunk<TQ, VEC>(zq, start, V, g);
+            else load_chunk_f32_as<T, VEC>(zq, start, V, g);
+        }
         float sw = 0.f, sp = 0.f;
 #pragma unroll
         for (int j = 0; j < VPER; ++j) {

@@ -52,6 +52,26 @@ class DraftSession:
                                     self.status, stream)
 
 
+class DflashSession(DraftSession):
+    """A drafter that proposes blocks (EAGLE-style DFlash): each call is one
+    forward over the anchor and block - 1 mask positions of every sequence."""
+
+    def __init__(self, shape: DrafterShape, weights_np: dict, page_table: np.ndarray, n_pages: int, block: int,
+                 device: str = "cuda"):
+        super().__init__(shape, weights_np, page_table, n_pages, block - 1, block - 1, device)
+        self.block = block
+        nbytes = ob.osprey_dflash_workspace_bytes(self.ctx, self.B, block, self.kv.max_pages)
+        self.workspace = torch.zeros(nbytes, dtype=torch.uint8, device=device)
+
+    def block_buffers(self, with_logits: bool = False) -> dict:
+        return self.draft_buffers(with_logits)
+
+    def propose(self, anchors, mask_token: int, feats, temperature: float, u_draft, out: dict, stream=None):
+        ob.osprey_dflash_step(self.ctx, self.kv, anchors, mask_token, feats, temperature, u_draft,
+                              out["draft_tokens"], out["draft_qx"], out["draft_stats"], out["draft_logits"],
+                              self.workspace, self.status, stream)
+
+
 class VerifyBuffers:
     def __init__(self, B: int, K: int, V: int, device: str = "cuda", workspace_bytes: int | None = None):
         self.out_tokens = torch.zeros((B, K + 1), dtype=torch.int32, device=device)

@@ -85,6 +85,14 @@ OSPREY_PAPER_DRAFTER = DrafterShape(d_model=2560, n_layers=2, n_q_heads=32, n_kv
                                     head_dim=128, ffn_dim=9728, vocab=151936,
                                     feat_dim=3 * 4096, rope_theta=1e6)
 
+# The appendix's DFlash drafter (Appendix, "Cross-Domain Warm-Start Ablation
+# under DFlash"): a four-layer LayerSkip-Llama-8B-shaped body (d 4096, 32/8
+# heads of 128, FFN 14336, rotary base 5e5) with its LM head row-mapped to the
+# Qwen3-8B target vocabulary and the EAGLE-style target interface (the target
+# feature 3 x 4096 projected to d and fed through the expanded QKV).
+DFLASH_DRAFTER = DrafterShape(d_model=4096, n_layers=4, n_q_heads=32, n_kv_heads=8, head_dim=128,
+                              ffn_dim=14336, vocab=151936, feat_dim=3 * 4096, rope_theta=5e5)
+
 WORKLOADS = {
     # tiny correctness case: fits the oracle in well under a second
     "tiny-d256-v4096-b1-k4": Workload("tiny-d256-v4096-b1-k4", TINY, batch=1, K=4,
@@ -107,6 +115,11 @@ WORKLOADS = {
     "osprey-d2560-v151936-b1-k7-ext3": Workload("osprey-d2560-v151936-b1-k7-ext3", OSPREY_PAPER_DRAFTER,
                                                 batch=1, K=7, ctx_lo=2048, ctx_hi=2048, temperature=1.0,
                                                 sigma_p=0.7, seed=1005, n_new=3),
+    # block drafting, one stream: one forward over anchor + 15 mask positions
+    # (block size 16, the appendix's setting) proposes K = 15 tokens
+    "dflash-d4096-l4-v151936-b1-blk16": Workload("dflash-d4096-l4-v151936-b1-blk16", DFLASH_DRAFTER,
+                                                 batch=1, K=15, ctx_lo=2048, ctx_hi=2048, temperature=1.0,
+                                                 sigma_p=0.7, seed=1006, extra={"block": 16}),
     # large vocabulary, verify-heavy
     "large-vocab-d1024-v200064-b64-k8": Workload("large-vocab-d1024-v200064-b64-k8",
                                                  LARGE_VOCAB_DRAFTER, batch=64, K=8,

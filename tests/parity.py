@@ -42,3 +42,21 @@ def bf16_to_f32(t):
     """torch bf16 tensor -> numpy float32 (exact)."""
     import torch
     return t.to(torch.float32).cpu().numpy()
+
+
+def check_kv_rows(got, want, mag):
+    """Cached bf16 K/V rows of the GPU against the oracle's.
+
+    Each side rounds its own unrounded value a (GPU, float32) or a* (oracle,
+    float64) to bf16, which moves it by at most half a bf16 step, 2^-8 |value|:
+        |got - want| <= 2^-8 (|got| + |want|) + |a - a*|.
+    a - a* is the float32 error of the projection that made the element, a dot
+    product of the row's inputs u with a row of W~_qkv, so it scales with
+    mag = sum_j |W_ij| |u_j| (the oracle's ``*_mag``; for a rotated key, summed
+    over its rotation pair): |a - a*| <= c * mag.  The inputs u of a chain row
+    carry the float32 error of every step before it (the fed-back state runs
+    through attention over up to 8k cached keys); over the workloads the
+    largest element needs c = 2^-15.3 (the two-layer Llama-shaped chain rows),
+    the others fit 2^-16.  c = 2^-14 keeps a factor 2.5 above that."""
+    import numpy as np
+    np.testing.assert_array_less(np.abs(got - want), 2.0 ** -8 * (np.abs(got) + np.abs(want)) + 2.0 ** -14 * mag + 1e-30)

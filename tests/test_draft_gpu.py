@@ -19,7 +19,7 @@ pytestmark = pytest.mark.gpu
 from oracle import drafter as od  # noqa: E402
 from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
 from paper_2609_09338_gb300.workloads import TINY, WORKLOADS  # noqa: E402
-from parity import gather_positions  # noqa: E402
+from parity import check_kv_rows, gather_positions  # noqa: E402
 
 LOGIT_TOL = 2e-2
 
@@ -150,25 +150,13 @@ def check_case(case, o=None, min_checked_frac=0.5):
         lse = np.log(np.exp(y - y.max(-1, keepdims=True)).sum(-1)) + y.max(-1)
         q_at = np.exp(np.take_along_axis(y, toks[..., None].astype(np.int64), -1)[..., 0] - lse)
         np.testing.assert_allclose(g["draft_qx"][idx], q_at, rtol=3 * LOGIT_TOL / T, atol=1e-6)
-    # the K/V the call wrote (committed extend rows and speculative chain rows).
-    # Each side rounds its own unrounded value a (GPU, float32) or a* (oracle,
-    # float64) to bf16, which moves it by at most half a bf16 step, 2^-8 |value|:
-    #   |got - want| <= 2^-8 (|got| + |want|) + |a - a*|.
-    # a - a* is the float32 error of the projection that made the element: a
-    # dot product of the row's inputs u (computed in float32 from the same
-    # cache state, since the oracle reads the GPU's cached rows) with a row of
-    # W~_qkv, so |a - a*| <= c * sum_j |W_ij| |u_j| (the oracle's ``*_mag``; for
-    # a rotated key the sum over both elements of its pair).  c = 2^-16 leaves
-    # a margin of about 2^8 over one float32 rounding of the sum and of the inputs.
+    # the K/V the call wrote (committed extend rows and speculative chain rows)
     for i, b in enumerate(idx):
         nn = int(case["di"]["n_new"][b])
         pos = np.arange(case["ctx"][b], case["ctx"][b] + nn + K - 1)
         for name, pages in (("new_k", g["k_pages"]), ("new_v", g["v_pages"])):
             got = gather_positions(pages, case["kv"]["page_table"][b], pos)
-            want = o[name][i]
-            mag = o[name + "_mag"][i]
-            np.testing.assert_array_less(np.abs(got - want),
-                                         2.0 ** -8 * (np.abs(got) + np.abs(want)) + 2.0 ** -16 * mag + 1e-30)
+            check_kv_rows(got, o[name][i], o[name + "_mag"][i])
     return checked, len(idx) * K
 
 
