@@ -258,7 +258,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
     const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
-    size_t o_lz = take(4ull * R_lm * D.V);
+    size_t o_lz = take(4ull * B * D.V);   // the streamed LM head's logits row (rows <= 2)
     size_t o_lc = take(16ull * B * lmp.blocks);
     // tensor-core path: bf16 operand planes, QKV output, row-sampler partials
     const long long tc_rows = std::min<long long>(std::max<long long>(R_ext, B), TC_MAX_ROWS);
@@ -268,7 +268,8 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_xq = take(tcw ? 2ull * TC_PLANES * np * 2 * D.d : 0), o_yq = take(tcw ? 4ull * np * nqkv : 0);
     size_t o_xo = take(tcw ? 2ull * TC_PLANES * np * D.Hq * D.hd : 0), o_xg = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
-    size_t o_rp = take(tcw ? 16ull * R_lm * row_sample_chunks(D.V) : 0);
+    const long long lm_nsub = (D.V + TC_LM_GROUP - 1) / TC_LM_GROUP;
+    size_t o_rp = take(tcw ? 16ull * R_lm * lm_nsub : 0);
     size_t o_tg = take(tcw ? 4ull * np * D.F : 0);
     // split-K partials: the largest nsplit x rows x outputs of the call's projections
     long long part = 0;
@@ -457,6 +458,42 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         ta.part_cap = ws.tc_part_cap;
         const cudaError_t e2 = launch_tc(ta, wa, xm, ctx->sms, s);
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
+    };
+    // the LM head of `rows` operand rows in ws.tc_xl on the tensor cores, with the
+    // sampling partials in its epilogue (logits stored only into z, when given),
+    // then one pick block per row
+    auto tc_lm = [&](int rows, float *z, long long ldz, const LmPickArgs &pick_in) -> int {
+        const int np = npad_of(rows);
+        CUtensorMap xm;
+        if (!tc_encode_operand(&xm, ws.tc_xl, TC_PLANES, np, D.d))
+            return fail(OSPREY_ERR_INVALID_ARG, "lm head: tensor map encoding failed");
+        TcArgs ta{};
+        ta.epi = TC_LM;
+        ta.R = rows;
+        ta.npad = np;
+        ta.K = D.d;
+        ta.nout = D.V;
+        ta.planes = TC_PLANES;
+        ta.y = z;
+        ta.ldy = (int)ldz;
+        ta.status = dev_status;
+        ta.lm_part = ws.rs_part;
+        ta.lm_nsub = (D.V + TC_LM_GROUP - 1) / TC_LM_GROUP;
+        ta.lm_invT = temperature > 0.f ? 1.f / temperature : 1.f;
+        cudaError_t e2 = launch_tc(ta, ctx->tm_lm, xm, ctx->sms, s);
+        if (e2 != cudaSuccess) return cuda_fail(e2, "lm head launch");
+        LmPickArgs pk = pick_in;
+        pk.dim = D;
+        pk.part = ws.rs_part;
+        pk.nsub = ta.lm_nsub;
+        pk.planes = ws.tc_xl;
+        pk.npad = np;
+        pk.W = (const uint16_t *)W.lm_head;
+        pk.temperature = temperature;
+        pk.u_draft = u_draft;
+        pk.embed = (const uint16_t *)W.embed;
+        e2 = launch_lm_pick(pk, s);
+        return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, "sampler launch");
     };
     auto planes = [&](const float *src, const uint16_t *gain, int d_, int rows, int ld, int col0, uint16_t *dst,
                       int rows_per_seq, bool last_of_seq, const char *what) -> int {
@@ -712,37 +749,25 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         if (probe && (e = probe_record(ctx->probe_begin[step], s)) != cudaSuccess)
             return cuda_fail(e, "probe record");
         if (block) {
-            // every extend row: final RMSNorm -> logits -> its own draw (row r of
+            // every extend row: final RMSNorm -> LM head -> its own draw (row r of
             // sequence r / max_new proposes the token after it)
             const int rows = B * max_new;
-            float *zb = draft_logits ? draft_logits : ws.lm_z;
             int rc;
             if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, rows, D.d, 0, ws.tc_xl, max_new, false,
-                             "lm operand")) != OSPREY_OK ||
-                (rc = tc_gemm(TC_STORE, rows, D.d, D.V, TC_PLANES, ctx->tm_lm, ws.tc_xl, false, zb, D.V, nullptr,
-                              "lm head launch")) != OSPREY_OK)
+                             "lm operand")) != OSPREY_OK)
                 return rc;
-            RowSampleArgs rs{};
-            rs.dim = D;
-            rs.B = rows;
-            rs.K = 1;
-            rs.step = 0;
-            rs.max_new = max_new;
-            rs.valid = ws.seq_valid;
-            rs.nnew = ws.seq_nnew;
-            rs.rows_per_valid = max_new;
-            rs.z = zb;
-            rs.ldz = D.V;
-            rs.temperature = temperature;
-            rs.u_draft = u_draft;
-            rs.tokens = draft_tokens;
-            rs.qx = draft_qx;
-            rs.stats = draft_stats;
-            rs.embed = (const uint16_t *)W.embed;
-            rs.part = ws.rs_part;
-            rs.ticket = ws.rs_ticket;
-            rs.nch = row_sample_chunks(D.V);
-            if ((e = launch_row_sample(rs, s)) != cudaSuccess) return cuda_fail(e, "sampler launch");
+            LmPickArgs pk{};
+            pk.B = rows;
+            pk.K = 1;
+            pk.step = 0;
+            pk.max_new = max_new;
+            pk.rows_per_valid = max_new;
+            pk.valid = ws.seq_valid;
+            pk.nnew = ws.seq_nnew;
+            pk.tokens = draft_tokens;
+            pk.qx = draft_qx;
+            pk.stats = draft_stats;
+            if ((rc = tc_lm(rows, draft_logits, D.V, pk)) != OSPREY_OK) return rc;
         } else if (B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
             plan_into(G_LM);
             sa.W = (const uint16_t *)W.lm_head;
@@ -762,39 +787,29 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             sa.ticket = ws.lm_ticket;
             if ((e = launch_stream(G_LM, sa, B, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
         } else if (tc_rows(B)) {
-            // final RMSNorm rows -> logits (draft_logits when requested) -> on-chip sampling
+            // final RMSNorm rows -> LM head with the sampling partials in its
+            // epilogue (logits stored only into draft_logits) -> one pick per row
             int rc;
-            float *zb = draft_logits ? draft_logits + (size_t)step * D.V : ws.lm_z;
-            const long long ldz = draft_logits ? (long long)K * D.V : D.V;
             if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand")) !=
-                    OSPREY_OK ||
-                (rc = tc_gemm(TC_STORE, B, D.d, D.V, TC_PLANES, ctx->tm_lm, ws.tc_xl, false, zb, (int)ldz, nullptr,
-                              "lm head launch")) != OSPREY_OK)
+                OSPREY_OK)
                 return rc;
-            RowSampleArgs rs{};
-            rs.dim = D;
-            rs.B = B;
-            rs.K = K;
-            rs.step = step;
-            rs.max_new = max_new;
-            rs.src_is_ext = ext;
-            rs.valid = ws.seq_valid;
-            rs.nnew = ws.seq_nnew;
-            rs.z = zb;
-            rs.ldz = ldz;
-            rs.temperature = temperature;
-            rs.u_draft = u_draft;
-            rs.tokens = draft_tokens;
-            rs.qx = draft_qx;
-            rs.stats = draft_stats;
-            rs.x_in = x;
-            rs.x_chain = ws.x_chain;
-            rs.s_chain = ws.s_chain;
-            rs.embed = (const uint16_t *)W.embed;
-            rs.part = ws.rs_part;
-            rs.ticket = ws.rs_ticket;
-            rs.nch = row_sample_chunks(D.V);
-            if ((e = launch_row_sample(rs, s)) != cudaSuccess) return cuda_fail(e, "sampler launch");
+            LmPickArgs pk{};
+            pk.B = B;
+            pk.K = K;
+            pk.step = step;
+            pk.max_new = max_new;
+            pk.src_is_ext = ext;
+            pk.valid = ws.seq_valid;
+            pk.nnew = ws.seq_nnew;
+            pk.tokens = draft_tokens;
+            pk.qx = draft_qx;
+            pk.stats = draft_stats;
+            pk.x_in = x;
+            pk.x_chain = ws.x_chain;
+            pk.s_chain = ws.s_chain;
+            if ((rc = tc_lm(B, draft_logits ? draft_logits + (size_t)step * D.V : nullptr, (long long)K * D.V, pk)) !=
+                OSPREY_OK)
+                return rc;
         } else {
             LmArgs lm{};
             lm.dim = D;

@@ -273,6 +273,24 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                         tc_st16(tt + (uint32_t)c0, v);
                         continue;
                     }
+                    if (EPI == TC_LM) {
+                        // per row: (max y, sum exp(y - max), argmax z) over this warp's 32 ids
+                        const int sub = (int)(((long long)((i0 + it) / a.nsplit) * 128 + lg) / TC_LM_GROUP);
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const int n = c0 + j;   // the same for every lane of the warp
+                            if (n >= a.R) break;
+                            const float zv = colok ? v[j] : -INFINITY;
+                            if (a.y && colok) a.y[(size_t)n * a.ldy + col] = zv;
+                            const AM am = warp_am(AM{zv, colok ? col : 0x7fffffff});
+                            const float mx = am.v * a.lm_invT;
+                            const float ev = colok ? __expf(zv * a.lm_invT - mx) : 0.f;
+                            const float se = warp_sum(ev);
+                            if (lane == 0 && sub < a.lm_nsub)
+                                a.lm_part[(size_t)n * a.lm_nsub + sub] = make_float4(mx, se, am.v, __int_as_float(am.i));
+                        }
+                        continue;
+                    }
 #pragma unroll
                     for (int j = 0; j < 16; ++j) {
                         const int n = c0 + j;
@@ -413,12 +431,8 @@ __global__ void __launch_bounds__(256) qkv_post_kernel(const QkvPostArgs a) {
     }
 }
 
-// ---------------------------------------------------------------- row sampler
-constexpr int RS_THREADS = 256;
-constexpr int RS_PER = 16;                      // logits per thread in a chunk
-constexpr int RS_CHUNK = RS_THREADS * RS_PER;   // 4096 ids
-
-int row_sample_chunks(int V) { return (V + RS_CHUNK - 1) / RS_CHUNK; }
+// ---------------------------------------------------------------- LM-head pick
+constexpr int PK_THREADS = 256;
 
 // Block-wide ordered pick over one weight per thread: the smallest index i
 // with t < C_i (inclusive cumulative weight, positive weights only); if
@@ -440,87 +454,109 @@ __device__ int rs_pick(float w, int idx, float t, float *before, float *sh, int 
     return pick;
 }
 
-__global__ void __launch_bounds__(RS_THREADS) row_sample_kernel(const RowSampleArgs a) {
-    __shared__ MS sm_ms[RS_THREADS / 32];
-    __shared__ AM sm_am[RS_THREADS / 32];
+// One block per row.  Level 1: the row's 32-id partials, a contiguous run per
+// thread, give M = max y, S = sum exp(y - M) and the group holding u * S.
+// Level 2: that group's 32 logits, recomputed as dot products of the LM-head
+// rows with the row's operand (the sum of its bf16 planes), in ascending ids.
+__global__ void __launch_bounds__(PK_THREADS) lm_pick_kernel(const LmPickArgs a) {
+    extern __shared__ float hrow[];   // [d] the row's LM-head operand
+    __shared__ MS sm_ms[PK_THREADS / 32];
+    __shared__ AM sm_am[PK_THREADS / 32];
     __shared__ float sh[34];
     __shared__ int si[2];
-    __shared__ int s_tok;
-    __shared__ float s_e;
+    __shared__ float s_z[TC_LM_GROUP];
+    __shared__ int s_grp, s_tok;
+    __shared__ float s_before, s_e;
     const Dims &D = a.dim;
-    const int c = blockIdx.x, b = blockIdx.y, t = threadIdx.x;
+    const int b = blockIdx.x, t = threadIdx.x, warp = t >> 5, lane = t & 31;
     pdl_trigger();
     pdl_wait();
-    if (!a.valid[a.rows_per_valid > 1 ? b / a.rows_per_valid : b]) return;   // every block of the row leaves here
+    if (!a.valid[a.rows_per_valid > 1 ? b / a.rows_per_valid : b]) return;
     const bool greedy = a.temperature == 0.f;
     const float invT = greedy ? 1.f : 1.f / a.temperature;
-    const float *z = a.z + (size_t)b * a.ldz;
-    // chunk statistics of y = z / T: (max, sum exp(y - max)), argmax of z (lowest id)
-    const int base = c * RS_CHUNK + t * RS_PER;
-    float y[RS_PER];
+    const float4 *pp = a.part + (size_t)b * a.nsub;
+    const int per = (a.nsub + PK_THREADS - 1) / PK_THREADS;
+    const int j0 = min(a.nsub, t * per), j1 = min(a.nsub, j0 + per);
     float m = -INFINITY;
     AM am{-INFINITY, 0x7fffffff};
-#pragma unroll
-    for (int k = 0; k < RS_PER; ++k) {
-        const int n = base + k;
-        const float zv = n < D.V ? __ldcg(z + n) : -INFINITY;
-        y[k] = zv * invT;
-        m = fmaxf(m, y[k]);
-        if (zv > am.v) am = AM{zv, n};
+    for (int j = j0; j < j1; ++j) {
+        const float4 p = __ldcg(pp + j);
+        m = fmaxf(m, p.x);
+        am = am_combine(am, AM{p.z, __float_as_int(p.w)});
     }
-    float s = 0.f;
-#pragma unroll
-    for (int k = 0; k < RS_PER; ++k) s += y[k] == -INFINITY ? 0.f : __expf(y[k] - m);
-    const MS ms = block_ms(MS{m, m == -INFINITY ? 0.f : s}, sm_ms);
-    const AM bam = block_am(am, sm_am);
-    if (t == 0) a.part[(size_t)b * a.nch + c] = make_float4(ms.m, ms.s, bam.v, __int_as_float(bam.i));
-    if (!arrive_last(a.ticket + b, a.nch)) return;
-
-    // last block of row b: level 1 over the chunk partials (one per thread)
-    const float4 pv = t < a.nch ? __ldcg(a.part + (size_t)b * a.nch + t) : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
-    const float M = block_ms(MS{pv.x, pv.y}, sm_ms).m;
-    const float cw = t < a.nch && pv.x != -INFINITY ? pv.y * __expf(pv.x - M) : 0.f;
+    const float M = block_ms(MS{m, 0.f}, sm_ms).m;
+    float w = 0.f;
+    for (int j = j0; j < j1; ++j) {
+        const float4 p = __ldcg(pp + j);
+        if (p.x != -INFINITY) w += p.y * __expf(p.x - M);
+    }
     int token;
     float S, qx = 1.f;
     if (greedy) {
-        token = block_am(AM{t < a.nch ? pv.z : -INFINITY, t < a.nch ? __float_as_int(pv.w) : 0x7fffffff}, sm_am).i;
-        S = block_ms(MS{0.f, cw}, sm_ms).s;
+        token = block_am(am, sm_am).i;
+        S = block_ms(MS{0.f, w}, sm_ms).s;
     } else {
         const float u = a.u_draft[(size_t)b * a.K + a.step];
         float tot;
-        block_excl_scan(cw, sh, &tot);
+        block_excl_scan(w, sh, &tot);
         S = tot;
         const float target = u * S;
         float before1;
-        const int ck = rs_pick(cw, t, target, &before1, sh, si);
-        // level 2: the chosen chunk, RS_PER consecutive ids per thread
-        const int b2 = ck * RS_CHUNK + t * RS_PER;
-        float e[RS_PER], mine = 0.f;
-#pragma unroll
-        for (int k = 0; k < RS_PER; ++k) {
-            const int n = b2 + k;
-            e[k] = n < D.V ? __expf(__ldcg(z + n) * invT - M) : 0.f;
-            mine += e[k];
+        const int ct = rs_pick(w, t, target, &before1, sh, si);
+        if (t == ct) {   // this thread's run holds the point: find its group
+            float cum = before1;
+            int grp = -1, lastg = -1;
+            float lastb = before1;
+            for (int j = j0; j < j1; ++j) {
+                const float4 p = __ldcg(pp + j);
+                const float wj = p.x != -INFINITY ? p.y * __expf(p.x - M) : 0.f;
+                if (wj > 0.f) { lastg = j; lastb = cum; }
+                if (wj > 0.f && target < cum + wj) { grp = j; break; }
+                cum += wj;
+            }
+            s_grp = grp >= 0 ? grp : (lastg >= 0 ? lastg : j0);
+            s_before = grp >= 0 ? cum : lastb;
         }
-        float tot2;
-        const float ex = block_excl_scan(mine, sh, &tot2);
-        float cum = before1 + ex;
-        int found = 0x7fffffff, lastp = -1;
-        float efound = 0.f, elast = 0.f;
+        // the row's operand: the sum of its planes (the values the tensor cores multiplied)
+        const size_t plane = (size_t)a.npad * D.d;
+        const uint16_t *q = a.planes + (size_t)b * D.d;
+        for (int k = t; k < D.d; k += PK_THREADS) {
+            float h = 0.f;
 #pragma unroll
-        for (int k = 0; k < RS_PER; ++k) {
-            cum += e[k];
-            if (e[k] > 0.f) { lastp = b2 + k; elast = e[k]; }
-            if (found == 0x7fffffff && e[k] > 0.f && target < cum) { found = b2 + k; efound = e[k]; }
+            for (int i = 0; i < TC_PLANES; ++i) h += bf_to_f(q[i * plane + k]);
+            hrow[k] = h;
         }
-        if (t == 0) { si[0] = 0x7fffffff; si[1] = -1; }
         __syncthreads();
-        if (found != 0x7fffffff) atomicMin(&si[0], found);
-        if (lastp >= 0) atomicMax(&si[1], lastp);
+        const int id0 = s_grp * TC_LM_GROUP;
+        // 8 warps x 4 ids: lanes split the reduction, 8 elements per 16-byte load
+        for (int i = 0; i < TC_LM_GROUP / (PK_THREADS / 32); ++i) {
+            const int id = id0 + warp * (TC_LM_GROUP / (PK_THREADS / 32)) + i;
+            float acc = 0.f;
+            if (id < D.V) {
+                const uint16_t *wr = a.W + (size_t)id * D.d;
+                for (int k = lane * 8; k < D.d; k += 256) {
+                    float wf[8];
+                    unpack8(ld_stream(wr + k), wf);
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], hrow[k + e], acc);
+                }
+            }
+            acc = warp_sum(acc);
+            if (lane == 0) s_z[id - id0] = acc;
+        }
         __syncthreads();
-        const int pick = si[0] != 0x7fffffff ? si[0] : (si[1] >= 0 ? si[1] : ck * RS_CHUNK);
-        if (found == pick) { s_tok = pick; s_e = efound; }
-        else if (si[0] == 0x7fffffff && lastp == pick) { s_tok = pick; s_e = elast; }
+        if (warp == 0) {
+            const int id = id0 + lane;
+            const float e = id < D.V ? __expf(s_z[lane] * invT - M) : 0.f;
+            const float cum = s_before + warp_incl_scan(e);
+            const unsigned hit = __ballot_sync(0xffffffffu, e > 0.f && target < cum);
+            const unsigned pos = __ballot_sync(0xffffffffu, e > 0.f);
+            const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+            if (lane == l) {
+                s_tok = id;
+                s_e = e;
+            }
+        }
         __syncthreads();
         token = s_tok;
         qx = s_e / S;
@@ -538,11 +574,9 @@ __global__ void __launch_bounds__(RS_THREADS) row_sample_kernel(const RowSampleA
         const int src = a.src_is_ext ? b * a.max_new + a.nnew[b] - 1 : b;
         const float *xl = a.x_in + (size_t)src * D.d;
         const uint16_t *er = a.embed + (size_t)token * D.d;
-        for (int k = t; k < D.d; k += RS_THREADS) {
-            const float xv = xl[k];
-            const float ev = bf_to_f(er[k]);
-            a.s_chain[(size_t)b * D.d + k] = xv;
-            a.x_chain[(size_t)b * D.d + k] = ev;
+        for (int k = t; k < D.d; k += PK_THREADS) {
+            a.s_chain[(size_t)b * D.d + k] = xl[k];
+            a.x_chain[(size_t)b * D.d + k] = bf_to_f(er[k]);
         }
     }
 }
@@ -632,6 +666,8 @@ cudaError_t tc_set_attributes() {
     cudaError_t e = cudaFuncSetAttribute(tc_kernel<TC_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_GLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_LM>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) e = allow_smem(lm_pick_kernel);
     return e;
 }
 
@@ -669,7 +705,9 @@ cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorM
     const int nst = tc_stages(a.npad, a.planes, false);
     if (nst < 2) return cudaErrorInvalidValue;
     const int nkb = a.K / 64;
-    a.nsplit = a.part ? tc_nsplit(a.nout, a.K, sms) : 1;
+    if (a.epi == TC_LM && (!a.lm_part || a.lm_nsub != (a.nout + TC_LM_GROUP - 1) / TC_LM_GROUP))
+        return cudaErrorInvalidValue;
+    a.nsplit = a.part && a.epi != TC_LM ? tc_nsplit(a.nout, a.K, sms) : 1;   // the LM epilogue needs whole sums
     if ((long long)a.nsplit * a.R * a.nout > a.part_cap) a.nsplit = 1;
     a.kbps = (nkb + a.nsplit - 1) / a.nsplit;
     const int nseg = (a.kbps + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
@@ -681,7 +719,8 @@ cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorM
     switch (a.epi) {
     case TC_STORE: e = pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
     case TC_RESID: e = pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
-    default: e = pdl_launch(tc_kernel<TC_GLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    case TC_GLU: e = pdl_launch(tc_kernel<TC_GLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    default: e = pdl_launch(tc_kernel<TC_LM>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
     }
     if (e != cudaSuccess || a.nsplit == 1) return e;
     const unsigned rblocks = (unsigned)(((long long)a.R * a.nout + 255) / 256);
@@ -705,9 +744,8 @@ cudaError_t launch_embed_rows(const EmbedArgs &a, cudaStream_t s) {
     return pdl_launch(embed_rows_kernel, dim3(a.R), dim3(256), 0, s, a);
 }
 
-cudaError_t launch_row_sample(const RowSampleArgs &a, cudaStream_t s) {
-    if (a.nch > RS_THREADS) return cudaErrorInvalidValue;
-    return pdl_launch(row_sample_kernel, dim3(a.nch, a.B), dim3(RS_THREADS), 0, s, a);
+cudaError_t launch_lm_pick(const LmPickArgs &a, cudaStream_t s) {
+    return pdl_launch(lm_pick_kernel, dim3(a.B), dim3(PK_THREADS), (size_t)a.dim.d * 4, s, a);
 }
 
 }  // namespace osp

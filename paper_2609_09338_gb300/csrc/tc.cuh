@@ -24,7 +24,11 @@
 
 namespace osp {
 
-enum TcEpi { TC_STORE = 0, TC_RESID = 1, TC_GLU = 2 };
+// TC_LM: the LM head; per row and 32-id group of the vocabulary the epilogue
+// keeps only (max of logits/T, sum of exp(logits/T - max), argmax logit and its
+// id), and stores the logits only when y is given.
+enum TcEpi { TC_STORE = 0, TC_RESID = 1, TC_GLU = 2, TC_LM = 3 };
+constexpr int TC_LM_GROUP = 32;    // vocabulary ids per LM-head partial (one epilogue warp's lanes)
 
 constexpr int TC_MAX_ROWS = 80;    // activation rows per GEMM: three accumulators fit a CTA's 256 TMEM columns
 constexpr int TC_PLANES = 3;       // bf16 planes of a float32 operand
@@ -40,6 +44,10 @@ struct TcArgs {
     float *x;          // TC_RESID: [R][ldy] float32, +=
     uint16_t *h;       // TC_GLU: [TC_PLANES][npad][nout] bf16 planes of silu(gate) * up
     int32_t *status;
+    // TC_LM: partials [R][lm_nsub] (lm_nsub = ceil(nout / 32)), 1/T (1 for greedy)
+    float4 *lm_part;
+    int lm_nsub;
+    float lm_invT;
     // split-K: per-range float32 partials [nsplit][R][nout] (null: no split)
     float *part;
     long long part_cap;   // floats available in part
@@ -93,17 +101,22 @@ struct QkvPostArgs {
 };
 cudaError_t launch_qkv_post(const QkvPostArgs &a, cudaStream_t s);
 
-// Sampling over B logits rows z [B][V] (Sec. 3.1 draft distribution q =
-// softmax(z / T)): inverse CDF at u_draft[b][step] over ascending ids, or the
-// argmax (T = 0); writes the token, q(token), (max, log-sum-exp) and, when a
-// next chain step follows, the next chain row (context slot = x_L, residual =
-// E[token]).
-struct RowSampleArgs {
+// Sampling each LM-head row (Sec. 3.1 draft distribution q = softmax(z / T))
+// from the TC_LM partials: the inverse CDF at u_draft[b][step] over ascending
+// ids picks a 32-id group from the partials, then the id inside it from that
+// group's logits, recomputed from the LM head's operand planes; T = 0 takes the
+// argmax (lowest id).  Writes the token, q(token), (max, log-sum-exp) and, when
+// a next chain step follows, the next chain row (context slot = x_L, residual =
+// E[token]).  Row b belongs to sequence b / rows_per_valid (0 or 1: itself).
+struct LmPickArgs {
     Dims dim;
-    int B, K, step, max_new, src_is_ext;
+    int B, K, step, max_new, src_is_ext, rows_per_valid;
     const int *valid, *nnew;
-    const float *z;            // row b at z + b * ldz
-    long long ldz;
+    const float4 *part;        // [B][nsub] TC_LM partials
+    int nsub;
+    const uint16_t *planes;    // [TC_PLANES][npad][d] bf16 planes of the LM head's rows
+    int npad;
+    const uint16_t *W;         // LM head [V][d]
     float temperature;
     const float *u_draft;
     int32_t *tokens;
@@ -111,12 +124,8 @@ struct RowSampleArgs {
     const float *x_in;         // residual rows of the step (x_ext or x_chain)
     float *x_chain, *s_chain;
     const uint16_t *embed;
-    float4 *part;              // [B][nch] chunk partials
-    int *ticket;               // [B]
-    int nch;
-    int rows_per_valid;        // row b belongs to sequence b / rows_per_valid (0 or 1: itself)
 };
-int row_sample_chunks(int V);
+cudaError_t launch_lm_pick(const LmPickArgs &a, cudaStream_t s);
 // Block drafting inputs (EAGLE-style DFlash): for row r = b*P + j of n
 // sequences, tokens[r] = anchor[b] (j = 0) or mask (j > 0); feats_rep[r] =
 // feats[b] (feat_dim bf16, broadcast over the block); nnew[b] = P.
@@ -138,6 +147,5 @@ struct EmbedArgs {
     float *x;
 };
 cudaError_t launch_embed_rows(const EmbedArgs &a, cudaStream_t s);
-cudaError_t launch_row_sample(const RowSampleArgs &a, cudaStream_t s);
 
 }  // namespace osp

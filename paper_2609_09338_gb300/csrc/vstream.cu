@@ -38,6 +38,9 @@ namespace osp {
 #ifndef OSP_VS_NST
 #define OSP_VS_NST 12  // ring slots per block
 #endif
+#ifndef OSP_VS_EARLY
+#define OSP_VS_EARLY 0   // 1: a consumer copies both rows of its tile to registers and frees the slot first
+#endif
 #ifndef OSP_VS_ROWB
 #define OSP_VS_ROWB 4096   // bytes of one row chunk (the workspace holds 4 KB float32 chunks at least)
 #endif
@@ -329,7 +332,7 @@ __device__ __forceinline__ void vs_row_done(const VerifyArgs &a, size_t row, int
 }
 
 template <typename T, bool GREEDY>
-__global__ void __launch_bounds__(VS_THREADS, 2) vs_stats(const VerifyArgs a) {
+__global__ void __launch_bounds__(VS_THREADS, OSP_VS_BPS) vs_stats(const VerifyArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t full[VS_NST], empty[VS_NST];
     __shared__ int s_abort;
@@ -433,6 +436,25 @@ __global__ void __launch_bounds__(VS_THREADS, 2) vs_stats(const VerifyArgs a) {
             }
             am = warp_am(am);
             part = make_float4(am.v, __int_as_float(am.i), 0.f, 0.f);
+        } else if (OSP_VS_EARLY) {
+            // both rows to registers, the slot freed, then the sums
+            uint4 rq[VS_NV];
+            if (has_q) {
+                vs_stage(chunk + VS_ROWB, lane, rq);
+                if (!whole) vs_mask<T>(rq, lane, nel);
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&empty[slot]);
+            const float xp = L::vmax(rv);
+            const float sp = xp == -INFINITY ? 0.f : vs_sum_exp<T>(rv, cexp, xp * cexp);
+            float xq = -INFINITY, sq = 0.f;
+            if (has_q) {
+                xq = L::vmax(rq);
+                sq = xq == -INFINITY ? 0.f : vs_sum_exp<T>(rq, cexp, xq * cexp);
+            }
+            const MS p = vs_warp_ms(xp * invT, sp);
+            const MS q = has_q ? vs_warp_ms(xq * invT, sq) : MS{-INFINITY, 0.f};
+            part = make_float4(p.m, p.s, q.m, q.s);
         } else {
             // maxima of the raw logits (order is kept by the positive 1/T), then
             // sums of exp((z - max) / T)
@@ -641,7 +663,7 @@ __device__ void vs_pick(const VerifyArgs &a, int b, const Decision &d) {
 }
 
 template <typename T>
-__global__ void __launch_bounds__(VS_THREADS, 2) vs_sample(const VerifyArgs a) {
+__global__ void __launch_bounds__(VS_THREADS, OSP_VS_BPS) vs_sample(const VerifyArgs a) {
     extern __shared__ __align__(128) uint8_t smem[];
     __shared__ __align__(8) uint64_t full[VS_NST], empty[VS_NST];
     __shared__ int s_abort;

@@ -35,7 +35,7 @@ def _dev(a):
 
 
 def run_case(shape, ctx, K, T, seed, n_new=None, max_new=1, zero=False, peaked=False, sample_seqs=None,
-             feats_seed=None):
+             feats_seed=None, with_logits=True):
     from paper_2609_09338_gb300.binding import to_device_bf16
     from paper_2609_09338_gb300.session import DraftSession
     ctx = np.asarray(ctx, np.int32)
@@ -49,7 +49,7 @@ def run_case(shape, ctx, K, T, seed, n_new=None, max_new=1, zero=False, peaked=F
         di["n_new"] = np.asarray(n_new, np.int32)
     sess = DraftSession(shape, w, kv["page_table"], kv["n_pages"], K, max_new)
     sess.append(ctx, kv["k_rows"], kv["v_rows"])
-    out = sess.draft_buffers(with_logits=True)
+    out = sess.draft_buffers(with_logits=with_logits)
     sess.draft(_dev(di["n_new"]), _dev(di["tokens"]), to_device_bf16(di["feats"]), T, _dev(di["u_draft"]), out)
     torch.cuda.synchronize()
     g = {k: (v.cpu().numpy() if v is not None else None) for k, v in out.items()}
@@ -192,6 +192,20 @@ def test_free_running_chain_error_growth(name):
                     max_new=wl.n_new, sample_seqs=[0, wl.batch - 1])
     per_step = check_free_running(case)
     print(f"free-running {name}: max abs logit error per chain step {per_step}")
+
+
+@pytest.mark.parametrize("name,T", [("qwen3-8b-d1024-v151936-b32-k7", 1.0), ("qwen3-8b-d1024-v151936-b32-k7", 0.0),
+                                    ("qwen3-8b-d1024-v151936-b1-k7", 1.0)])
+def test_logits_kept_on_chip_same_draft(name, T):
+    """The LM head samples from its epilogue's partials and recomputes only the
+    chosen 32-id group: storing the logits (a test-only output) changes no
+    token, q(token), statistic or cached row."""
+    wl = WORKLOADS[name]
+    ctx = syn.make_contexts(wl)
+    a = run_case(wl.shape, ctx, wl.K, T, wl.seed, with_logits=True)
+    b = run_case(wl.shape, ctx, wl.K, T, wl.seed, with_logits=False)
+    for k in ("draft_tokens", "draft_qx", "draft_stats", "k_pages", "v_pages"):
+        np.testing.assert_array_equal(a["g"][k], b["g"][k])
 
 
 @pytest.mark.parametrize("T", [0.0, 1.0])
