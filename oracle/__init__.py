@@ -16,9 +16,12 @@ Everything is plain numpy in float64, written from the paper:
   uniforms;
 * ``oracle.dflash`` - the EAGLE-style DFlash block drafter (Appendix, "EAGLE-
   Style Target Interface for DFlash"): one causal forward over an anchor and
-  mask placeholders, the target feature broadcast through the expanded QKV.
+  mask placeholders, the target feature broadcast through the expanded QKV;
+* ``oracle.tree`` - verification of a draft tree (topk > 1): the multi-
+  candidate form of the Sec. 3.1 rule over a branching chain, which is the
+  chain rule at topk = 1.
 
 Every function below is pinned by a ``-m "not gpu"`` test against something
 other than itself (closed forms, library routines, invariants, brute force).
 """
-from . import bf16, dflash, drafter, verify  # noqa: F401
+from . import bf16, dflash, drafter, tree, verify  # noqa: F401
