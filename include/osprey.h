@@ -184,6 +184,55 @@ int osprey_draft_step_hidden(osprey_ctx *ctx, const osprey_kv *kv, int B, int K,
                              float *draft_qx, float *draft_stats, float *draft_hidden,
                              void *workspace, size_t workspace_bytes, int32_t *dev_status, void *stream);
 
+/* Tree drafting (topk > 1; the paper serves chains, topk = 1, Sec. 4 inference
+ * settings): osprey_draft_step whose LM head draws topk candidates per chain
+ * step.  Candidate j of step k is the inverse CDF of q_k at u_draft[b][k][j]
+ * (independent draws; at T = 0 the topk highest logits in descending order,
+ * ties to the lowest id); candidate 0 continues the chain (Sec. 3.4), the
+ * others are leaves of the branching chain that osprey_verify_tree checks.
+ *   topk 1 .. 8; topk > 1 needs the tensor-core LM head (B <= 80 and a device
+ *        with tcgen05, else SHAPE)
+ *   u_draft [B][K][topk]; cand [B][K][topk] int32; cand_qx [B][K][topk] q of
+ *   each candidate (1 for greedy; may be NULL); draft_stats [B][K][2] and
+ *   draft_logits [B][K][V] as osprey_draft_step.  Workspace: as
+ *   osprey_draft_step (osprey_draft_workspace_bytes). */
+int osprey_draft_step_topk(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int topk, int max_new,
+                           const int32_t *n_new, const int32_t *tokens, const void *feats, float temperature,
+                           const float *u_draft, int32_t *cand, float *cand_qx, float *draft_stats,
+                           float *draft_logits, void *workspace, size_t workspace_bytes, int32_t *dev_status,
+                           void *stream);
+
+/* Verification of a draft tree (the multi-candidate form of the Sec. 3.1 rule;
+ * topk = 1 gives osprey_verify's result).  The tree is a branching chain: at
+ * depth i < K the topk candidates cand[b][i][*] were drawn from the drafter's
+ * q_i = softmax(draft_logits[b][i] / T); candidate 0 continues the chain.
+ *   target_logits [B][1 + K*topk][V]: row 0 is the target's distribution after
+ *          the verified prefix, row 1 + i*topk + j the one after the path to
+ *          candidate j of depth i
+ *   draft_logits [B][K][V] (NULL iff T == 0), same dtype
+ *   u_accept [B][K][topk], u_sample [B][K+1] float in [0,1)
+ * The walk: at depth i, with p the current node's row and the residual r = p,
+ * candidate j is accepted iff u_accept[i][j] < r(x) / q_i(x), and a rejection
+ * sets r = norm(max(0, r - q_i)).  An accepted candidate 0 below depth K - 1
+ * moves on to depth i + 1; an accepted leaf or depth K - 1 ends the walk with a
+ * draw from that node's row at u_sample[i + 1]; topk rejections end it with a
+ * draw from r at u_sample[i].  Greedy: the current node's argmax is accepted
+ * when it is a candidate (the first such).  Draws are inverse CDFs over
+ * ascending ids.
+ * Outputs (device): out_tokens [B][K+1] (accepted candidates, the drawn
+ *   token, then -1), n_accepted [B], branch [B] (the candidate index accepted
+ *   at the last accepted depth, -1 if none), flags [B][K+1] (bit 3: a residual
+ *   without float32 mass, p sampled instead; bit 4: the draw clamped to the
+ *   last id with weight).
+ * No workspace: one block per sequence keeps its walk on chip; rows off the
+ * walked path are never read.  V <= 2^20.
+ * Device errors: INVALID_ARG for a candidate outside [0, V) (that sequence gets
+ * n_accepted 0 and out_tokens -1). */
+int osprey_verify_tree(int B, int K, int topk, int V, int logits_dtype, const void *target_logits,
+                       const void *draft_logits, const int32_t *cand, float temperature, const float *u_accept,
+                       const float *u_sample, int32_t *out_tokens, int32_t *n_accepted, int32_t *branch,
+                       uint8_t *flags, int32_t *dev_status, void *stream);
+
 /* Bytes of workspace osprey_dflash_step needs.  0 on bad arguments. */
 size_t osprey_dflash_workspace_bytes(const osprey_ctx *ctx, int B, int block, int max_pages_per_seq);
 

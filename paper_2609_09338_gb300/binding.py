@@ -81,6 +81,12 @@ _c_draft = _sig("osprey_draft_step", ctypes.c_int,
 _c_draft_hidden = _sig("osprey_draft_step_hidden", ctypes.c_int,
                        [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp, _f32,
                         _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp])
+_c_draft_topk = _sig("osprey_draft_step_topk", ctypes.c_int,
+                     [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp,
+                      _vp, ctypes.c_float, _vp, _vp, _vp, _vp, _vp, _vp, _sz, _vp, _vp])
+_c_verify_tree = _sig("osprey_verify_tree", ctypes.c_int,
+                      [ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int, _vp, _vp, _vp,
+                       ctypes.c_float, _vp, _vp, _vp, _vp, _vp, _vp, _vp, _vp])
 _c_dflash_ws = _sig("osprey_dflash_workspace_bytes", _sz, [_vp, ctypes.c_int, ctypes.c_int, ctypes.c_int])
 _c_dflash = _sig("osprey_dflash_step", ctypes.c_int,
                  [_vp, ctypes.POINTER(osprey_kv), ctypes.c_int, ctypes.c_int, _vp, ctypes.c_int32, _vp,
@@ -103,7 +109,8 @@ _c_launch_count = _sig("osprey_launch_count", _i64, [])
 _c_selftest_wait = _sig("osprey_selftest_wait_timeout", ctypes.c_int, [_i64, _vp, _vp])
 
 EXPORTED = ["osprey_last_error", "osprey_create", "osprey_destroy", "osprey_draft_workspace_bytes",
-            "osprey_kv_append", "osprey_draft_step", "osprey_draft_step_hidden", "osprey_dflash_workspace_bytes",
+            "osprey_kv_append", "osprey_draft_step", "osprey_draft_step_hidden", "osprey_draft_step_topk",
+            "osprey_verify_tree", "osprey_dflash_workspace_bytes",
             "osprey_dflash_step", "osprey_verify_workspace_bytes",
             "osprey_verify", "osprey_verify_static", "osprey_verify_hidden_workspace_bytes", "osprey_verify_hidden",
             "osprey_probe_enable", "osprey_probe_select", "osprey_probe_read", "osprey_launch_count", "osprey_selftest_wait_timeout"]
@@ -311,6 +318,63 @@ def osprey_draft_step_hidden(ctx: Ctx, kv: KvCache, n_new: torch.Tensor, tokens:
     _check(_c_draft_hidden(ctx.handle, ctypes.byref(kvs), B, K, max_new, _ptr(n_new), _ptr(tokens), _ptr(feats),
                            float(temperature), _ptr(u_draft), _ptr(draft_tokens), _ptr(draft_qx), _ptr(draft_stats),
                            _ptr(draft_hidden), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+
+
+def osprey_draft_step_topk(ctx: Ctx, kv: KvCache, n_new: torch.Tensor, tokens: torch.Tensor, feats: torch.Tensor,
+                           temperature: float, u_draft, cand: torch.Tensor, cand_qx=None, draft_stats=None,
+                           draft_logits=None, workspace: torch.Tensor = None, status: torch.Tensor = None, stream=None):
+    """A draft call drawing topk candidates per chain step (cand [B, K, topk]);
+    candidate 0 continues the chain."""
+    s = ctx.shape
+    B, max_new = tokens.shape
+    K, k = cand.shape[1], cand.shape[2]
+    _need(n_new, torch.int32, (B,), "n_new")
+    _need(tokens, torch.int32, (B, max_new), "tokens")
+    _need(feats, torch.bfloat16, (B, max_new, s.feat_dim), "feats")
+    _need(cand, torch.int32, (B, K, k), "cand")
+    if u_draft is not None:
+        _need(u_draft, torch.float32, (B, K, k), "u_draft")
+    if cand_qx is not None:
+        _need(cand_qx, torch.float32, (B, K, k), "cand_qx")
+    if draft_stats is not None:
+        _need(draft_stats, torch.float32, (B, K, 2), "draft_stats")
+    if draft_logits is not None:
+        _need(draft_logits, torch.float32, (B, K, s.vocab), "draft_logits")
+    _need(workspace, torch.uint8, None, "workspace")
+    _need(status, torch.int32, (1,), "status")
+    if kv.page_table.shape[0] != B:
+        raise ValueError("page table rows must equal the batch")
+    kvs = kv.c_struct()
+    _check(_c_draft_topk(ctx.handle, ctypes.byref(kvs), B, K, k, max_new, _ptr(n_new), _ptr(tokens), _ptr(feats),
+                         float(temperature), _ptr(u_draft), _ptr(cand), _ptr(cand_qx), _ptr(draft_stats),
+                         _ptr(draft_logits), _ptr(workspace), workspace.numel(), _ptr(status), _stream(stream)))
+
+
+def osprey_verify_tree(target_logits: torch.Tensor, draft_logits, cand: torch.Tensor, temperature: float, u_accept,
+                       u_sample, out_tokens: torch.Tensor, n_accepted: torch.Tensor, branch: torch.Tensor,
+                       flags: torch.Tensor, status: torch.Tensor, stream=None):
+    """Verify a branching-chain draft tree: target [B, 1 + K*topk, V], draft
+    [B, K, V] (None when greedy), cand [B, K, topk]."""
+    B, K, k = cand.shape
+    V = target_logits.shape[-1]
+    dt = {torch.float32: OSPREY_F32, torch.bfloat16: OSPREY_BF16}.get(target_logits.dtype)
+    if dt is None:
+        raise ValueError("logits must be float32 or bfloat16")
+    _need(target_logits, target_logits.dtype, (B, 1 + K * k, V), "target_logits")
+    if draft_logits is not None:
+        _need(draft_logits, target_logits.dtype, (B, K, V), "draft_logits")
+    _need(cand, torch.int32, (B, K, k), "cand")
+    if temperature > 0:
+        _need(u_accept, torch.float32, (B, K, k), "u_accept")
+        _need(u_sample, torch.float32, (B, K + 1), "u_sample")
+    _need(out_tokens, torch.int32, (B, K + 1), "out_tokens")
+    _need(n_accepted, torch.int32, (B,), "n_accepted")
+    _need(branch, torch.int32, (B,), "branch")
+    _need(flags, torch.uint8, (B, K + 1), "flags")
+    _need(status, torch.int32, (1,), "status")
+    _check(_c_verify_tree(B, K, k, V, dt, _ptr(target_logits), _ptr(draft_logits), _ptr(cand), float(temperature),
+                          _ptr(u_accept), _ptr(u_sample), _ptr(out_tokens), _ptr(n_accepted), _ptr(branch),
+                          _ptr(flags), _ptr(status), _stream(stream)))
 
 
 def osprey_dflash_workspace_bytes(ctx: Ctx, B: int, block: int, max_pages: int) -> int:

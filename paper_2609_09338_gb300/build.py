@@ -19,7 +19,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libosprey.so")
-SOURCES = ["api.cu", "verify.cu", "vstream.cu", "kv.cu", "draft.cu", "stream.cu", "tc.cu", "mlp.cu"]
+SOURCES = ["api.cu", "verify.cu", "vstream.cu", "kv.cu", "draft.cu", "stream.cu", "tc.cu", "mlp.cu", "tree.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

@@ -382,7 +382,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
                            const int32_t *n_new, const int32_t *tokens, const void *feats, float temperature,
                            const float *u_draft, int32_t *draft_tokens, float *draft_qx, float *draft_stats,
                            float *draft_logits, float *draft_hidden, void *workspace, size_t workspace_bytes,
-                           int32_t *dev_status, void *stream, bool block = false) {
+                           int32_t *dev_status, void *stream, bool block = false, int topk = 1) {
     g_err[0] = 0;
     if (!ctx || !kv) return fail(OSPREY_ERR_INVALID_ARG, "null context or kv");
     if (B == 0) return OSPREY_OK;
@@ -403,6 +403,9 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         return fail(OSPREY_ERR_CAPACITY, "workspace too small: %zu < %zu bytes", workspace_bytes, need);
     if (block && (K != 1 || !ctx->tc || B * max_new < 3 || B * max_new > TC_MAX_ROWS))
         return fail(OSPREY_ERR_SHAPE, "block drafting runs 3..%d rows per group on the tensor cores", TC_MAX_ROWS);
+    if (topk > 1 && (!ctx->tc || B > TC_MAX_ROWS))
+        return fail(OSPREY_ERR_SHAPE, "topk > 1 samples on the tensor-core LM head: at most %d sequences and a "
+                                      "device with tcgen05 (not OSPREY_TC=0)", TC_MAX_ROWS);
 
     cudaStream_t s = (cudaStream_t)stream;
     const Dims &D = ctx->dim;
@@ -414,7 +417,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
     PrepArgs pa{B, K, max_new, kv->max_pages_per_seq, kv->n_pages, D.P, D.V,
                 kv->seq_len, n_new, tokens, kv->page_table,
                 ws.seq_valid, ws.seq_pos0, ws.seq_nnew, draft_tokens, dev_status, ws.counters, ws.n_counters,
-                block ? 1 : 0, block ? max_new : 0};
+                block ? 1 : 0, block ? max_new : (topk > 1 ? K * topk : 0)};
     if ((e = launch_prepare(pa, s)) != cudaSuccess) return cuda_fail(e, "prepare launch");
 
     GemvArgs g{};
@@ -768,7 +771,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             pk.qx = draft_qx;
             pk.stats = draft_stats;
             if ((rc = tc_lm(rows, draft_logits, D.V, pk)) != OSPREY_OK) return rc;
-        } else if (B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
+        } else if (topk <= 1 && B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) {
             plan_into(G_LM);
             sa.W = (const uint16_t *)W.lm_head;
             sa.gain = (const uint16_t *)W.final_norm;
@@ -786,9 +789,10 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             sa.cta_stats = ws.lm_cta_stats;
             sa.ticket = ws.lm_ticket;
             if ((e = launch_stream(G_LM, sa, B, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");
-        } else if (tc_rows(B)) {
+        } else if (tc_rows(B) || topk > 1) {
             // final RMSNorm rows -> LM head with the sampling partials in its
             // epilogue (logits stored only into draft_logits) -> one pick per row
+            // (topk candidates per row when drafting a tree)
             int rc;
             if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand")) !=
                 OSPREY_OK)
@@ -799,6 +803,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             pk.step = step;
             pk.max_new = max_new;
             pk.src_is_ext = ext;
+            pk.topk = topk;
             pk.valid = ws.seq_valid;
             pk.nnew = ws.seq_nnew;
             pk.tokens = draft_tokens;
@@ -867,6 +872,20 @@ extern "C" int osprey_draft_step_hidden(osprey_ctx *ctx, const osprey_kv *kv, in
     }
     return draft_step_impl(ctx, kv, B, K, max_new, n_new, tokens, feats, temperature, u_draft, draft_tokens, draft_qx,
                            draft_stats, nullptr, draft_hidden, workspace, workspace_bytes, dev_status, stream);
+}
+
+extern "C" int osprey_draft_step_topk(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, int topk, int max_new,
+                                      const int32_t *n_new, const int32_t *tokens, const void *feats,
+                                      float temperature, const float *u_draft, int32_t *cand, float *cand_qx,
+                                      float *draft_stats, float *draft_logits, void *workspace,
+                                      size_t workspace_bytes, int32_t *dev_status, void *stream) {
+    if (topk < 1 || topk > 8) {
+        g_err[0] = 0;
+        return fail(OSPREY_ERR_INVALID_ARG, "topk must be in 1..8");
+    }
+    return draft_step_impl(ctx, kv, B, K, max_new, n_new, tokens, feats, temperature, u_draft, cand, cand_qx,
+                           draft_stats, draft_logits, nullptr, workspace, workspace_bytes, dev_status, stream, false,
+                           topk);
 }
 
 // ------------------------------------------------------------------ block drafting
@@ -1009,6 +1028,30 @@ extern "C" int osprey_verify(int B, int K, int V, int logits_dtype, const void *
     if (e != cudaSuccess) return cuda_fail(e, "clearing the verify counters");
     e = launch_verify(a, (cudaStream_t)stream);
     return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "verify launch");
+}
+
+// ------------------------------------------------------------------ tree verify
+extern "C" int osprey_verify_tree(int B, int K, int topk, int V, int logits_dtype, const void *target_logits,
+                                  const void *draft_logits, const int32_t *cand, float temperature,
+                                  const float *u_accept, const float *u_sample, int32_t *out_tokens,
+                                  int32_t *n_accepted, int32_t *branch, uint8_t *flags, int32_t *dev_status,
+                                  void *stream) {
+    g_err[0] = 0;
+    if (B == 0) return OSPREY_OK;
+    if (B < 0 || B > 65535 || K < 1 || K > 64 || topk < 1 || topk > 8 || V < 1 || V > (1 << 20))
+        return fail(OSPREY_ERR_INVALID_ARG, "B in 0..65535, K in 1..64, topk in 1..8 and V in 1..2^20 required");
+    if (logits_dtype != OSPREY_F32 && logits_dtype != OSPREY_BF16)
+        return fail(OSPREY_ERR_DTYPE, "logits_dtype must be OSPREY_F32 or OSPREY_BF16");
+    if (!(temperature >= 0.f) || !std::isfinite(temperature))
+        return fail(OSPREY_ERR_INVALID_ARG, "temperature must be finite and >= 0");
+    if (!target_logits || !cand || !out_tokens || !n_accepted || !branch || !flags)
+        return fail(OSPREY_ERR_INVALID_ARG, "null pointer");
+    if (temperature > 0.f && (!draft_logits || !u_accept || !u_sample))
+        return fail(OSPREY_ERR_INVALID_ARG, "draft_logits, u_accept and u_sample are required when temperature > 0");
+    VerifyTreeArgs a{B, K, topk, V, logits_dtype, temperature, target_logits, draft_logits, cand, u_accept, u_sample,
+                     out_tokens, n_accepted, branch, flags, dev_status};
+    const cudaError_t e = launch_verify_tree(a, (cudaStream_t)stream);
+    return e == cudaSuccess ? OSPREY_OK : cuda_fail(e, "tree verify launch");
 }
 
 // ------------------------------------------------------------------ logits-free verify

@@ -111,6 +111,20 @@ cudaError_t launch_verify_hidden_sample(const VerifyArgs &a, int b0, int n, cuda
 cudaError_t launch_decision_rows(const void *dec, const float *hidden, int K, int d, int b0, int n, float *dst,
                                  cudaStream_t s);
 
+// ---------------------------------------------------------------- tree verify
+struct VerifyTreeArgs {
+    int B, K, k, V, dtype;
+    float temperature;
+    const void *target;   // [B][1 + K k][V]: the root, then node (i, j) at row 1 + i k + j
+    const void *draft;    // [B][K][V] (null when greedy)
+    const int32_t *cand;  // [B][K][k]
+    const float *u_accept, *u_sample;   // [B][K][k], [B][K+1]
+    int32_t *out_tokens, *n_accepted, *branch;
+    uint8_t *flags;
+    int32_t *status;
+};
+cudaError_t launch_verify_tree(const VerifyTreeArgs &a, cudaStream_t s);
+
 // ---------------------------------------------------------------- kv append
 struct KvAppendArgs {
     void *k_pages, *v_pages;

@@ -103,6 +103,19 @@ __device__ __forceinline__ void tc_split(float x, uint16_t (&q)[TC_PLANES]) {
     }
 }
 
+// Merges two (argmax logit a with its id i, sum s of exp((z - a) / T)) pairs
+// into the first: the larger logit wins (the lower id on ties) and the
+// other's sum is rescaled to it.
+__device__ __forceinline__ void lm_combine(float &a1, int &i1, float &s1, float a2, int i2, float s2, float invT) {
+    const bool two = a2 > a1 || (a2 == a1 && i2 < i1);
+    const float aw = two ? a2 : a1, al = two ? a1 : a2;
+    const float sw = two ? s2 : s1, sl = two ? s1 : s2;
+    const float f = al == -INFINITY ? 0.f : __expf((al - aw) * invT);
+    a1 = aw;
+    i1 = two ? i2 : i1;
+    s1 = sw + sl * f;
+}
+
 // ---------------------------------------------------------------- GEMM kernel
 template <int EPI>
 __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
@@ -274,21 +287,48 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                         continue;
                     }
                     if (EPI == TC_LM) {
-                        // per row: (max y, sum exp(y - max), argmax z) over this warp's 32 ids
+                        // per row: (argmax z, sum exp((z - max z) / T)) over this warp's 32
+                        // ids, for the 16 rows c0.. at once: each butterfly round halves the
+                        // rows a lane carries (it keeps one half and receives the partner's
+                        // share of it), so after four rounds lane l holds row l / 2 over 16
+                        // lanes and one more exchange completes it over all 32
                         const int sub = (int)(((long long)((i0 + it) / a.nsplit) * 128 + lg) / TC_LM_GROUP);
+                        float av[16], sv[16];
+                        int ai[16];
 #pragma unroll
                         for (int j = 0; j < 16; ++j) {
-                            const int n = c0 + j;   // the same for every lane of the warp
-                            if (n >= a.R) break;
-                            const float zv = colok ? v[j] : -INFINITY;
-                            if (a.y && colok) a.y[(size_t)n * a.ldy + col] = zv;
-                            const AM am = warp_am(AM{zv, colok ? col : 0x7fffffff});
-                            const float mx = am.v * a.lm_invT;
-                            const float ev = colok ? __expf(zv * a.lm_invT - mx) : 0.f;
-                            const float se = warp_sum(ev);
-                            if (lane == 0 && sub < a.lm_nsub)
-                                a.lm_part[(size_t)n * a.lm_nsub + sub] = make_float4(mx, se, am.v, __int_as_float(am.i));
+                            av[j] = colok ? v[j] : -INFINITY;
+                            ai[j] = colok ? col : 0x7fffffff;
+                            sv[j] = colok ? 1.f : 0.f;
+                            if (a.y && colok && c0 + j < a.R) a.y[(size_t)(c0 + j) * a.ldy + col] = v[j];
                         }
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            const int off = 16 >> r, w = 8 >> r;
+                            const bool up = lane & off;
+#pragma unroll
+                            for (int i = 0; i < w; ++i) {
+                                const float ra = __shfl_xor_sync(0xffffffffu, up ? av[i] : av[i + w], off);
+                                const int ri = __shfl_xor_sync(0xffffffffu, up ? ai[i] : ai[i + w], off);
+                                const float rs = __shfl_xor_sync(0xffffffffu, up ? sv[i] : sv[i + w], off);
+                                float ka = up ? av[i + w] : av[i], ks = up ? sv[i + w] : sv[i];
+                                int ki = up ? ai[i + w] : ai[i];
+                                lm_combine(ka, ki, ks, ra, ri, rs, a.lm_invT);
+                                av[i] = ka;
+                                ai[i] = ki;
+                                sv[i] = ks;
+                            }
+                        }
+                        {
+                            const float ra = __shfl_xor_sync(0xffffffffu, av[0], 1);
+                            const int ri = __shfl_xor_sync(0xffffffffu, ai[0], 1);
+                            const float rs = __shfl_xor_sync(0xffffffffu, sv[0], 1);
+                            lm_combine(av[0], ai[0], sv[0], ra, ri, rs, a.lm_invT);
+                        }
+                        const int n = c0 + (lane >> 1);
+                        if (!(lane & 1) && n < a.R && sub < a.lm_nsub)
+                            a.lm_part[(size_t)n * a.lm_nsub + sub] =
+                                make_float4(av[0] * a.lm_invT, sv[0], av[0], __int_as_float(ai[0]));
                         continue;
                     }
 #pragma unroll
@@ -434,41 +474,50 @@ __global__ void __launch_bounds__(256) qkv_post_kernel(const QkvPostArgs a) {
 // ---------------------------------------------------------------- LM-head pick
 constexpr int PK_THREADS = 256;
 
-// Block-wide ordered pick over one weight per thread: the smallest index i
-// with t < C_i (inclusive cumulative weight, positive weights only); if
-// rounding leaves t past the total, the last index with weight.  Returns the
-// index and the cumulative weight before it in *before.
-__device__ int rs_pick(float w, int idx, float t, float *before, float *sh, int *si) {
-    float tot;
-    const float ex = block_excl_scan(w, sh, &tot);
-    if (threadIdx.x == 0) { si[0] = 0x7fffffff; si[1] = -1; }
-    __syncthreads();
-    if (w > 0.f && t < ex + w) atomicMin(&si[0], idx);
-    if (w > 0.f) atomicMax(&si[1], idx);
-    __syncthreads();
-    const int pick = si[0] != 0x7fffffff ? si[0] : (si[1] >= 0 ? si[1] : 0);
-    if (idx == pick) sh[32] = ex;
-    __syncthreads();
-    *before = sh[32];
-    __syncthreads();
-    return pick;
+constexpr int PK_MAXK = 8;   // candidates per row at most
+
+// Recomputes the 32 logits of group g (ids 32 g ..): 8 warps x 4 ids, lanes
+// split the reduction over the row's operand in shared memory.
+__device__ __forceinline__ void pk_group_logits(const LmPickArgs &a, const float *hrow, int g, float *z) {
+    const Dims &D = a.dim;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    constexpr int PER = TC_LM_GROUP / (PK_THREADS / 32);
+    for (int i = 0; i < PER; ++i) {
+        const int id = g * TC_LM_GROUP + warp * PER + i;
+        float acc = 0.f;
+        if (id < D.V) {
+            const uint16_t *wr = a.W + (size_t)id * D.d;
+            for (int k = lane * 8; k < D.d; k += 256) {
+                float wf[8];
+                unpack8(ld_stream(wr + k), wf);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], hrow[k + e], acc);
+            }
+        }
+        acc = warp_sum(acc);
+        if (lane == 0) z[warp * PER + i] = id < D.V ? acc : -INFINITY;
+    }
 }
 
 // One block per row.  Level 1: the row's 32-id partials, a contiguous run per
-// thread, give M = max y, S = sum exp(y - M) and the group holding u * S.
-// Level 2: that group's 32 logits, recomputed as dot products of the LM-head
-// rows with the row's operand (the sum of its bf16 planes), in ascending ids.
+// thread, give M = max y, S = sum exp(y - M) and, per draw, the group holding
+// u * S.  Level 2: that group's 32 logits, recomputed as dot products of the
+// LM-head rows with the row's operand (the sum of its bf16 planes), scanned in
+// ascending ids.  Greedy: the argmax from the partials; with topk > 1 the next
+// candidates come from the topk groups of largest maximum (the only groups
+// that can hold one of the topk largest logits), recomputed and ranked.
 __global__ void __launch_bounds__(PK_THREADS) lm_pick_kernel(const LmPickArgs a) {
     extern __shared__ float hrow[];   // [d] the row's LM-head operand
     __shared__ MS sm_ms[PK_THREADS / 32];
     __shared__ AM sm_am[PK_THREADS / 32];
     __shared__ float sh[34];
     __shared__ int si[2];
-    __shared__ float s_z[TC_LM_GROUP];
-    __shared__ int s_grp, s_tok;
-    __shared__ float s_before, s_e;
+    __shared__ float s_z[PK_MAXK * TC_LM_GROUP];
+    __shared__ int s_grp[PK_MAXK], s_tok[PK_MAXK];
+    __shared__ float s_before, s_e[PK_MAXK];
     const Dims &D = a.dim;
     const int b = blockIdx.x, t = threadIdx.x, warp = t >> 5, lane = t & 31;
+    const int topk = a.topk > 1 ? a.topk : 1;
     pdl_trigger();
     pdl_wait();
     if (!a.valid[a.rows_per_valid > 1 ? b / a.rows_per_valid : b]) return;
@@ -477,46 +526,24 @@ __global__ void __launch_bounds__(PK_THREADS) lm_pick_kernel(const LmPickArgs a)
     const float4 *pp = a.part + (size_t)b * a.nsub;
     const int per = (a.nsub + PK_THREADS - 1) / PK_THREADS;
     const int j0 = min(a.nsub, t * per), j1 = min(a.nsub, j0 + per);
-    float m = -INFINITY;
+    // one pass over the thread's run: its argmax and its (max, sum) rescaled online
+    float m = -INFINITY, sm = 0.f;
     AM am{-INFINITY, 0x7fffffff};
     for (int j = j0; j < j1; ++j) {
         const float4 p = __ldcg(pp + j);
-        m = fmaxf(m, p.x);
         am = am_combine(am, AM{p.z, __float_as_int(p.w)});
-    }
-    const float M = block_ms(MS{m, 0.f}, sm_ms).m;
-    float w = 0.f;
-    for (int j = j0; j < j1; ++j) {
-        const float4 p = __ldcg(pp + j);
-        if (p.x != -INFINITY) w += p.y * __expf(p.x - M);
-    }
-    int token;
-    float S, qx = 1.f;
-    if (greedy) {
-        token = block_am(am, sm_am).i;
-        S = block_ms(MS{0.f, w}, sm_ms).s;
-    } else {
-        const float u = a.u_draft[(size_t)b * a.K + a.step];
-        float tot;
-        block_excl_scan(w, sh, &tot);
-        S = tot;
-        const float target = u * S;
-        float before1;
-        const int ct = rs_pick(w, t, target, &before1, sh, si);
-        if (t == ct) {   // this thread's run holds the point: find its group
-            float cum = before1;
-            int grp = -1, lastg = -1;
-            float lastb = before1;
-            for (int j = j0; j < j1; ++j) {
-                const float4 p = __ldcg(pp + j);
-                const float wj = p.x != -INFINITY ? p.y * __expf(p.x - M) : 0.f;
-                if (wj > 0.f) { lastg = j; lastb = cum; }
-                if (wj > 0.f && target < cum + wj) { grp = j; break; }
-                cum += wj;
-            }
-            s_grp = grp >= 0 ? grp : (lastg >= 0 ? lastg : j0);
-            s_before = grp >= 0 ? cum : lastb;
+        if (p.x == -INFINITY) continue;
+        if (p.x > m) {
+            sm = (m == -INFINITY ? 0.f : sm * __expf(m - p.x)) + p.y;
+            m = p.x;
+        } else {
+            sm += p.y * __expf(p.x - m);
         }
+    }
+    const MS tot = block_ms(MS{m, sm}, sm_ms);
+    const float M = tot.m, S = tot.s;
+    const float w = m == -INFINITY ? 0.f : sm * __expf(m - M);   // the run's weight
+    if (topk > 1 || !greedy) {
         // the row's operand: the sum of its planes (the values the tensor cores multiplied)
         const size_t plane = (size_t)a.npad * D.d;
         const uint16_t *q = a.planes + (size_t)b * D.d;
@@ -526,51 +553,98 @@ __global__ void __launch_bounds__(PK_THREADS) lm_pick_kernel(const LmPickArgs a)
             for (int i = 0; i < TC_PLANES; ++i) h += bf_to_f(q[i * plane + k]);
             hrow[k] = h;
         }
-        __syncthreads();
-        const int id0 = s_grp * TC_LM_GROUP;
-        // 8 warps x 4 ids: lanes split the reduction, 8 elements per 16-byte load
-        for (int i = 0; i < TC_LM_GROUP / (PK_THREADS / 32); ++i) {
-            const int id = id0 + warp * (TC_LM_GROUP / (PK_THREADS / 32)) + i;
-            float acc = 0.f;
-            if (id < D.V) {
-                const uint16_t *wr = a.W + (size_t)id * D.d;
-                for (int k = lane * 8; k < D.d; k += 256) {
-                    float wf[8];
-                    unpack8(ld_stream(wr + k), wf);
-#pragma unroll
-                    for (int e = 0; e < 8; ++e) acc = fmaf(wf[e], hrow[k + e], acc);
+    }
+    if (greedy) {
+        const AM top = block_am(am, sm_am);   // candidate 0: the argmax of the tensor-core logits
+        if (t == 0) { s_tok[0] = top.i; s_e[0] = 1.f; }
+        if (topk > 1) {
+            // the topk groups of largest maximum, one block argmax per round
+            for (int r = 0; r < topk; ++r) {
+                AM loc{-INFINITY, 0x7fffffff};
+                for (int j = j0; j < j1; ++j) {
+                    bool taken = false;
+                    for (int rr = 0; rr < r; ++rr) taken |= s_grp[rr] == j;
+                    const float4 p = __ldcg(pp + j);
+                    if (!taken) loc = am_combine(loc, AM{p.z, j});
                 }
+                const AM g = block_am(loc, sm_am);
+                if (t == 0) s_grp[r] = g.v == -INFINITY ? -1 : g.i;
+                __syncthreads();
             }
-            acc = warp_sum(acc);
-            if (lane == 0) s_z[id - id0] = acc;
+            __syncthreads();
+            for (int r = 0; r < topk; ++r)
+                if (s_grp[r] >= 0) pk_group_logits(a, hrow, s_grp[r], s_z + r * TC_LM_GROUP);
+                else if (t < TC_LM_GROUP) s_z[r * TC_LM_GROUP + t] = -INFINITY;
+            __syncthreads();
+            // rank: candidates 1.. are the largest recomputed logits other than candidate 0
+            for (int c = 1; c < topk; ++c) {
+                AM loc{-INFINITY, 0x7fffffff};
+                if (t < topk * TC_LM_GROUP) {
+                    const int r = t / TC_LM_GROUP, l = t - r * TC_LM_GROUP;
+                    const int id = s_grp[r] < 0 ? -1 : s_grp[r] * TC_LM_GROUP + l;
+                    bool taken = id < 0;
+                    for (int cc = 0; cc < c; ++cc) taken |= s_tok[cc] == id;
+                    if (!taken) loc = AM{s_z[t], id};
+                }
+                const AM best = block_am(loc, sm_am);
+                if (t == 0) { s_tok[c] = best.i == 0x7fffffff ? s_tok[0] : best.i; s_e[c] = 1.f; }
+                __syncthreads();
+            }
         }
         __syncthreads();
-        if (warp == 0) {
-            const int id = id0 + lane;
-            const float e = id < D.V ? __expf(s_z[lane] * invT - M) : 0.f;
-            const float cum = s_before + warp_incl_scan(e);
-            const unsigned hit = __ballot_sync(0xffffffffu, e > 0.f && target < cum);
-            const unsigned pos = __ballot_sync(0xffffffffu, e > 0.f);
-            const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
-            if (lane == l) {
-                s_tok = id;
-                s_e = e;
+    } else {
+        // each draw: its group from the partials, then its id inside the recomputed group
+        float tot;
+        const float ex = block_excl_scan(w, sh, &tot);
+        for (int c = 0; c < topk; ++c) {
+            const float target = a.u_draft[((size_t)b * a.K + a.step) * topk + c] * S;
+            if (t == 0) { si[0] = 0x7fffffff; si[1] = -1; }
+            __syncthreads();
+            if (w > 0.f && target < ex + w) atomicMin(&si[0], t);
+            if (w > 0.f) atomicMax(&si[1], t);
+            __syncthreads();
+            const int ct = si[0] != 0x7fffffff ? si[0] : (si[1] >= 0 ? si[1] : 0);
+            if (t == ct) {   // this thread's run holds the point: find its group
+                float cum = ex;
+                int grp = -1, lastg = -1;
+                float lastb = ex;
+                for (int j = j0; j < j1; ++j) {
+                    const float4 p = __ldcg(pp + j);
+                    const float wj = p.x != -INFINITY ? p.y * __expf(p.x - M) : 0.f;
+                    if (wj > 0.f) { lastg = j; lastb = cum; }
+                    if (wj > 0.f && target < cum + wj) { grp = j; break; }
+                    cum += wj;
+                }
+                s_grp[c] = grp >= 0 ? grp : (lastg >= 0 ? lastg : j0);
+                s_before = grp >= 0 ? cum : lastb;
             }
+            __syncthreads();
+            pk_group_logits(a, hrow, s_grp[c], s_z);
+            __syncthreads();
+            if (warp == 0) {
+                const int id = s_grp[c] * TC_LM_GROUP + lane;
+                const float e = id < D.V ? __expf(s_z[lane] * invT - M) : 0.f;
+                const float cum = s_before + warp_incl_scan(e);
+                const unsigned hit = __ballot_sync(0xffffffffu, e > 0.f && target < cum);
+                const unsigned pos = __ballot_sync(0xffffffffu, e > 0.f);
+                const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+                if (lane == l) { s_tok[c] = id; s_e[c] = e; }
+            }
+            __syncthreads();
         }
-        __syncthreads();
-        token = s_tok;
-        qx = s_e / S;
     }
-    if (t == 0) {
-        a.tokens[(size_t)b * a.K + a.step] = token;
-        if (a.qx) a.qx[(size_t)b * a.K + a.step] = qx;
-        if (a.stats) {
-            a.stats[((size_t)b * a.K + a.step) * 2 + 0] = M;
-            a.stats[((size_t)b * a.K + a.step) * 2 + 1] = logf(S);
-        }
+    const size_t o = (size_t)b * a.K + a.step;
+    if (t < topk) {
+        a.tokens[o * topk + t] = s_tok[t];
+        if (a.qx) a.qx[o * topk + t] = greedy ? 1.f : s_e[t] / S;
     }
+    if (t == 0 && a.stats) {
+        a.stats[o * 2 + 0] = M;
+        a.stats[o * 2 + 1] = logf(S);
+    }
+    const int token = s_tok[0];
     if (a.step + 1 < a.K) {
-        // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[token]
+        // next chain row: context slot <- x_L (Sec. 3.4), residual <- E[candidate 0]
         const int src = a.src_is_ext ? b * a.max_new + a.nnew[b] - 1 : b;
         const float *xl = a.x_in + (size_t)src * D.d;
         const uint16_t *er = a.embed + (size_t)token * D.d;

@@ -108,9 +108,14 @@ cudaError_t launch_qkv_post(const QkvPostArgs &a, cudaStream_t s);
 // argmax (lowest id).  Writes the token, q(token), (max, log-sum-exp) and, when
 // a next chain step follows, the next chain row (context slot = x_L, residual =
 // E[token]).  Row b belongs to sequence b / rows_per_valid (0 or 1: itself).
+// topk > 1 (tree drafting): k candidates per row, [B][K][k] in tokens and qx;
+// sampled: k independent inverse-CDF draws at u_draft[b][step][j]; greedy: the
+// k highest logits in descending order (ties to the lowest id).  Candidate 0
+// continues the chain.
 struct LmPickArgs {
     Dims dim;
     int B, K, step, max_new, src_is_ext, rows_per_valid;
+    int topk;                  // candidates per row (0 or 1: one)
     const int *valid, *nnew;
     const float4 *part;        // [B][nsub] TC_LM partials
     int nsub;

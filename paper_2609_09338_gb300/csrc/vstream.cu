@@ -1,10 +1,12 @@
 // Streamed speculative-sampling verification (Sec. 3.1) for 16-byte-aligned
-// logits: persistent blocks (8 consumer warps + 1 producer warp, two per SM)
+// logits: persistent blocks (8 consumer warps + 1 producer warp, three per SM)
 // pull 4 KB chunks of the target row (and of the draft row, for rows i < K)
-// through a 12-slot shared-memory ring with 1-D bulk copies (TMA).  With more
-// slots than consumer warps, copies stay in flight while a warp works on its
-// tile; the fence and atomic that publish a result happen after the slot is
-// freed, once per run of tiles.
+// through an 8-slot shared-memory ring with 1-D bulk copies (TMA): the copies
+// of the other warps' tiles stay in flight while a warp works on its own, 24
+// slots per SM in all (three blocks fit the SM's registers and shared memory;
+// two blocks of 12 slots kept fewer warps resident and were slower).  The
+// fence and atomic that publish a result happen after the slot is freed, once
+// per run of tiles.
 //
 // vs_stats:  a tile is (sequence b, row i, chunk c).  The owning warp reduces
 //   it to (max, sum exp) of logits/T for p and q (argmax in greedy mode) and
@@ -32,11 +34,11 @@
 namespace osp {
 
 #ifndef OSP_VS_BPS
-#define OSP_VS_BPS 2   // resident blocks per SM (grid = OSP_VS_BPS x SMs at most)
+#define OSP_VS_BPS 3   // resident blocks per SM (grid = OSP_VS_BPS x SMs at most)
 #endif
 
 #ifndef OSP_VS_NST
-#define OSP_VS_NST 12  // ring slots per block
+#define OSP_VS_NST 8   // ring slots per block: 3 x 8 x 8 KB of the SM's shared memory
 #endif
 #ifndef OSP_VS_EARLY
 #define OSP_VS_EARLY 0   // 1: a consumer copies both rows of its tile to registers and frees the slot first

@@ -45,6 +45,22 @@ class DraftSession:
                              out["draft_qx"], out["draft_stats"], out["draft_logits"], self.workspace,
                              self.status, stream)
 
+    def tree_buffers(self, topk: int, with_logits: bool = False) -> dict:
+        B, K, dev = self.B, self.K, self.device
+        return {
+            "cand": torch.full((B, K, topk), -7, dtype=torch.int32, device=dev),
+            "cand_qx": torch.zeros((B, K, topk), dtype=torch.float32, device=dev),
+            "draft_stats": torch.zeros((B, K, 2), dtype=torch.float32, device=dev),
+            "draft_logits": torch.zeros((B, K, self.shape.vocab), dtype=torch.float32, device=dev)
+            if with_logits else None,
+        }
+
+    def draft_tree(self, n_new, tokens, feats, temperature: float, u_draft, out: dict, stream=None):
+        """The draft call with topk candidates per chain step (out from tree_buffers)."""
+        ob.osprey_draft_step_topk(self.ctx, self.kv, n_new, tokens, feats, temperature, u_draft, out["cand"],
+                                  out["cand_qx"], out["draft_stats"], out["draft_logits"], self.workspace,
+                                  self.status, stream)
+
     def draft_hidden(self, n_new, tokens, feats, temperature: float, u_draft, out: dict, hidden, stream=None):
         """The draft call without logits, keeping each draft token's state in hidden [B, K, d]."""
         ob.osprey_draft_step_hidden(self.ctx, self.kv, n_new, tokens, feats, temperature, u_draft,
@@ -86,6 +102,21 @@ class VerifyBuffers:
     def run(self, target, draft, tokens, temperature, u_accept, u_sample, stream=None):
         ob.osprey_verify(target, draft, tokens, temperature, u_accept, u_sample, self.out_tokens,
                          self.n_accepted, self.flags, self.probs, self.workspace, self.status, stream)
+
+
+class TreeVerifyBuffers:
+    """Outputs of osprey_verify_tree for B sequences of depth K (no workspace)."""
+
+    def __init__(self, B: int, K: int, device: str = "cuda"):
+        self.out_tokens = torch.zeros((B, K + 1), dtype=torch.int32, device=device)
+        self.n_accepted = torch.zeros(B, dtype=torch.int32, device=device)
+        self.branch = torch.zeros(B, dtype=torch.int32, device=device)
+        self.flags = torch.zeros((B, K + 1), dtype=torch.uint8, device=device)
+        self.status = torch.zeros(1, dtype=torch.int32, device=device)
+
+    def run(self, target, draft, cand, temperature, u_accept, u_sample, stream=None):
+        ob.osprey_verify_tree(target, draft, cand, temperature, u_accept, u_sample, self.out_tokens,
+                              self.n_accepted, self.branch, self.flags, self.status, stream)
 
 
 class VerifyHiddenBuffers(VerifyBuffers):

@@ -179,3 +179,42 @@ def make_verify_inputs(V: int, batch: int, K: int, temperature: float, sigma_p: 
         "u_accept": rng.random((batch, K), dtype=np.float32),
         "u_sample": rng.random((batch, K + 1), dtype=np.float32),
     }
+
+
+def make_tree_inputs(V: int, batch: int, K: int, k: int, temperature: float, sigma_p: float, seed: int) -> dict:
+    """Draft and target logits of a branching-chain draft tree, its candidates
+    and the uniforms.
+
+    Draft row i of a sequence: the Zipf-shaped base + N(0, 1).  Candidates:
+    k independent draws from softmax(row / T) by the Gumbel-max trick (the k
+    highest logits when greedy).  Target rows (row 0 the root, row 1 + i*k + j
+    the node (i, j)): the root is draft row 0 + N(0, sigma^2); a chain node
+    (i, 0) with i < K - 1 is draft row i + 1 + N(0, sigma^2) (the target after
+    the chain token the drafter continued from); the other nodes draw their
+    own base-shaped rows."""
+    rng = np.random.default_rng(seed)
+    base = _zipf_base(np.random.default_rng(seed + 7), V)
+    zq = np.empty((batch, K, V), np.float32)
+    zp = np.empty((batch, 1 + K * k, V), np.float32)
+    cand = np.empty((batch, K, k), np.int32)
+    for b in range(batch):
+        for i in range(K):
+            zq[b, i] = base + rng.standard_normal(V, dtype=np.float32)
+            if temperature > 0:
+                for j in range(k):
+                    g = -np.log(-np.log(rng.random(V) + 1e-300))
+                    cand[b, i, j] = int(np.argmax(zq[b, i].astype(np.float64) / temperature + g))
+            else:
+                order = np.lexsort((np.arange(V), -zq[b, i]))
+                cand[b, i] = order[:k]
+        zp[b, 0] = zq[b, 0] + np.float32(sigma_p) * rng.standard_normal(V, dtype=np.float32)
+        for i in range(K):
+            for j in range(k):
+                r = 1 + i * k + j
+                if j == 0 and i < K - 1:
+                    zp[b, r] = zq[b, i + 1] + np.float32(sigma_p) * rng.standard_normal(V, dtype=np.float32)
+                else:
+                    zp[b, r] = base + rng.standard_normal(V, dtype=np.float32)
+    return {"draft_logits": zq, "target_logits": zp, "cand": cand,
+            "u_accept": rng.random((batch, K, k), dtype=np.float32),
+            "u_sample": rng.random((batch, K + 1), dtype=np.float32)}
