@@ -74,7 +74,7 @@ def parse():
 # measured after the headline workload, each with its own dominant kernel
 EXTRA_WORKLOADS = ["qwen3-8b-d1024-v151936-b1-k7", "qwen3-8b-d1024-v151936-b32-k7",
                    "llama70b-d2048-v128256-b16-k7", "osprey-d2560-v151936-b1-k7-ext3",
-                   "dflash-d4096-l4-v151936-b1-blk16"]
+                   "dflash-d4096-l4-v151936-b1-blk16", "qwen3-8b-d1024-v151936-b8-k5-topk4"]
 
 
 def make_inputs(wl, rank=0, weights_path=None):
@@ -91,7 +91,12 @@ def make_inputs(wl, rank=0, weights_path=None):
             checkpoint.save_weights(weights_path, sh, w)
     kv = syn.make_kv_prefix(sh, ctx, wl.extra.get("block", wl.n_new + wl.K), seed + 1)
     di = syn.make_draft_inputs(sh, wl.batch, wl.n_new, wl.K, seed + 2)
-    vi = syn.make_verify_inputs(sh.vocab, wl.batch, wl.K, wl.temperature, wl.sigma_p, seed + 3)
+    topk = wl.extra.get("topk", 1)
+    if topk > 1:
+        vi = syn.make_tree_inputs(sh.vocab, wl.batch, wl.K, topk, wl.temperature, wl.sigma_p, seed + 3)
+        di["u_draft"] = np.random.default_rng(seed + 4).random((wl.batch, wl.K, topk), dtype=np.float32)
+    else:
+        vi = syn.make_verify_inputs(sh.vocab, wl.batch, wl.K, wl.temperature, wl.sigma_p, seed + 3)
     return ctx, w, kv, di, vi
 
 
@@ -120,6 +125,8 @@ def algorithmic_bytes(wl, ctx):
     kv = sum(kv_row * (int(c) + wl.n_new + k) for c in ctx for k in range(K))
     draft = K * w_step + 2 * sh.d_model * sh.feat_dim + kv + B * wl.n_new * sh.feat_dim * 2
     s = 4 if wl.logits_dtype == "f32" else 2
+    # chain: every target and draft row once; tree: the rows of one root-to-leaf path
+    # (K + 1 target rows and K draft rows), what a walk that accepts the chain reads
     verify = B * (K + 1) * sh.vocab * s + B * K * sh.vocab * s
     lm_launch = sh.vocab * sh.d_model * 2 * 1 + 2 * sh.d_model
     return {"draft": draft, "verify": verify, "lm_head_launch": lm_launch, "attn_call": kv,
@@ -527,9 +534,16 @@ def measure(wl, args, rank, world, local, full):
     else:
         v_in = {"target": ob.to_device_bf16(syn.bf16_bits(vi["target_logits"])),
                 "draft": ob.to_device_bf16(syn.bf16_bits(vi["draft_logits"]))}
-    v_in.update({"tokens": T_(vi["draft_tokens"]), "u_accept": T_(vi["u_accept"]), "u_sample": T_(vi["u_sample"])})
-    out = sess.draft_buffers()
-    vb = VerifyBuffers(B, K, sh.vocab)
+    v_in.update({"tokens": T_(vi["cand"] if "cand" in vi else vi["draft_tokens"]), "u_accept": T_(vi["u_accept"]),
+                 "u_sample": T_(vi["u_sample"])})
+    topk = wl.extra.get("topk", 1)
+    if topk > 1:
+        from paper_2609_09338_gb300.session import TreeVerifyBuffers
+        out = sess.tree_buffers(topk)
+        vb = TreeVerifyBuffers(B, K)
+    else:
+        out = sess.draft_buffers()
+        vb = VerifyBuffers(B, K, sh.vocab)
     n_probe = nb["attn_launches"] if dom == "attention" else nb["lm_launches"]
     ob.osprey_probe_select(sess.ctx, ob.PROBE_ATTENTION if dom == "attention" else ob.PROBE_LM_HEAD)
     ob.osprey_probe_enable(sess.ctx, n_probe)
@@ -544,6 +558,8 @@ def measure(wl, args, rank, world, local, full):
         sess.kv.seq_len.copy_(seq0)
         if blk:
             sess.propose(d_in["anchors"], 0, d_in["feats1"], T, d_in["u_draft"], out)
+        elif topk > 1:
+            sess.draft_tree(d_in["n_new"], d_in["tokens"], d_in["feats"], T, d_in["u_draft"], out)
         else:
             sess.draft(d_in["n_new"], d_in["tokens"], d_in["feats"], T, d_in["u_draft"], out)
         vb.run(v_in["target"], v_in["draft"] if T > 0 else None, v_in["tokens"], T, v_in["u_accept"],

@@ -472,7 +472,7 @@ __global__ void __launch_bounds__(256) qkv_post_kernel(const QkvPostArgs a) {
 }
 
 // ---------------------------------------------------------------- LM-head pick
-constexpr int PK_THREADS = 256;
+constexpr int PK_THREADS = 1024;   // each thread walks about V / 32 / 1024 partials
 
 constexpr int PK_MAXK = 8;   // candidates per row at most
 

@@ -120,6 +120,11 @@ WORKLOADS = {
     "dflash-d4096-l4-v151936-b1-blk16": Workload("dflash-d4096-l4-v151936-b1-blk16", DFLASH_DRAFTER,
                                                  batch=1, K=15, ctx_lo=2048, ctx_hi=2048, temperature=1.0,
                                                  sigma_p=0.7, seed=1006, extra={"block": 16}),
+    # tree drafting: K = 5 chain steps (the paper's serving steps) with topk = 4
+    # candidates each, batch 8, verified as a branching chain
+    "qwen3-8b-d1024-v151936-b8-k5-topk4": Workload("qwen3-8b-d1024-v151936-b8-k5-topk4", QWEN3_8B_DRAFTER,
+                                                   batch=8, K=5, ctx_lo=1024, ctx_hi=4096, temperature=1.0,
+                                                   sigma_p=0.7, seed=1007, extra={"topk": 4}),
     # large vocabulary, verify-heavy
     "large-vocab-d1024-v200064-b64-k8": Workload("large-vocab-d1024-v200064-b64-k8",
                                                  LARGE_VOCAB_DRAFTER, batch=64, K=8,
