@@ -468,7 +468,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
     auto tc_lm = [&](int rows, float *z, long long ldz, const LmPickArgs &pick_in) -> int {
         const int np = npad_of(rows);
         CUtensorMap xm;
-        if (!tc_encode_operand(&xm, ws.tc_xl, TC_PLANES, np, D.d))
+        if (!tc_encode_operand(&xm, ws.tc_xl, TC_LM_PLANES, np, D.d))
             return fail(OSPREY_ERR_INVALID_ARG, "lm head: tensor map encoding failed");
         TcArgs ta{};
         ta.epi = TC_LM;
@@ -476,7 +476,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         ta.npad = np;
         ta.K = D.d;
         ta.nout = D.V;
-        ta.planes = TC_PLANES;
+        ta.planes = TC_LM_PLANES;
         ta.y = z;
         ta.ldy = (int)ldz;
         ta.status = dev_status;
@@ -499,8 +499,9 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, "sampler launch");
     };
     auto planes = [&](const float *src, const uint16_t *gain, int d_, int rows, int ld, int col0, uint16_t *dst,
-                      int rows_per_seq, bool last_of_seq, const char *what) -> int {
+                      int rows_per_seq, bool last_of_seq, const char *what, int npl = TC_PLANES) -> int {
         PlaneArgs pl{};
+        pl.npl = npl;
         pl.src = src;
         pl.gain = gain;
         pl.eps = D.eps;
@@ -757,7 +758,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             const int rows = B * max_new;
             int rc;
             if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, rows, D.d, 0, ws.tc_xl, max_new, false,
-                             "lm operand")) != OSPREY_OK)
+                             "lm operand", TC_LM_PLANES)) != OSPREY_OK)
                 return rc;
             LmPickArgs pk{};
             pk.B = rows;
@@ -794,8 +795,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             // epilogue (logits stored only into draft_logits) -> one pick per row
             // (topk candidates per row when drafting a tree)
             int rc;
-            if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand")) !=
-                OSPREY_OK)
+            if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand",
+                             TC_LM_PLANES)) != OSPREY_OK)
                 return rc;
             LmPickArgs pk{};
             pk.B = B;
@@ -1058,14 +1059,12 @@ extern "C" int osprey_verify_tree(int B, int K, int topk, int V, int logits_dtyp
 // Workspace: the verify layout (counters, partials, decisions, chunk sums), then
 // for one group of up to TC_MAX_ROWS sequences the gathered kept states
 // [rows][d] float, their operand planes [TC_PLANES][npad][d] bf16, the
-// recomputed decision-row logits [rows][V] float and the split-K partials of
-// that GEMM (the draft step's LM-head split, so the rows come out the same).
+// recomputed decision-row logits [rows][V] float (the draft step's LM-head GEMM:
+// the same operand planes, unsplit, so the rows come out the same).
 struct HiddenWs {
     float *rows;
     uint16_t *planes;
     float *z;
-    float *part;
-    long long part_cap;
     int group, npad;
 };
 
@@ -1080,17 +1079,11 @@ static size_t verify_hidden_layout(const osprey_ctx *ctx, int B, int K, VerifyAr
     off = align256(off + 2ull * TC_PLANES * npad * D.d);
     const size_t o_z = off;
     off = align256(off + 4ull * group * D.V);
-    const int ns = tc_nsplit(D.V, D.d, ctx->sms);
-    const long long part = ns > 1 ? (long long)ns * group * D.V : 0;
-    const size_t o_t = off;
-    off = align256(off + 4ull * part);
     if (hw && base) {
         char *p = (char *)base;
         hw->rows = (float *)(p + o_r);
         hw->planes = (uint16_t *)(p + o_p);
         hw->z = (float *)(p + o_z);
-        hw->part = part ? (float *)(p + o_t) : nullptr;
-        hw->part_cap = part;
         hw->group = group;
         hw->npad = npad;
     }
@@ -1175,10 +1168,11 @@ extern "C" int osprey_verify_hidden(osprey_ctx *ctx, int B, int K, int logits_dt
         pl.dst = hw.planes;
         pl.max_new = 1;
         pl.rows_per_seq = 1;
+        pl.npl = TC_LM_PLANES;
         if ((e = launch_planes(pl, s)) != cudaSuccess) return cuda_fail(e, "decision-row operand launch");
         // 3. their draft logits on the tensor cores (the draft step's LM head GEMM)
         CUtensorMap xm;
-        if (!tc_encode_operand(&xm, hw.planes, TC_PLANES, npad, D.d))
+        if (!tc_encode_operand(&xm, hw.planes, TC_LM_PLANES, npad, D.d))
             return fail(OSPREY_ERR_INVALID_ARG, "decision-row tensor map encoding failed");
         TcArgs ta{};
         ta.epi = TC_STORE;
@@ -1186,13 +1180,11 @@ extern "C" int osprey_verify_hidden(osprey_ctx *ctx, int B, int K, int logits_dt
         ta.npad = npad;
         ta.K = D.d;
         ta.nout = V;
-        ta.planes = TC_PLANES;
+        ta.planes = TC_LM_PLANES;
         ta.y = hw.z;
         ta.x = hw.z;
         ta.ldy = V;
-        ta.status = dev_status;
-        ta.part = hw.part;
-        ta.part_cap = hw.part_cap;
+        ta.status = dev_status;   // unsplit, like the draft step's LM head: the same logits bit for bit
         if ((e = launch_tc(ta, ctx->tm_lm, xm, ctx->sms, s)) != cudaSuccess) return cuda_fail(e, "decision-row lm head");
         // 4. the emitted token of each sequence of the group
         if ((e = launch_verify_hidden_sample(a, b0, n, s)) != cudaSuccess) return cuda_fail(e, "verify sample launch");

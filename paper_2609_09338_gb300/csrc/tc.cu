@@ -425,13 +425,15 @@ __global__ void __launch_bounds__(256) planes_kernel(const PlaneArgs a) {
     }
     uint16_t *p0 = a.dst + (size_t)r * a.ld + a.col0;
     const size_t plane = (size_t)a.npad * a.ld;
+    const int npl = a.npl > 0 ? a.npl : TC_PLANES;
     for (int k = threadIdx.x; k < a.d; k += blockDim.x) {
         float v = act ? x[k] : 0.f;
         if (a.gain) v = v * inv * bf_to_f(a.gain[k]);
         uint16_t q[TC_PLANES];
         tc_split(v, q);
 #pragma unroll
-        for (int i = 0; i < TC_PLANES; ++i) p0[i * plane + k] = q[i];
+        for (int i = 0; i < TC_PLANES; ++i)
+            if (i < npl) p0[i * plane + k] = q[i];
     }
 }
 
@@ -550,7 +552,7 @@ __global__ void __launch_bounds__(PK_THREADS) lm_pick_kernel(const LmPickArgs a)
         for (int k = t; k < D.d; k += PK_THREADS) {
             float h = 0.f;
 #pragma unroll
-            for (int i = 0; i < TC_PLANES; ++i) h += bf_to_f(q[i * plane + k]);
+            for (int i = 0; i < TC_LM_PLANES; ++i) h += bf_to_f(q[i * plane + k]);
             hrow[k] = h;
         }
     }
@@ -764,11 +766,14 @@ static cudaError_t pdl_launch(void (*k)(P...), dim3 grid, dim3 block, size_t sme
 
 // k-ranges per output tile so that tiles x ranges fill the CTA slots (few
 // output tiles, long K: the layer projections); 1 for wide outputs.
+#ifndef OSP_TC_MIN_KB
+#define OSP_TC_MIN_KB 1   // k-blocks (of 64) per range at least: fewer, longer ranges write fewer partials
+#endif
 int tc_nsplit(int nout, int K, int sms) {
     const int tiles = (nout + 127) / 128, nkb = K / 64;
     int want = (OSP_TC_CTAS_PER_SM * sms + tiles - 1) / tiles;
     if (want < 1) want = 1;
-    if (want > nkb) want = nkb;
+    if (want > nkb / OSP_TC_MIN_KB) want = nkb / OSP_TC_MIN_KB > 1 ? nkb / OSP_TC_MIN_KB : 1;
     const int kbps = (nkb + want - 1) / want;
     return (nkb + kbps - 1) / kbps;
 }

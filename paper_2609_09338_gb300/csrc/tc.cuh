@@ -29,6 +29,11 @@ namespace osp {
 // id), and stores the logits only when y is given.
 enum TcEpi { TC_STORE = 0, TC_RESID = 1, TC_GLU = 2, TC_LM = 3 };
 constexpr int TC_LM_GROUP = 32;    // vocabulary ids per LM-head partial (one epilogue warp's lanes)
+// The LM head's operand rows enter as two bf16 planes (16 significant bits):
+// a logit's error from the dropped bits is a sum of d random terms of
+// 2^-17 |h_k| |W_jk|, about 5e-6 at d 1024, the float32 GEMV's own level; the
+// smaller stage lets three weight tiles per CTA be in flight instead of two.
+constexpr int TC_LM_PLANES = 2;
 
 constexpr int TC_MAX_ROWS = 80;    // activation rows per GEMM: three accumulators fit a CTA's 256 TMEM columns
 constexpr int TC_PLANES = 3;       // bf16 planes of a float32 operand
@@ -84,6 +89,7 @@ struct PlaneArgs {
     int max_new, last_of_seq;
     const int *valid;          // rows of invalid sequences are written as zeros (may be null)
     int rows_per_seq;
+    int npl;                   // planes written (0: TC_PLANES)
 };
 cudaError_t launch_planes(const PlaneArgs &a, cudaStream_t s);
 
