@@ -164,8 +164,11 @@ def test_draft_topk_candidates(name, B, T):
         np.testing.assert_array_equal(tr["draft_stats"], ch["draft_stats"])
     else:
         # one or two rows: the chain samples on the streamed LM head, topk on the
-        # tensor-core one; candidate 0 agrees wherever its draw is clear of a bin edge
-        np.testing.assert_allclose(tr["draft_logits"], ch["draft_logits"], atol=1e-4)
+        # tensor-core one; candidate 0 agrees wherever its draw is clear of a bin edge.
+        # The tensor-core head carries each final-norm activation in two bf16 planes
+        # (error at most 2^-18 relative per element), so the two heads' logits part by
+        # a few parts in 1e6 of their magnitude on top of the accumulation order.
+        np.testing.assert_allclose(tr["draft_logits"], ch["draft_logits"], atol=1e-4, rtol=1e-5)
         for b in range(B):
             for i in range(K):
                 own = od.sample(z[b, i], T, float(inp["u"][b, i, 0]))
