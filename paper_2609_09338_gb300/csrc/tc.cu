@@ -35,6 +35,9 @@ constexpr size_t TC_SMEM_CAP = (OSP_TC_CTAS_PER_SM == 1 ? 200 : 100) * 1024;
 #ifndef OSP_TC_SEGKB
 #define OSP_TC_SEGKB 8   // k-blocks (64 wide) per accumulation segment
 #endif
+#ifndef OSP_TC_LM_NA
+#define OSP_TC_LM_NA 2   // LM head: weight tiles per stage that share one operand stage
+#endif
 
 // ---------------------------------------------------------------- tcgen05 PTX
 __device__ __forceinline__ void tma_2d(void *dst, const CUtensorMap *m, int x, int y, uint64_t *bar) {
@@ -117,18 +120,20 @@ __device__ __forceinline__ void lm_combine(float &a1, int &i1, float &s1, float 
 }
 
 // ---------------------------------------------------------------- GEMM kernel
-template <int EPI>
+// NA weight tiles (NA x 128 output features) share each stage's operand
+// planes: one work item is NA adjacent tiles, accumulated side by side in TMEM.
+template <int EPI, int NA>
 __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
     tc_kernel(const __grid_constant__ CUtensorMap wa, const __grid_constant__ CUtensorMap xm, const TcArgs a, int nst) {
-    constexpr int NA = 1;
     extern __shared__ uint8_t raw[];
     uint8_t *sm = (uint8_t *)(((uintptr_t)raw + 1023) & ~(uintptr_t)1023);
     __shared__ __align__(8) uint64_t full[TC_MAXST], empty[TC_MAXST], accf[2], acce[2], fin;
     __shared__ uint32_t s_tmem;
     __shared__ int s_abort;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    // work item = (output tile of 128 features, k-range); items of a CTA are contiguous
-    const int n_items = (a.nout + 127) / 128 * a.nsplit;
+    // work item = (NA output tiles of 128 features, k-range); items of a CTA are contiguous
+    const int segkb = a.segkb;
+    const int n_items = (a.nout + 128 * NA - 1) / (128 * NA) * a.nsplit;
     const int i0 = (int)((long long)n_items * blockIdx.x / gridDim.x);
     const int i1 = (int)((long long)n_items * (blockIdx.x + 1) / gridDim.x);
     const int nloc = i1 - i0, nkb = a.K / 64, npad = a.npad;
@@ -142,7 +147,7 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
     // TMEM: two segment buffers and (when a tile has several segments) the
     // running float32 total of the tile
     const uint32_t acc_cols = NA * npad;
-    const int nseg_max = (min(nkb, a.kbps) + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+    const int nseg_max = (min(nkb, a.kbps) + segkb - 1) / segkb;
     uint32_t ncols = 32;
     while (ncols < (nseg_max > 1 ? 3 : 2) * acc_cols) ncols <<= 1;
 
@@ -176,7 +181,7 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
             long long g = 0;
             bool stop = false;
             for (int it = 0; it < nloc && !stop; ++it) {
-                const int y = (i0 + it) / a.nsplit * 128;
+                const int y = (i0 + it) / a.nsplit * 128 * NA;
                 int klo, khi;
                 krange(i0 + it, klo, khi);
                 for (int kb = klo; kb < khi; ++kb, ++g) {
@@ -190,7 +195,8 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     if (*(volatile int *)&s_abort) { stop = true; break; }
                     uint8_t *st = sm + (size_t)s * stage;
                     mbar_arrive_expect_tx(&full[s], stage);
-                    tma_2d(st, &wa, kb * 64, y, &full[s]);
+#pragma unroll
+                    for (int t = 0; t < NA; ++t) tma_2d(st + t * TC_ABYTES, &wa, kb * 64, y + 128 * t, &full[s]);
                     for (int p = 0; p < a.planes; ++p)
                         tma_2d(st + NA * TC_ABYTES + (size_t)p * npad * 128, &xm, kb * 64, p * npad, &full[s]);
                 }
@@ -208,7 +214,7 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
             for (int it = 0; it < nloc && !stop; ++it) {
                 int klo, khi;
                 krange(i0 + it, klo, khi);
-                const int nseg = (khi - klo + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+                const int nseg = (khi - klo + segkb - 1) / segkb;
                 for (int sg = 0; sg < nseg && !stop; ++sg, ++u) {
                     const int buf = (int)(u & 1);
                     if (u >= 2 && !mbar_wait(&acce[buf], (uint32_t)((u >> 1) - 1) & 1)) {
@@ -219,7 +225,7 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     }
                     tc_fence_after();
                     const uint32_t d0 = tmem + (uint32_t)buf * acc_cols;
-                    const int kb0 = klo + sg * OSP_TC_SEGKB, kb1 = min(khi, kb0 + OSP_TC_SEGKB);
+                    const int kb0 = klo + sg * segkb, kb1 = min(khi, kb0 + segkb);
                     for (int kb = kb0; kb < kb1; ++kb, ++g) {
                         const int s = (int)(g % nst);
                         if (!mbar_wait(&full[s], (uint32_t)(g / nst) & 1) || *(volatile int *)&s_abort) {
@@ -230,13 +236,15 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                         }
                         tc_fence_after();
                         const uint32_t st = smem_u32(sm + (size_t)s * stage);
-                        const uint64_t da = tc_desc(st);
 #pragma unroll
                         for (int kk = 0; kk < 4; ++kk) {
                             for (int p = 0; p < a.planes; ++p) {
                                 const uint64_t db = tc_desc(st + NA * TC_ABYTES + (uint32_t)p * npad * 128);
                                 const uint32_t acc = (kb != kb0) || kk || p;
-                                tc_mma(d0, da + 2 * kk, db + 2 * kk, idesc, acc);
+#pragma unroll
+                                for (int t = 0; t < NA; ++t)
+                                    tc_mma(d0 + (uint32_t)(t * npad), tc_desc(st + t * TC_ABYTES) + 2 * kk, db + 2 * kk,
+                                           idesc, acc);
                             }
                         }
                         tc_commit(&empty[s]);
@@ -256,12 +264,11 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
         long long u = 0;
         bool stop = false;
         for (int it = 0; it < nloc && !stop; ++it) {
-            const int col = (i0 + it) / a.nsplit * 128 + m, sp = (i0 + it) % a.nsplit;
-            const bool colok = col < a.nout;
+            const int col0 = (i0 + it) / a.nsplit * 128 * NA + m, sp = (i0 + it) % a.nsplit;
             const uint32_t tt = tmem + ((uint32_t)lg << 16) + 2u * acc_cols;
             int klo, khi;
             krange(i0 + it, klo, khi);
-            const int nseg = (khi - klo + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
+            const int nseg = (khi - klo + segkb - 1) / segkb;
             for (int sg = 0; sg < nseg; ++sg, ++u) {
                 const int buf = (int)(u & 1);
                 if (!mbar_wait(&accf[buf], (uint32_t)(u >> 1) & 1) || *(volatile int *)&s_abort) {
@@ -273,17 +280,21 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                 tc_fence_after();
                 const bool last = sg == nseg - 1;
                 const uint32_t t0 = tmem + ((uint32_t)lg << 16) + (uint32_t)buf * acc_cols;
-                for (int c0 = 0; c0 < npad; c0 += 16) {
+                for (int cc = 0; cc < NA * npad; cc += 16) {
+                    // accumulator columns [t npad, (t + 1) npad) hold tile t's rows
+                    const int tile = cc / npad, c0 = cc - tile * npad;
+                    const int col = col0 + 128 * tile;
+                    const bool colok = col < a.nout;
                     float v[16], tv[16];
-                    tc_ld16(t0 + (uint32_t)c0, v);
-                    if (sg > 0) tc_ld16(tt + (uint32_t)c0, tv);
+                    tc_ld16(t0 + (uint32_t)cc, v);
+                    if (sg > 0) tc_ld16(tt + (uint32_t)cc, tv);
                     tc_ld_wait();
                     if (sg > 0) {
 #pragma unroll
                         for (int j = 0; j < 16; ++j) v[j] += tv[j];
                     }
                     if (!last) {
-                        tc_st16(tt + (uint32_t)c0, v);
+                        tc_st16(tt + (uint32_t)cc, v);
                         continue;
                     }
                     if (EPI == TC_LM) {
@@ -292,7 +303,8 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                         // rows a lane carries (it keeps one half and receives the partner's
                         // share of it), so after four rounds lane l holds row l / 2 over 16
                         // lanes and one more exchange completes it over all 32
-                        const int sub = (int)(((long long)((i0 + it) / a.nsplit) * 128 + lg) / TC_LM_GROUP);
+                        const int sub = (int)(((long long)((i0 + it) / a.nsplit) * 128 * NA + 128 * tile + lg) /
+                                              TC_LM_GROUP);
                         float av[16], sv[16];
                         int ai[16];
 #pragma unroll
@@ -727,22 +739,26 @@ bool tc_encode_operand(CUtensorMap *m, const void *x, int planes, int npad, int 
     return encode2d(m, x, K, (uint64_t)planes * npad, npad);
 }
 
-static int tc_stages(int npad, int planes, bool pair) {
-    const size_t stage = (size_t)(pair ? 2 : 1) * TC_ABYTES + (size_t)planes * npad * 128;
+static int tc_stages(int npad, int planes, int na) {
+    const size_t stage = (size_t)na * TC_ABYTES + (size_t)planes * npad * 128;
     int n = (int)((TC_SMEM_CAP - 1024) / stage);
     return n > TC_MAXST ? TC_MAXST : n;
 }
-size_t tc_smem_bytes(int npad, int planes, bool pair) {
-    const size_t stage = (size_t)(pair ? 2 : 1) * TC_ABYTES + (size_t)planes * npad * 128;
-    return (size_t)tc_stages(npad, planes, pair) * stage + 1024;
+size_t tc_smem_bytes(int npad, int planes, int na) {
+    const size_t stage = (size_t)na * TC_ABYTES + (size_t)planes * npad * 128;
+    return (size_t)tc_stages(npad, planes, na) * stage + 1024;
 }
 
 cudaError_t tc_set_attributes() {
     const int bytes = (int)TC_SMEM_CAP;
-    cudaError_t e = cudaFuncSetAttribute(tc_kernel<TC_STORE>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_RESID>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_GLU>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
-    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_LM>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    cudaError_t e = cudaFuncSetAttribute(tc_kernel<TC_STORE, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(tc_kernel<TC_RESID, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess)
+        e = cudaFuncSetAttribute(tc_kernel<TC_GLU, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess) e = cudaFuncSetAttribute(tc_kernel<TC_LM, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
+    if (e == cudaSuccess && OSP_TC_LM_NA > 1)
+        e = cudaFuncSetAttribute(tc_kernel<TC_LM, OSP_TC_LM_NA>, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes);
     if (e == cudaSuccess) e = allow_smem(lm_pick_kernel);
     return e;
 }
@@ -781,25 +797,40 @@ int tc_nsplit(int nout, int K, int sms) {
 cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s) {
     TcArgs a = a_in;
     if (a.npad % 16 || a.npad < 16 || a.npad > TC_MAX_ROWS || a.K % 64 || a.R > a.npad) return cudaErrorInvalidValue;
-    const int nst = tc_stages(a.npad, a.planes, false);
-    if (nst < 2) return cudaErrorInvalidValue;
     const int nkb = a.K / 64;
     if (a.epi == TC_LM && (!a.lm_part || a.lm_nsub != (a.nout + TC_LM_GROUP - 1) / TC_LM_GROUP))
         return cudaErrorInvalidValue;
     a.nsplit = a.part && a.epi != TC_LM ? tc_nsplit(a.nout, a.K, sms) : 1;   // the LM epilogue needs whole sums
     if ((long long)a.nsplit * a.R * a.nout > a.part_cap) a.nsplit = 1;
     a.kbps = (nkb + a.nsplit - 1) / a.nsplit;
-    const int nseg = (a.kbps + OSP_TC_SEGKB - 1) / OSP_TC_SEGKB;
-    if ((nseg > 1 ? 3 : 2) * a.npad > 512 / OSP_TC_CTAS_PER_SM) return cudaErrorInvalidValue;   // TMEM columns
-    const int items = (a.nout + 127) / 128 * a.nsplit;
+    a.segkb = OSP_TC_SEGKB;
+    constexpr int tmem_cols = 512 / OSP_TC_CTAS_PER_SM;
+    // the LM head takes OSP_TC_LM_NA weight tiles per stage when two stages fit
+    // and the double-buffered accumulators fit TMEM in one segment (the LM head's
+    // reduction over d is short: one segment keeps its MMA chain at 4 d / 64 steps
+    // per plane)
+    int na = 1;
+    if (a.epi == TC_LM && OSP_TC_LM_NA > 1 && tc_stages(a.npad, a.planes, OSP_TC_LM_NA) >= 2 &&
+        2 * OSP_TC_LM_NA * a.npad <= tmem_cols && a.kbps <= 32) {
+        na = OSP_TC_LM_NA;
+        a.segkb = a.kbps;
+    }
+    const int nst = tc_stages(a.npad, a.planes, na);
+    if (nst < 2) return cudaErrorInvalidValue;
+    const int nseg = (a.kbps + a.segkb - 1) / a.segkb;
+    if ((nseg > 1 ? 3 : 2) * na * a.npad > tmem_cols) return cudaErrorInvalidValue;   // TMEM columns
+    const int items = (a.nout + 128 * na - 1) / (128 * na) * a.nsplit;
     const int grid = items < OSP_TC_CTAS_PER_SM * sms ? items : OSP_TC_CTAS_PER_SM * sms;
-    const size_t smem = tc_smem_bytes(a.npad, a.planes, false);
+    const size_t smem = tc_smem_bytes(a.npad, a.planes, na);
     cudaError_t e;
     switch (a.epi) {
-    case TC_STORE: e = pdl_launch(tc_kernel<TC_STORE>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
-    case TC_RESID: e = pdl_launch(tc_kernel<TC_RESID>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
-    case TC_GLU: e = pdl_launch(tc_kernel<TC_GLU>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
-    default: e = pdl_launch(tc_kernel<TC_LM>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    case TC_STORE: e = pdl_launch(tc_kernel<TC_STORE, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    case TC_RESID: e = pdl_launch(tc_kernel<TC_RESID, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    case TC_GLU: e = pdl_launch(tc_kernel<TC_GLU, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    default:
+        e = na > 1 ? pdl_launch(tc_kernel<TC_LM, OSP_TC_LM_NA>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst)
+                   : pdl_launch(tc_kernel<TC_LM, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
+        break;
     }
     if (e != cudaSuccess || a.nsplit == 1) return e;
     const unsigned rblocks = (unsigned)(((long long)a.R * a.nout + 255) / 256);

@@ -4,7 +4,8 @@
 //
 // Weights are the M = 128 operand, streamed tile by tile with 2-D TMA (128-byte
 // swizzle); the R activation rows are the N operand (padded to a multiple of
-// 16).  Activations are float32 between kernels; for the tensor cores each is
+// 16).  The LM head multiplies two weight tiles against each stage's operand
+// planes (twice the weight bytes in flight per byte of operand reloaded).  Activations are float32 between kernels; for the tensor cores each is
 // split into three bf16 planes, q0 = bf16(x), q1 = bf16(x - q0), q2 =
 // bf16(x - q0 - q1), and every k-step issues one MMA per plane into the same
 // float32 accumulator, so the product keeps the 24 mantissa bits of x (bf16
@@ -57,6 +58,7 @@ struct TcArgs {
     float *part;
     long long part_cap;   // floats available in part
     int nsplit, kbps;     // set by launch_tc
+    int segkb;            // k-blocks per accumulation segment, set by launch_tc
 };
 
 // Host side.  Tensor maps: weights [rows][K] bf16 with a 64 x 128 box, operand
@@ -66,7 +68,7 @@ bool tc_encode_weight(CUtensorMap *m, const void *w, int rows, int K);
 bool tc_encode_operand(CUtensorMap *m, const void *x, int planes, int npad, int K);
 // a single bf16 plane of `rows` rows read in place (rows past `rows` read as zero)
 bool tc_encode_rows(CUtensorMap *m, const void *x, int rows, int npad, int K);
-size_t tc_smem_bytes(int npad, int planes, bool pair);
+size_t tc_smem_bytes(int npad, int planes, int na);
 cudaError_t tc_set_attributes();
 // SwiGLU runs as two passes: the gate projection (TC_STORE into a float32
 // buffer), then the up projection whose epilogue (TC_GLU) forms silu(gate) * up.
