@@ -270,7 +270,6 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_xh = take(tcw ? 2ull * TC_PLANES * np * D.F : 0), o_xl = take(tcw ? 2ull * TC_PLANES * np * D.d : 0);
     const long long lm_nsub = (D.V + TC_LM_GROUP - 1) / TC_LM_GROUP;
     size_t o_rp = take(tcw ? 16ull * R_lm * lm_nsub : 0);
-    size_t o_tg = take(tcw ? 4ull * np * D.F : 0);
     // split-K partials: the largest nsplit x rows x outputs of the call's projections
     long long part = 0;
     if (tcw) {
@@ -282,7 +281,8 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         need(D.d, D.feat);
         need((D.Hq + 2 * D.Hkv) * D.hd, 2 * D.d);
         need(D.d, D.Hq * D.hd);
-        need(D.F, D.d);
+        // gate/up: one GEMM whose partials always go through the buffer
+        part = std::max(part, (long long)std::max(tc_nsplit(2 * D.F, D.d, ctx->sms), 1) * rows * 2 * D.F);
         need(D.d, D.F);
         need(D.V, D.d);
     }
@@ -316,7 +316,6 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->rs_ticket = (int *)(p + o_rt);
         ws->counters = (int *)(p + o_at);
         ws->n_counters = (int)n_counters;
-        ws->tc_g = (float *)(p + o_tg);
         ws->tc_part = (float *)(p + o_tp);
         ws->tc_part_cap = part;
         ws->n_splits_max = ns;
@@ -440,7 +439,7 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
     auto npad_of = [](int rows) { return (rows + 15) / 16 * 16; };
     auto tc_gemm = [&](int epi, int rows, int K_, int nout, int planes, const CUtensorMap &wa,
                        const void *xbuf, bool in_place_rows, float *y, int ldy, uint16_t *h,
-                       const char *what) -> int {
+                       const char *what, const CUtensorMap *wb = nullptr) -> int {
         const int np = npad_of(rows);
         CUtensorMap xm;
         const bool ok = in_place_rows ? tc_encode_rows(&xm, xbuf, rows, np, K_) : tc_encode_operand(&xm, xbuf, planes, np, K_);
@@ -459,7 +458,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         ta.status = dev_status;
         ta.part = ws.tc_part;
         ta.part_cap = ws.tc_part_cap;
-        const cudaError_t e2 = launch_tc(ta, wa, xm, ctx->sms, s);
+        ta.nout_a = wb ? nout / 2 : nout;
+        const cudaError_t e2 = launch_tc2(ta, wa, wb ? *wb : wa, xm, ctx->sms, s);
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
     };
     // the LM head of `rows` operand rows in ws.tc_xl on the tensor cores, with the
@@ -499,9 +499,12 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, "sampler launch");
     };
     auto planes = [&](const float *src, const uint16_t *gain, int d_, int rows, int ld, int col0, uint16_t *dst,
-                      int rows_per_seq, bool last_of_seq, const char *what, int npl = TC_PLANES) -> int {
+                      int rows_per_seq, bool last_of_seq, const char *what, int npl = TC_PLANES,
+                      const float *src2 = nullptr, int col2 = 0) -> int {
         PlaneArgs pl{};
         pl.npl = npl;
+        pl.src2 = src2;
+        pl.col2 = col2;
         pl.src = src;
         pl.gain = gain;
         pl.eps = D.eps;
@@ -597,10 +600,10 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             uint16_t *vp = (uint16_t *)kv->v_pages + l * layer_pages;
             const int nqkv = (D.Hq + 2 * D.Hkv) * D.hd;
             int rc;
-            // [s; RMSNorm(x)] -> QKV (Eq. 2-3) -> RoPE and the paged K/V rows
-            if ((rc = planes(sb, nullptr, D.d, R, 2 * D.d, 0, ws.tc_xq, rows_per_seq, false, "qkv operand")) != OSPREY_OK ||
-                (rc = planes(x, (const uint16_t *)W.attn_norm[l], D.d, R, 2 * D.d, D.d, ws.tc_xq, rows_per_seq, false,
-                             "qkv operand")) != OSPREY_OK ||
+            // [s; RMSNorm(x)] -> QKV (Eq. 2-3) -> RoPE and the paged K/V rows; the s half
+            // of the operand is the same for every layer of the step
+            if ((rc = planes(x, (const uint16_t *)W.attn_norm[l], D.d, R, 2 * D.d, D.d, ws.tc_xq, rows_per_seq, false,
+                             "qkv operand", TC_PLANES, l == 0 ? sb : nullptr, 0)) != OSPREY_OK ||
                 (rc = tc_gemm(TC_STORE, R, 2 * D.d, nqkv, TC_PLANES, ctx->tm_qkv[l], ws.tc_xq, false, ws.tc_yq, nqkv,
                               nullptr, "qkv launch")) != OSPREY_OK)
                 return rc;
@@ -643,10 +646,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
                               "o-proj launch")) != OSPREY_OK ||
                 (rc = planes(x, (const uint16_t *)W.ffn_norm[l], D.d, R, D.d, 0, ws.tc_xg, rows_per_seq, false,
                              "gate/up operand")) != OSPREY_OK ||
-                (rc = tc_gemm(TC_STORE, R, D.d, D.F, TC_PLANES, ctx->tm_gate[l], ws.tc_xg, false, ws.tc_g, D.F, nullptr,
-                              "gate launch")) != OSPREY_OK ||
-                (rc = tc_gemm(TC_GLU, R, D.d, D.F, TC_PLANES, ctx->tm_up[l], ws.tc_xg, false, ws.tc_g, D.F, ws.tc_xh,
-                              "up launch")) != OSPREY_OK ||
+                (rc = tc_gemm(TC_GLU, R, D.d, 2 * D.F, TC_PLANES, ctx->tm_gate[l], ws.tc_xg, false, nullptr, 0,
+                              ws.tc_xh, "gate/up launch", &ctx->tm_up[l])) != OSPREY_OK ||
                 (rc = tc_gemm(TC_RESID, R, D.F, D.d, TC_PLANES, ctx->tm_down[l], ws.tc_xh, false, x, D.d, nullptr,
                               "down launch")) != OSPREY_OK)
                 return rc;

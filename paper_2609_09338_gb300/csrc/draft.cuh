@@ -36,7 +36,6 @@ struct DraftWs {
     float *tc_yq;                          // [np][(Hq+2Hkv)hd] QKV output before RoPE
     uint16_t *tc_xo;                       // [P][np][Hq*hd] attention output
     uint16_t *tc_xg;                       // [P][np][d]     RMSNorm(x) for gate/up
-    float *tc_g;                           // [np][F]        gate projection (float32)
     float *tc_part;                        // split-K partials of the projections
     long long tc_part_cap;
     uint16_t *tc_xh;                       // [P][np][F]     SwiGLU hidden (down operand)

@@ -122,9 +122,12 @@ __device__ __forceinline__ void lm_combine(float &a1, int &i1, float &s1, float 
 // ---------------------------------------------------------------- GEMM kernel
 // NA weight tiles (NA x 128 output features) share each stage's operand
 // planes: one work item is NA adjacent tiles, accumulated side by side in TMEM.
+// Output features [0, nout_a) come from the weights of map wa, the rest from
+// wb (row f - nout_a): the SwiGLU gate and up projections run as one GEMM.
 template <int EPI, int NA>
 __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
-    tc_kernel(const __grid_constant__ CUtensorMap wa, const __grid_constant__ CUtensorMap xm, const TcArgs a, int nst) {
+    tc_kernel(const __grid_constant__ CUtensorMap wa, const __grid_constant__ CUtensorMap wb,
+              const __grid_constant__ CUtensorMap xm, const TcArgs a, int nst) {
     extern __shared__ uint8_t raw[];
     uint8_t *sm = (uint8_t *)(((uintptr_t)raw + 1023) & ~(uintptr_t)1023);
     __shared__ __align__(8) uint64_t full[TC_MAXST], empty[TC_MAXST], accf[2], acce[2], fin;
@@ -196,7 +199,11 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     uint8_t *st = sm + (size_t)s * stage;
                     mbar_arrive_expect_tx(&full[s], stage);
 #pragma unroll
-                    for (int t = 0; t < NA; ++t) tma_2d(st + t * TC_ABYTES, &wa, kb * 64, y + 128 * t, &full[s]);
+                    for (int t = 0; t < NA; ++t) {
+                        const int f = y + 128 * t;   // tiles never straddle nout_a (a multiple of 128)
+                        tma_2d(st + t * TC_ABYTES, f < a.nout_a ? &wa : &wb, kb * 64, f < a.nout_a ? f : f - a.nout_a,
+                               &full[s]);
+                    }
                     for (int p = 0; p < a.planes; ++p)
                         tma_2d(st + NA * TC_ABYTES + (size_t)p * npad * 128, &xm, kb * 64, p * npad, &full[s]);
                 }
@@ -347,19 +354,12 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     for (int j = 0; j < 16; ++j) {
                         const int n = c0 + j;
                         if (n >= a.R || !colok) continue;
-                        if (a.nsplit > 1) {   // partial of this k-range; tc_reduce applies the epilogue
+                        if (a.nsplit > 1 || EPI == TC_GLU) {   // partial of this k-range; tc_reduce applies the epilogue
                             a.part[((size_t)sp * a.R + n) * a.nout + col] = v[j];
                         } else if (EPI == TC_STORE) {
                             a.y[(size_t)n * a.ldy + col] = v[j];
                         } else if (EPI == TC_RESID) {
                             a.x[(size_t)n * a.ldy + col] += v[j];
-                        } else {   // up projection: h = silu(gate) * up, gate from the previous pass
-                            const float g = a.y[(size_t)n * a.ldy + col];
-                            const float h = g / (1.f + expf(-g)) * v[j];
-                            uint16_t q[TC_PLANES];
-                            tc_split(h, q);
-#pragma unroll
-                            for (int i = 0; i < TC_PLANES; ++i) a.h[((size_t)i * npad + n) * a.nout + col] = q[i];
                         }
                     }
                 }
@@ -378,14 +378,16 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
 
 // ---------------------------------------------------------------- split-K reduction
 // out[n][col] = sum over the k-ranges (in order) of the partials, then the
-// GEMM's epilogue.
+// GEMM's epilogue.  TC_GLU: gate = output col, up = output nout_a + col, and
+// the planes of h = silu(gate) * up go to h [TC_PLANES][npad][nout_a].
 template <int EPI>
 __global__ void __launch_bounds__(256) tc_reduce_kernel(const TcArgs a) {
     pdl_trigger();
     pdl_wait();
     const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
-    if (idx >= (long long)a.R * a.nout) return;
-    const int n = (int)(idx / a.nout), col = (int)(idx % a.nout);
+    const int w = EPI == TC_GLU ? a.nout_a : a.nout;
+    if (idx >= (long long)a.R * w) return;
+    const int n = (int)(idx / w), col = (int)(idx % w);
     float v = 0.f;
     for (int sp = 0; sp < a.nsplit; ++sp) v += __ldcg(a.part + ((size_t)sp * a.R + n) * a.nout + col);
     if (EPI == TC_STORE) {
@@ -393,12 +395,13 @@ __global__ void __launch_bounds__(256) tc_reduce_kernel(const TcArgs a) {
     } else if (EPI == TC_RESID) {
         a.x[(size_t)n * a.ldy + col] += v;
     } else {
-        const float g = a.y[(size_t)n * a.ldy + col];
-        const float h = g / (1.f + expf(-g)) * v;
+        float u = 0.f;
+        for (int sp = 0; sp < a.nsplit; ++sp) u += __ldcg(a.part + ((size_t)sp * a.R + n) * a.nout + w + col);
+        const float h = v / (1.f + expf(-v)) * u;
         uint16_t q[TC_PLANES];
         tc_split(h, q);
 #pragma unroll
-        for (int i = 0; i < TC_PLANES; ++i) a.h[((size_t)i * a.npad + n) * a.nout + col] = q[i];
+        for (int i = 0; i < TC_PLANES; ++i) a.h[((size_t)i * a.npad + n) * w + col] = q[i];
     }
 }
 
@@ -446,6 +449,17 @@ __global__ void __launch_bounds__(256) planes_kernel(const PlaneArgs a) {
 #pragma unroll
         for (int i = 0; i < TC_PLANES; ++i)
             if (i < npl) p0[i * plane + k] = q[i];
+    }
+    if (a.src2) {   // a second part of the row, copied without normalisation
+        const float *x2 = a.src2 + (size_t)srow * a.d;
+        uint16_t *p2 = a.dst + (size_t)r * a.ld + a.col2;
+        for (int k = threadIdx.x; k < a.d; k += blockDim.x) {
+            uint16_t q[TC_PLANES];
+            tc_split(act ? x2[k] : 0.f, q);
+#pragma unroll
+            for (int i = 0; i < TC_PLANES; ++i)
+                if (i < npl) p2[i * plane + k] = q[i];
+        }
     }
 }
 
@@ -796,12 +810,22 @@ int tc_nsplit(int nout, int K, int sms) {
 
 cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s) {
     TcArgs a = a_in;
+    a.nout_a = a.nout;
+    return launch_tc2(a, wa, wa, xm, sms, s);
+}
+
+cudaError_t launch_tc2(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorMap &wb, const CUtensorMap &xm, int sms,
+                       cudaStream_t s) {
+    TcArgs a = a_in;
     if (a.npad % 16 || a.npad < 16 || a.npad > TC_MAX_ROWS || a.K % 64 || a.R > a.npad) return cudaErrorInvalidValue;
+    if (a.nout_a < 1 || a.nout_a > a.nout || (a.nout_a < a.nout && a.nout_a % 128)) return cudaErrorInvalidValue;
+    if (a.epi == TC_GLU && (a.nout != 2 * a.nout_a || !a.part || !a.h)) return cudaErrorInvalidValue;
     const int nkb = a.K / 64;
     if (a.epi == TC_LM && (!a.lm_part || a.lm_nsub != (a.nout + TC_LM_GROUP - 1) / TC_LM_GROUP))
         return cudaErrorInvalidValue;
     a.nsplit = a.part && a.epi != TC_LM ? tc_nsplit(a.nout, a.K, sms) : 1;   // the LM epilogue needs whole sums
     if ((long long)a.nsplit * a.R * a.nout > a.part_cap) a.nsplit = 1;
+    if (a.epi == TC_GLU && (long long)a.nsplit * a.R * a.nout > a.part_cap) return cudaErrorInvalidValue;
     a.kbps = (nkb + a.nsplit - 1) / a.nsplit;
     a.segkb = OSP_TC_SEGKB;
     constexpr int tmem_cols = 512 / OSP_TC_CTAS_PER_SM;
@@ -824,16 +848,22 @@ cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorM
     const size_t smem = tc_smem_bytes(a.npad, a.planes, na);
     cudaError_t e;
     switch (a.epi) {
-    case TC_STORE: e = pdl_launch(tc_kernel<TC_STORE, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
-    case TC_RESID: e = pdl_launch(tc_kernel<TC_RESID, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
-    case TC_GLU: e = pdl_launch(tc_kernel<TC_GLU, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst); break;
+    case TC_STORE:
+        e = pdl_launch(tc_kernel<TC_STORE, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, wb, xm, a, nst);
+        break;
+    case TC_RESID:
+        e = pdl_launch(tc_kernel<TC_RESID, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, wb, xm, a, nst);
+        break;
+    case TC_GLU: e = pdl_launch(tc_kernel<TC_GLU, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, wb, xm, a, nst); break;
     default:
-        e = na > 1 ? pdl_launch(tc_kernel<TC_LM, OSP_TC_LM_NA>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst)
-                   : pdl_launch(tc_kernel<TC_LM, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, xm, a, nst);
+        e = na > 1
+                ? pdl_launch(tc_kernel<TC_LM, OSP_TC_LM_NA>, dim3(grid), dim3(TC_THREADS), smem, s, wa, wb, xm, a, nst)
+                : pdl_launch(tc_kernel<TC_LM, 1>, dim3(grid), dim3(TC_THREADS), smem, s, wa, wb, xm, a, nst);
         break;
     }
-    if (e != cudaSuccess || a.nsplit == 1) return e;
-    const unsigned rblocks = (unsigned)(((long long)a.R * a.nout + 255) / 256);
+    if (e != cudaSuccess || (a.nsplit == 1 && a.epi != TC_GLU)) return e;
+    const unsigned rblocks =
+        (unsigned)(((long long)a.R * (a.epi == TC_GLU ? a.nout_a : a.nout) + 255) / 256);
     switch (a.epi) {
     case TC_STORE: return pdl_launch(tc_reduce_kernel<TC_STORE>, dim3(rblocks), dim3(256), 0, s, a);
     case TC_RESID: return pdl_launch(tc_reduce_kernel<TC_RESID>, dim3(rblocks), dim3(256), 0, s, a);

@@ -44,11 +44,12 @@ struct TcArgs {
     int R, npad;       // rows, rows padded to a multiple of 16
     int K;             // reduction length (multiple of 64)
     int nout;          // output features (tiles of 128, the last one may be partial)
+    int nout_a;        // features [0, nout_a) from the first weight map, the rest from the second
     int planes;        // 1 (bf16 input) or TC_PLANES (split float32 input)
-    float *y;          // TC_STORE: [R][ldy] float32 output; TC_GLU: the gate values read
+    float *y;          // TC_STORE: [R][ldy] float32 output
     int ldy;
     float *x;          // TC_RESID: [R][ldy] float32, +=
-    uint16_t *h;       // TC_GLU: [TC_PLANES][npad][nout] bf16 planes of silu(gate) * up
+    uint16_t *h;       // TC_GLU: [TC_PLANES][npad][nout_a] bf16 planes of silu(gate) * up
     int32_t *status;
     // TC_LM: partials [R][lm_nsub] (lm_nsub = ceil(nout / 32)), 1/T (1 for greedy)
     float4 *lm_part;
@@ -70,13 +71,15 @@ bool tc_encode_operand(CUtensorMap *m, const void *x, int planes, int npad, int 
 bool tc_encode_rows(CUtensorMap *m, const void *x, int rows, int npad, int K);
 size_t tc_smem_bytes(int npad, int planes, int na);
 cudaError_t tc_set_attributes();
-// SwiGLU runs as two passes: the gate projection (TC_STORE into a float32
-// buffer), then the up projection whose epilogue (TC_GLU) forms silu(gate) * up.
-// Outputs narrower than the CTA slots are split along K (tc_nsplit ranges per
-// 128-feature tile); the float32 partials are then summed in range order by a
-// reduction kernel that applies the epilogue.
+// SwiGLU runs as one GEMM over the gate rows (map wa) and the up rows (map wb),
+// nout = 2 nout_a; its partials always go to `part`, and the reduction forms
+// silu(gate) * up.  Outputs narrower than the CTA slots are split along K
+// (tc_nsplit ranges per 128-feature tile); the float32 partials are then summed
+// in range order by a reduction kernel that applies the epilogue.
 int tc_nsplit(int nout, int K, int sms);
 cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s);
+cudaError_t launch_tc2(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &wb, const CUtensorMap &xm, int sms,
+                       cudaStream_t s);
 
 // Operand preparation: rows of float32 (optionally RMS-normalised with a bf16
 // gain) written as bf16 planes [TC_PLANES][npad][ld] starting at column col0.
@@ -92,6 +95,8 @@ struct PlaneArgs {
     const int *valid;          // rows of invalid sequences are written as zeros (may be null)
     int rows_per_seq;
     int npl;                   // planes written (0: TC_PLANES)
+    const float *src2;         // optional second source, same rows, written plain at column col2
+    int col2;
 };
 cudaError_t launch_planes(const PlaneArgs &a, cudaStream_t s);
 
