@@ -437,9 +437,16 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
     // tensor-core path for 3..TC_MAX_ROWS activation rows
     auto tc_rows = [&](int rows) { return ctx->tc && rows >= 3 && rows <= TC_MAX_ROWS; };
     auto npad_of = [](int rows) { return (rows + 15) / 16 * 16; };
+    // the next GEMM's operand planes, written by a residual GEMM's reduction when it has one
+    struct NextPlanes {
+        uint16_t *dst;
+        const uint16_t *gain;
+        int ld, col0, npl, map, rows_per_seq, npad;
+    };
     auto tc_gemm = [&](int epi, int rows, int K_, int nout, int planes, const CUtensorMap &wa,
                        const void *xbuf, bool in_place_rows, float *y, int ldy, uint16_t *h,
-                       const char *what, const CUtensorMap *wb = nullptr) -> int {
+                       const char *what, const CUtensorMap *wb = nullptr, const NextPlanes *nxt = nullptr,
+                       bool *nxt_done = nullptr, const QkvPostArgs *rope = nullptr) -> int {
         const int np = npad_of(rows);
         CUtensorMap xm;
         const bool ok = in_place_rows ? tc_encode_rows(&xm, xbuf, rows, np, K_) : tc_encode_operand(&xm, xbuf, planes, np, K_);
@@ -459,7 +466,21 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         ta.part = ws.tc_part;
         ta.part_cap = ws.tc_part_cap;
         ta.nout_a = wb ? nout / 2 : nout;
-        const cudaError_t e2 = launch_tc2(ta, wa, wb ? *wb : wa, xm, ctx->sms, s);
+        if (nxt) {
+            ta.pl_dst = nxt->dst;
+            ta.pl_gain = nxt->gain;
+            ta.pl_eps = D.eps;
+            ta.pl_ld = nxt->ld;
+            ta.pl_col0 = nxt->col0;
+            ta.pl_npl = nxt->npl;
+            ta.pl_npad = nxt->npad;
+            ta.pl_map = nxt->map;
+            ta.pl_rows_per_seq = nxt->rows_per_seq;
+            ta.pl_max_new = max_new;
+            ta.pl_valid = ws.seq_valid;
+            ta.pl_nnew = ws.seq_nnew;
+        }
+        const cudaError_t e2 = launch_tc2(ta, wa, wb ? *wb : wa, xm, ctx->sms, s, nxt_done, rope);
         return e2 == cudaSuccess ? OSPREY_OK : cuda_fail(e2, what);
     };
     // the LM head of `rows` operand rows in ws.tc_xl on the tensor cores, with the
@@ -537,10 +558,15 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
         if (ctx->probe_kind != OSPREY_PROBE_ATTENTION || slot >= ctx->n_probe) return cudaSuccess;
         return probe_record(begin ? ctx->probe_begin[slot] : ctx->probe_end[slot], s);
     };
+    // the LM head's operand comes from the tensor-core planes (block drafting, or
+    // the tensor-core LM head) rather than the streamed or CUDA-core heads
+    const bool lm_tc = block || (!(topk <= 1 && B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) &&
+                                 (tc_rows(B) || topk > 1));
     for (int step = 0; step < K; ++step) {
         const bool ext = step == 0;
         const int rows_per_seq = ext ? max_new : 1;
         const int R = B * rows_per_seq;
+        bool xq_ready = false, xl_ready = false;   // operand planes already written by a reduction
         RowMap map{ws.seq_valid, ws.seq_pos0, ws.seq_nnew, rows_per_seq, step};
         float *x = ext ? ws.x_ext : ws.x_chain;
         float *sb = ext ? ws.s_ext : ws.s_chain;
@@ -601,12 +627,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             const int nqkv = (D.Hq + 2 * D.Hkv) * D.hd;
             int rc;
             // [s; RMSNorm(x)] -> QKV (Eq. 2-3) -> RoPE and the paged K/V rows; the s half
-            // of the operand is the same for every layer of the step
-            if ((rc = planes(x, (const uint16_t *)W.attn_norm[l], D.d, R, 2 * D.d, D.d, ws.tc_xq, rows_per_seq, false,
-                             "qkv operand", TC_PLANES, l == 0 ? sb : nullptr, 0)) != OSPREY_OK ||
-                (rc = tc_gemm(TC_STORE, R, 2 * D.d, nqkv, TC_PLANES, ctx->tm_qkv[l], ws.tc_xq, false, ws.tc_yq, nqkv,
-                              nullptr, "qkv launch")) != OSPREY_OK)
-                return rc;
+            // of the operand is the same for every layer of the step, and the x half of
+            // a later layer comes from the previous layer's down-projection reduction
             QkvPostArgs qp{};
             qp.dim = D;
             qp.map = map;
@@ -618,7 +640,15 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             qp.page_table = kv->page_table;
             qp.max_pages = kv->max_pages_per_seq;
             for (int i = 0; i < D.hd / 2; ++i) qp.inv_freq[i] = ctx->inv_freq[i];
-            if ((e = launch_qkv_post(qp, s)) != cudaSuccess) return cuda_fail(e, "rope launch");
+            // the QKV GEMM's reduction does RoPE and the K/V write when it runs
+            bool rope_done = false;
+            if ((!xq_ready &&
+                 (rc = planes(x, (const uint16_t *)W.attn_norm[l], D.d, R, 2 * D.d, D.d, ws.tc_xq, rows_per_seq, false,
+                              "qkv operand", TC_PLANES, l == 0 ? sb : nullptr, 0)) != OSPREY_OK) ||
+                (rc = tc_gemm(TC_STORE, R, 2 * D.d, nqkv, TC_PLANES, ctx->tm_qkv[l], ws.tc_xq, false, ws.tc_yq, nqkv,
+                              nullptr, "qkv launch", nullptr, nullptr, &rope_done, &qp)) != OSPREY_OK)
+                return rc;
+            if (!rope_done && (e = launch_qkv_post(qp, s)) != cudaSuccess) return cuda_fail(e, "rope launch");
             AttnArgs at{};
             at.dim = D;
             at.map = map;
@@ -632,6 +662,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             at.max_pages = kv->max_pages_per_seq;
             at.part = ws.attn_part;
             at.out = ws.attn_out;
+            at.out_planes = ws.tc_xo;   // the O projection's operand, written by attention itself
+            at.npad = npad_of(R);
             at.ticket = ws.attn_ticket;
             at.status = dev_status;
             if ((e = attn_probe(step * D.L + l, true)) != cudaSuccess) return cuda_fail(e, "probe record");
@@ -640,17 +672,36 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             if ((e = attn_probe(step * D.L + l, false)) != cudaSuccess) return cuda_fail(e, "probe record");
             // x += W_o attn;  x += W_down (silu(W_g n) * W_u n),  n = RMSNorm(x)
             const int ha = D.Hq * D.hd;
-            if ((rc = planes(ws.attn_out, nullptr, ha, R, ha, 0, ws.tc_xo, rows_per_seq, false, "o-proj operand")) !=
-                    OSPREY_OK ||
-                (rc = tc_gemm(TC_RESID, R, ha, D.d, TC_PLANES, ctx->tm_o[l], ws.tc_xo, false, x, D.d, nullptr,
-                              "o-proj launch")) != OSPREY_OK ||
-                (rc = planes(x, (const uint16_t *)W.ffn_norm[l], D.d, R, D.d, 0, ws.tc_xg, rows_per_seq, false,
-                             "gate/up operand")) != OSPREY_OK ||
+            const NextPlanes ffn{ws.tc_xg, (const uint16_t *)W.ffn_norm[l], D.d, 0, TC_PLANES, 0, rows_per_seq,
+                                 npad_of(R)};
+            bool ffn_ready = false;
+            if ((rc = tc_gemm(TC_RESID, R, ha, D.d, TC_PLANES, ctx->tm_o[l], ws.tc_xo, false, x, D.d, nullptr,
+                              "o-proj launch", nullptr, &ffn, &ffn_ready)) != OSPREY_OK ||
+                (!ffn_ready && (rc = planes(x, (const uint16_t *)W.ffn_norm[l], D.d, R, D.d, 0, ws.tc_xg, rows_per_seq,
+                                            false, "gate/up operand")) != OSPREY_OK) ||
                 (rc = tc_gemm(TC_GLU, R, D.d, 2 * D.F, TC_PLANES, ctx->tm_gate[l], ws.tc_xg, false, nullptr, 0,
-                              ws.tc_xh, "gate/up launch", &ctx->tm_up[l])) != OSPREY_OK ||
-                (rc = tc_gemm(TC_RESID, R, D.F, D.d, TC_PLANES, ctx->tm_down[l], ws.tc_xh, false, x, D.d, nullptr,
-                              "down launch")) != OSPREY_OK)
+                              ws.tc_xh, "gate/up launch", &ctx->tm_up[l])) != OSPREY_OK)
                 return rc;
+            // the down projection's reduction prepares the next layer's x half, or the
+            // LM head's operand rows after the last layer
+            NextPlanes nxt{};
+            const NextPlanes *nxtp = nullptr;
+            if (l + 1 < D.L) {
+                nxt = NextPlanes{ws.tc_xq, (const uint16_t *)W.attn_norm[l + 1], 2 * D.d, D.d, TC_PLANES, 0,
+                                 rows_per_seq, npad_of(R)};
+                nxtp = &nxt;
+            } else if (lm_tc) {
+                const bool last_rows = ext && !block;   // one LM row per sequence: its last new row
+                nxt = NextPlanes{ws.tc_xl, (const uint16_t *)W.final_norm, D.d, 0, TC_LM_PLANES, last_rows ? 1 : 0,
+                                 rows_per_seq, npad_of(last_rows ? B : R)};
+                nxtp = &nxt;
+            }
+            bool nxt_ready = false;
+            if ((rc = tc_gemm(TC_RESID, R, D.F, D.d, TC_PLANES, ctx->tm_down[l], ws.tc_xh, false, x, D.d, nullptr,
+                              "down launch", nullptr, nxtp, &nxt_ready)) != OSPREY_OK)
+                return rc;
+            xq_ready = nxt_ready && l + 1 < D.L;
+            xl_ready = nxt_ready && l + 1 == D.L;
         }
         for (int l = 0; l < D.L && !tcp; ++l) {
             if (streamed && R == 1 && ctx->fused_layer) {
@@ -758,8 +809,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             // sequence r / max_new proposes the token after it)
             const int rows = B * max_new;
             int rc;
-            if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, rows, D.d, 0, ws.tc_xl, max_new, false,
-                             "lm operand", TC_LM_PLANES)) != OSPREY_OK)
+            if (!xl_ready && (rc = planes(x, (const uint16_t *)W.final_norm, D.d, rows, D.d, 0, ws.tc_xl, max_new, false,
+                                          "lm operand", TC_LM_PLANES)) != OSPREY_OK)
                 return rc;
             LmPickArgs pk{};
             pk.B = rows;
@@ -796,8 +847,8 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             // epilogue (logits stored only into draft_logits) -> one pick per row
             // (topk candidates per row when drafting a tree)
             int rc;
-            if ((rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext, "lm operand",
-                             TC_LM_PLANES)) != OSPREY_OK)
+            if (!xl_ready && (rc = planes(x, (const uint16_t *)W.final_norm, D.d, B, D.d, 0, ws.tc_xl, 1, ext,
+                                          "lm operand", TC_LM_PLANES)) != OSPREY_OK)
                 return rc;
             LmPickArgs pk{};
             pk.B = B;

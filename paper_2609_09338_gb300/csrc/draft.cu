@@ -238,6 +238,26 @@ __global__ void __launch_bounds__(GT) gemv_kernel(const GemvArgs a) {
     }
 }
 
+// Attention output element (row r, column col of the Hq hd heads): float32
+// into out, or the three bf16 planes x ~= q0 + q1 + q2 (q_i the bf16 rounding of
+// what the earlier planes leave) of the O projection's tensor-core operand.
+__device__ __forceinline__ void attn_store(const AttnArgs &a, int r, int col, float v) {
+    const int ha = a.dim.Hq * a.dim.hd;
+    if (!a.out_planes) {
+        a.out[(size_t)r * ha + col] = v;
+        return;
+    }
+    const size_t plane = (size_t)a.npad * ha;
+    uint16_t *p = a.out_planes + (size_t)r * ha + col;
+    float rem = v;
+#pragma unroll
+    for (int i = 0; i < 3; ++i) {
+        const uint16_t q = f_to_bf(rem);
+        p[i * plane] = q;
+        rem -= bf_to_f(q);
+    }
+}
+
 // ---------------------------------------------------------------------------
 // Split-KV GQA decode attention (Sec. 4, paged serving).  Both kernels below
 // give a block (key range, KV head, row) and its warps the range's pages
@@ -592,7 +612,7 @@ __global__ void __launch_bounds__(AT) attn_kernel(const AttnArgs a) {
         const int idx = threadIdx.x + it * AT;
         if (idx >= G * HD) continue;
         const int g = idx / HD, dim = idx % HD;
-        a.out[(size_t)r * Hq * HD + (size_t)(kvh * G + g) * HD + dim] = num[it] / s_den[g];
+        attn_store(a, r, (kvh * G + g) * HD + dim, num[it] / s_den[g]);
     }
 }
 
@@ -689,7 +709,7 @@ __global__ void __launch_bounds__(AttnCluster<HD, G, CS>::THREADS, 1) attn_clust
             num = fmaf(f, gacc[k][g][dim], num);
             den = fmaf(f, gl[k][g], den);
         }
-        a.out[(size_t)r * D.Hq * HD + (size_t)(qh0 + g) * HD + dim] = num / den;
+        attn_store(a, r, (qh0 + g) * HD + dim, num / den);
     }
 }
 

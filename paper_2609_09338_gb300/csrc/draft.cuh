@@ -99,6 +99,10 @@ struct AttnArgs {
     int max_pages;
     float *part;
     float *out;
+    // when set, the output rows go to the O projection's tensor-core operand
+    // instead of out: three bf16 planes [3][npad][Hq hd]
+    uint16_t *out_planes;
+    int npad;
     int *ticket;
     int32_t *status;
 };

@@ -15,6 +15,7 @@
 //              other TMEM buffer.
 // Every wait is bounded; on expiry the CTA records OSPREY_ERR_TIMEOUT, stops
 // issuing, lets its copies and MMAs land and frees its TMEM.
+#include <cooperative_groups.h>
 #include <cudaTypedefs.h>
 #include <math.h>
 
@@ -24,6 +25,8 @@
 #include "tma.cuh"
 
 namespace osp {
+
+namespace cg = cooperative_groups;
 
 constexpr int TC_THREADS = 192;
 constexpr int TC_ABYTES = 128 * 128;    // weight tile: 128 rows x 64 bf16
@@ -405,6 +408,90 @@ __global__ void __launch_bounds__(256) tc_reduce_kernel(const TcArgs a) {
     }
 }
 
+// TC_RESID reduction with the next operand's planes: a cluster of RP_CS blocks
+// per row n, each summing the partials (in range order) of its share of the
+// columns into x[n]; the blocks' sums of squares are exchanged through
+// distributed shared memory, then each writes the RMS-normalised planes of its
+// columns.
+constexpr int RP_CS = 8;     // blocks per row (one cluster)
+constexpr int RP_VPT = 4;    // columns per thread at most (nout <= RP_CS * 256 * RP_VPT)
+__device__ __forceinline__ void rp_cluster_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void rp_cluster_arrive_release() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void rp_cluster_wait_acquire() {
+    asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+__global__ void __launch_bounds__(256) tc_resid_planes_kernel(const TcArgs a) {
+    __shared__ float red[8];
+    __shared__ float css[RP_CS];   // every block's sum of squares, pushed by its owner
+    cg::cluster_group cluster = cg::this_cluster();
+    const int rank = (int)cluster.block_rank(), n = blockIdx.y, t = threadIdx.x;
+    rp_cluster_arrive_relaxed();   // started: the cluster may write this block's shared memory
+    pdl_trigger();
+    pdl_wait();
+    int prow = -1;
+    bool act = false;
+    if (a.pl_map == 0) {
+        const int b = n / a.pl_rows_per_seq, j = n - b * a.pl_rows_per_seq;
+        act = a.pl_valid[b] && (a.pl_rows_per_seq == 1 || j < a.pl_nnew[b]);
+        prow = n;
+    } else {
+        const int b = n / a.pl_max_new, j = n - b * a.pl_max_new;
+        if (a.pl_valid[b] ? j == a.pl_nnew[b] - 1 : j == 0) {
+            prow = b;
+            act = a.pl_valid[b] != 0;
+        }
+    }
+    const int per = (a.nout + RP_CS - 1) / RP_CS;
+    const int c0 = rank * per, c1 = min(a.nout, c0 + per);
+    float xv[RP_VPT];
+    float ss = 0.f;
+#pragma unroll
+    for (int i = 0; i < RP_VPT; ++i) {
+        const int col = c0 + t + 256 * i;
+        xv[i] = 0.f;
+        if (col >= c1) continue;
+        float v = 0.f;
+        for (int sp = 0; sp < a.nsplit; ++sp) v += __ldcg(a.part + ((size_t)sp * a.R + n) * a.nout + col);
+        const float xn = a.x[(size_t)n * a.ldy + col] + v;
+        a.x[(size_t)n * a.ldy + col] = xn;
+        xv[i] = xn;
+        ss = fmaf(xn, xn, ss);
+    }
+    if (prow < 0) return;   // the whole cluster (same row) leaves here
+    ss = warp_sum(ss);
+    if ((t & 31) == 0) red[t >> 5] = ss;
+    __syncthreads();
+    rp_cluster_wait_acquire();   // every block of the cluster has started
+    if (t == 0) {
+        float tot = 0.f;
+        for (int w = 0; w < 8; ++w) tot += red[w];
+        for (int k = 0; k < RP_CS; ++k) *cluster.map_shared_rank(&css[rank], k) = tot;
+    }
+    rp_cluster_arrive_release();
+    rp_cluster_wait_acquire();   // every block's sum has arrived here
+    float tot = 0.f;
+#pragma unroll
+    for (int k = 0; k < RP_CS; ++k) tot += css[k];
+    const float inv = rsqrtf(tot / (float)a.nout + a.pl_eps);
+    uint16_t *p0 = a.pl_dst + (size_t)prow * a.pl_ld + a.pl_col0;
+    const size_t plane = (size_t)a.pl_npad * a.pl_ld;
+#pragma unroll
+    for (int i = 0; i < RP_VPT; ++i) {
+        const int col = c0 + t + 256 * i;
+        if (col >= c1) continue;
+        const float v = act ? xv[i] * inv * bf_to_f(a.pl_gain[col]) : 0.f;
+        uint16_t q[TC_PLANES];
+        tc_split(v, q);
+#pragma unroll
+        for (int j = 0; j < TC_PLANES; ++j)
+            if (j < a.pl_npl) p0[j * plane + col] = q[j];
+    }
+}
+
 // ---------------------------------------------------------------- operand planes
 __global__ void __launch_bounds__(256) planes_kernel(const PlaneArgs a) {
     __shared__ float red[33];
@@ -494,6 +581,49 @@ __global__ void __launch_bounds__(256) qkv_post_kernel(const QkvPostArgs a) {
         const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
         const int page = a.page_table[(size_t)b * a.max_pages + pos / D.P];
         uint16_t *dst = (is_k ? a.k_pages : a.v_pages) + (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * D.hd;
+        dst[ii] = f_to_bf(x1);
+        dst[ii + half] = f_to_bf(x2);
+    }
+}
+
+// The QKV GEMM's split-K reduction with RoPE and the paged K/V write folded
+// in: each thread sums the partials (in range order) of one rotary pair
+// (ii, ii + hd / 2) of one head, then does what qkv_post_kernel does with it.
+__global__ void __launch_bounds__(256) tc_reduce_rope_kernel(const TcArgs a, const QkvPostArgs p) {
+    const Dims &D = p.dim;
+    const int half = D.hd / 2;
+    const int per_row = (D.Hq + 2 * D.Hkv) * half;
+    pdl_trigger();
+    pdl_wait();
+    const long long idx = (long long)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= (long long)a.R * per_row) return;
+    const int r = (int)(idx / per_row), item = (int)(idx % per_row);
+    int b, pos;
+    if (!p.map.row(r, b, pos)) return;
+    const int h = item / half, ii = item % half;
+    const int col = h * D.hd + ii;
+    float x1 = 0.f, x2 = 0.f;
+    for (int sp = 0; sp < a.nsplit; ++sp) {
+        const float *pr = a.part + ((size_t)sp * a.R + r) * a.nout;
+        x1 += __ldcg(pr + col);
+        x2 += __ldcg(pr + col + half);
+    }
+    if (h < D.Hq + D.Hkv) {
+        float c, sn;
+        rope_cs2(p.inv_freq[ii], pos, c, sn);
+        const float y1 = x1 * c - x2 * sn, y2 = x2 * c + x1 * sn;
+        x1 = y1;
+        x2 = y2;
+    }
+    if (h < D.Hq) {
+        float *q = p.q + (size_t)r * D.Hq * D.hd + (size_t)h * D.hd;
+        q[ii] = x1;
+        q[ii + half] = x2;
+    } else {
+        const bool is_k = h < D.Hq + D.Hkv;
+        const int kvh = is_k ? h - D.Hq : h - D.Hq - D.Hkv;
+        const int page = p.page_table[(size_t)b * p.max_pages + pos / D.P];
+        uint16_t *dst = (is_k ? p.k_pages : p.v_pages) + (((size_t)page * D.Hkv + kvh) * D.P + pos % D.P) * D.hd;
         dst[ii] = f_to_bf(x1);
         dst[ii + half] = f_to_bf(x2);
     }
@@ -815,8 +945,9 @@ cudaError_t launch_tc(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorM
 }
 
 cudaError_t launch_tc2(const TcArgs &a_in, const CUtensorMap &wa, const CUtensorMap &wb, const CUtensorMap &xm, int sms,
-                       cudaStream_t s) {
+                       cudaStream_t s, bool *planes_done, const QkvPostArgs *rope) {
     TcArgs a = a_in;
+    if (planes_done) *planes_done = false;
     if (a.npad % 16 || a.npad < 16 || a.npad > TC_MAX_ROWS || a.K % 64 || a.R > a.npad) return cudaErrorInvalidValue;
     if (a.nout_a < 1 || a.nout_a > a.nout || (a.nout_a < a.nout && a.nout_a % 128)) return cudaErrorInvalidValue;
     if (a.epi == TC_GLU && (a.nout != 2 * a.nout_a || !a.part || !a.h)) return cudaErrorInvalidValue;
@@ -862,6 +993,31 @@ cudaError_t launch_tc2(const TcArgs &a_in, const CUtensorMap &wa, const CUtensor
         break;
     }
     if (e != cudaSuccess || (a.nsplit == 1 && a.epi != TC_GLU)) return e;
+    if (a.epi == TC_RESID && a.pl_dst && a.nout <= RP_CS * 256 * RP_VPT) {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(RP_CS, a.R);
+        cfg.blockDim = dim3(256);
+        cfg.stream = s;
+        cudaLaunchAttribute attr[2];
+        attr[0].id = cudaLaunchAttributeClusterDimension;
+        attr[0].val.clusterDim.x = RP_CS;
+        attr[0].val.clusterDim.y = 1;
+        attr[0].val.clusterDim.z = 1;
+        attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[1].val.programmaticStreamSerializationAllowed = 1;
+        cfg.attrs = attr;
+        cfg.numAttrs = 2;
+        e = cudaLaunchKernelEx(&cfg, tc_resid_planes_kernel, a);
+        count_launch();
+        if (e == cudaSuccess && planes_done) *planes_done = true;
+        return e;
+    }
+    if (a.epi == TC_STORE && rope) {
+        const long long n = (long long)a.R * (rope->dim.Hq + 2 * rope->dim.Hkv) * (rope->dim.hd / 2);
+        e = pdl_launch(tc_reduce_rope_kernel, dim3((unsigned)((n + 255) / 256)), dim3(256), 0, s, a, *rope);
+        if (e == cudaSuccess && planes_done) *planes_done = true;
+        return e;
+    }
     const unsigned rblocks =
         (unsigned)(((long long)a.R * (a.epi == TC_GLU ? a.nout_a : a.nout) + 255) / 256);
     switch (a.epi) {

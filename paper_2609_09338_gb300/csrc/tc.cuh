@@ -55,6 +55,18 @@ struct TcArgs {
     float4 *lm_part;
     int lm_nsub;
     float lm_invT;
+    // TC_RESID with a split-K reduction and pl_dst set: the reduction runs one
+    // block per row and also writes the updated rows' RMS-normalised planes for
+    // the next GEMM (gain pl_gain, pl_npl planes [pl_npl][pl_npad][pl_ld] from
+    // column pl_col0).  pl_map 0: row n to planes row n (zeros unless sequence
+    // n / pl_rows_per_seq is valid and, with several rows per sequence, n is one
+    // of its new rows); 1: the last new row of each sequence to its planes row
+    // (zeros for an invalid sequence).
+    uint16_t *pl_dst;
+    const uint16_t *pl_gain;
+    float pl_eps;
+    int pl_ld, pl_col0, pl_npl, pl_npad, pl_map, pl_rows_per_seq, pl_max_new;
+    const int *pl_valid, *pl_nnew;
     // split-K: per-range float32 partials [nsplit][R][nout] (null: no split)
     float *part;
     long long part_cap;   // floats available in part
@@ -78,8 +90,13 @@ cudaError_t tc_set_attributes();
 // in range order by a reduction kernel that applies the epilogue.
 int tc_nsplit(int nout, int K, int sms);
 cudaError_t launch_tc(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &xm, int sms, cudaStream_t s);
+// *planes_done (when given) tells whether the reduction did the follow-up work:
+// wrote the pl_* planes (TC_RESID), or RoPE and the K/V write of `rope`
+// (TC_STORE of the QKV projection) instead of storing y.  Otherwise the caller
+// does it itself.
+struct QkvPostArgs;
 cudaError_t launch_tc2(const TcArgs &a, const CUtensorMap &wa, const CUtensorMap &wb, const CUtensorMap &xm, int sms,
-                       cudaStream_t s);
+                       cudaStream_t s, bool *planes_done = nullptr, const QkvPostArgs *rope = nullptr);
 
 // Operand preparation: rows of float32 (optionally RMS-normalised with a bf16
 // gain) written as bf16 planes [TC_PLANES][npad][ld] starting at column col0.
