@@ -562,11 +562,14 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
     // the tensor-core LM head) rather than the streamed or CUDA-core heads
     const bool lm_tc = block || (!(topk <= 1 && B <= 2 && stream_supported(G_LM, D, B, ctx->sms)) &&
                                  (tc_rows(B) || topk > 1));
+    bool xq_next = false;   // the previous step's pick wrote this step's first QKV operand
     for (int step = 0; step < K; ++step) {
         const bool ext = step == 0;
         const int rows_per_seq = ext ? max_new : 1;
         const int R = B * rows_per_seq;
-        bool xq_ready = false, xl_ready = false;   // operand planes already written by a reduction
+        // operand planes already written by an earlier kernel (a reduction, the pick)
+        bool xq_ready = xq_next, xl_ready = false;
+        xq_next = false;
         RowMap map{ws.seq_valid, ws.seq_pos0, ws.seq_nnew, rows_per_seq, step};
         float *x = ext ? ws.x_ext : ws.x_chain;
         float *sb = ext ? ws.s_ext : ws.s_chain;
@@ -865,6 +868,13 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             pk.x_in = x;
             pk.x_chain = ws.x_chain;
             pk.s_chain = ws.s_chain;
+            if (step + 1 < K && B > 2 && tc_rows(B)) {   // the next step's layers run on the tensor cores
+                pk.qkv_planes = ws.tc_xq;
+                pk.qkv_gain = (const uint16_t *)W.attn_norm[0];
+                pk.eps = D.eps;
+                pk.qkv_npad = npad_of(B);
+                xq_next = true;
+            }
             if ((rc = tc_lm(B, draft_logits ? draft_logits + (size_t)step * D.V : nullptr, (long long)K * D.V, pk)) !=
                 OSPREY_OK)
                 return rc;

@@ -806,9 +806,37 @@ __global__ void __launch_bounds__(PK_THREADS) lm_pick_kernel(const LmPickArgs a)
         const int src = a.src_is_ext ? b * a.max_new + a.nnew[b] - 1 : b;
         const float *xl = a.x_in + (size_t)src * D.d;
         const uint16_t *er = a.embed + (size_t)token * D.d;
+        float ss = 0.f;
         for (int k = t; k < D.d; k += PK_THREADS) {
+            const float e = bf_to_f(er[k]);
             a.s_chain[(size_t)b * D.d + k] = xl[k];
-            a.x_chain[(size_t)b * D.d + k] = bf_to_f(er[k]);
+            a.x_chain[(size_t)b * D.d + k] = e;
+            ss = fmaf(e, e, ss);
+        }
+        if (a.qkv_planes) {   // and its first layer's operand, [s; RMSNorm(x)]
+            ss = warp_sum(ss);
+            if (lane == 0) sh[warp] = ss;
+            __syncthreads();
+            if (t == 0) {
+                float tot = 0.f;
+                for (int w = 0; w < PK_THREADS / 32; ++w) tot += sh[w];
+                sh[33] = rsqrtf(tot / (float)D.d + a.eps);
+            }
+            __syncthreads();
+            const float inv = sh[33];
+            const size_t ld = 2 * (size_t)D.d, plane = (size_t)a.qkv_npad * ld;
+            uint16_t *p0 = a.qkv_planes + (size_t)b * ld;
+            for (int k = t; k < D.d; k += PK_THREADS) {
+                // the s half from this thread's own copy in s_chain: x_in may be x_chain,
+                // whose row b now holds the embedding
+                uint16_t q[TC_PLANES];
+                tc_split(a.s_chain[(size_t)b * D.d + k], q);
+#pragma unroll
+                for (int i = 0; i < TC_PLANES; ++i) p0[i * plane + k] = q[i];
+                tc_split(bf_to_f(er[k]) * inv * bf_to_f(a.qkv_gain[k]), q);
+#pragma unroll
+                for (int i = 0; i < TC_PLANES; ++i) p0[i * plane + D.d + k] = q[i];
+            }
         }
     }
 }

@@ -159,6 +159,12 @@ struct LmPickArgs {
     const float *x_in;         // residual rows of the step (x_ext or x_chain)
     float *x_chain, *s_chain;
     const uint16_t *embed;
+    // when set (chain drafting on the tensor cores), the next chain row's QKV
+    // operand too: [TC_PLANES][qkv_npad][2 d] bf16 planes of [s; RMSNorm(x) * qkv_gain]
+    uint16_t *qkv_planes;
+    const uint16_t *qkv_gain;
+    float eps;
+    int qkv_npad;
 };
 cudaError_t launch_lm_pick(const LmPickArgs &a, cudaStream_t s);
 // Block drafting inputs (EAGLE-style DFlash): for row r = b*P + j of n
