@@ -959,7 +959,9 @@ static cudaError_t pdl_launch(void (*k)(P...), dim3 grid, dim3 block, size_t sme
 #endif
 int tc_nsplit(int nout, int K, int sms) {
     const int tiles = (nout + 127) / 128, nkb = K / 64;
-    int want = (OSP_TC_CTAS_PER_SM * sms + tiles - 1) / tiles;
+    // at most one item per CTA slot: one item more than the slots would take two
+    // item times for barely more than one wave of work
+    int want = OSP_TC_CTAS_PER_SM * sms / tiles;
     if (want < 1) want = 1;
     if (want > nkb / OSP_TC_MIN_KB) want = nkb / OSP_TC_MIN_KB > 1 ? nkb / OSP_TC_MIN_KB : 1;
     const int kbps = (nkb + want - 1) / want;
