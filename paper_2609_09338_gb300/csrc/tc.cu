@@ -180,10 +180,31 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
     tc_fence_after();
     const uint32_t tmem = s_tmem;
     pdl_trigger();
-    pdl_wait();   // the activation planes and the residual come from earlier kernels
+    // the activation planes and the residual come from earlier kernels; the
+    // producer first requests the weight tiles of the ring's first stages,
+    // which do not, and waits after that
+    if (warp != 0) pdl_wait();
 
     if (warp == 0) {
         if (lane == 0) {
+            auto weights = [&](uint8_t *st, int y, int kb, uint64_t *bar) {
+#pragma unroll
+                for (int t = 0; t < NA; ++t) {
+                    const int f = y + 128 * t;   // tiles never straddle nout_a (a multiple of 128)
+                    tma_2d(st + t * TC_ABYTES, f < a.nout_a ? &wa : &wb, kb * 64, f < a.nout_a ? f : f - a.nout_a, bar);
+                }
+            };
+            long long npre = 0;   // stages whose weights were requested before the wait
+            for (int it = 0; it < nloc && npre < nst; ++it) {
+                const int y = (i0 + it) / a.nsplit * 128 * NA;
+                int klo, khi;
+                krange(i0 + it, klo, khi);
+                for (int kb = klo; kb < khi && npre < nst; ++kb, ++npre) {
+                    mbar_expect_tx(&full[npre], NA * TC_ABYTES);
+                    weights(sm + (size_t)npre * stage, y, kb, &full[npre]);
+                }
+            }
+            pdl_wait();
             long long g = 0;
             bool stop = false;
             for (int it = 0; it < nloc && !stop; ++it) {
@@ -200,20 +221,24 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                     }
                     if (*(volatile int *)&s_abort) { stop = true; break; }
                     uint8_t *st = sm + (size_t)s * stage;
-                    mbar_arrive_expect_tx(&full[s], stage);
-#pragma unroll
-                    for (int t = 0; t < NA; ++t) {
-                        const int f = y + 128 * t;   // tiles never straddle nout_a (a multiple of 128)
-                        tma_2d(st + t * TC_ABYTES, f < a.nout_a ? &wa : &wb, kb * 64, f < a.nout_a ? f : f - a.nout_a,
-                               &full[s]);
+                    if (g < npre) {
+                        mbar_arrive_expect_tx(&full[s], bbytes);
+                    } else {
+                        mbar_arrive_expect_tx(&full[s], stage);
+                        weights(st, y, kb, &full[s]);
                     }
                     for (int p = 0; p < a.planes; ++p)
                         tma_2d(st + NA * TC_ABYTES + (size_t)p * npad * 128, &xm, kb * 64, p * npad, &full[s]);
                 }
             }
-            if (stop)   // let the copies this thread issued land before the CTA can exit
-                for (long long q = g - nst > 0 ? g - nst : 0; q < g; ++q)
+            if (stop) {   // let the copies this thread issued land before the CTA can exit
+                // stages whose weights were requested early but never armed: arrive, so
+                // that their phase completes when the weights land
+                for (long long q = g; q < npre; ++q) mbar_arrive(&full[q]);
+                const long long end = g > npre ? g : npre;
+                for (long long q = end - nst > 0 ? end - nst : 0; q < end; ++q)
                     mbar_wait(&full[q % nst], (uint32_t)(q / nst) & 1, 200000000LL);
+            }
         }
     } else if (warp == 1) {
         if (lane == 0) {
