@@ -42,6 +42,12 @@ from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: 
 LM_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/stream.cu",
               "sha256": "90d10a609dc3cdd6796755d7c6ff7213e7e7ddeb5064fcb5779e04778e7230de",
               "bytes_per_launch": 314_359_808}
+# DRAM bytes (read + write) of one attention launch at the large-vocabulary
+# workload, from one ncu capture of this source (profiles/attn_large-vocab-*.md)
+ATTN_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/draft.cu",
+                "sha256": "945657d709f2eaf25536b42ea209467dc8ded111749c3da39e67f610b277bde6",
+                "workload": "large-vocab-d1024-v200064-b64-k8",
+                "bytes_per_launch": 2_162_905_856 + 16_101_376}
 
 
 def _sha(path):
@@ -346,11 +352,13 @@ def lm_head_label(B, block=False):
     """The LM-head launches the probes bracket, by the number of rows (the draft
     step's kernel selection)."""
     if block:
-        return "planes_kernel + tc_kernel<STORE> + row_sample_kernel over every block row (tcgen05 LM head)"
+        return ("tc_kernel<LM> + lm_pick_kernel over every block row (tcgen05 LM head with per-32-id sampling "
+                "partials in its epilogue, then the pick; the operand planes come from the last down projection)")
     if B <= 2:
         return "stream_kernel<LM> (final RMSNorm + TMA-streamed LM-head GEMV + on-chip sampling)"
     if B <= 80:
-        return "planes_kernel + tc_kernel<STORE> + row_sample_kernel (tcgen05 LM head, then sampling)"
+        return ("tc_kernel<LM> + lm_pick_kernel (tcgen05 LM head, two weight tiles per stage, per-32-id sampling "
+                "partials in its epilogue, then the pick)")
     return "lm_head_kernel (CUDA-core LM head + on-chip sampling)"
 
 
@@ -626,9 +634,12 @@ def measure(wl, args, rank, world, local, full):
         # bytes of all the call's attention launches / their summed duration
         call_ms = sum(sum(p) for p in probe_ms) / len(probe_ms)
         achieved = nb["attn_call"] / (call_ms * 1e-3) / 1e9
+        attn_sha = _sha(os.path.join(ROOT, ATTN_TRAFFIC["source"]))
+        traffic = (ATTN_TRAFFIC["bytes_per_launch"]
+                   if attn_sha == ATTN_TRAFFIC["sha256"] and wl.name == ATTN_TRAFFIC["workload"] else None)
         roof = {"kernel": "split-KV GQA decode attention (attn_kernel / attn_cluster_kernel), all launches of a call",
                 "bound": "hbm", "achieved": achieved, "peak": peak, "unit": "GB/s", "frac": achieved / peak,
-                "traffic": None, "peak_kind": peak_kind,
+                "traffic": traffic, "peak_kind": peak_kind,
                 "bytes_per_launch": nb["attn_call"] / nb["attn_launches"],
                 "mean_launch_us": 1e3 * call_ms / nb["attn_launches"], "launches_timed": len(probe_ms) * n_probe}
     else:
