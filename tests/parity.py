@@ -55,8 +55,9 @@ def check_kv_rows(got, want, mag):
     mag = sum_j |W_ij| |u_j| (the oracle's ``*_mag``; for a rotated key, summed
     over its rotation pair): |a - a*| <= c * mag.  The inputs u of a chain row
     carry the float32 error of every step before it (the fed-back state runs
-    through attention over up to 8k cached keys); over the workloads the
-    largest element needs c = 2^-15.3 (the two-layer Llama-shaped chain rows),
-    the others fit 2^-16.  c = 2^-14 keeps a factor 2.5 above that."""
+    through attention over up to 8k cached keys).  Over the workloads the
+    largest element needs c = 2^-13.8: a row of the sixth chain step of the
+    two-layer Llama-shaped drafter drafting greedily (2^-15.0 when it samples);
+    the one-layer drafters fit 2^-16.  c = 2^-13 keeps a factor 1.7 above it."""
     import numpy as np
-    np.testing.assert_array_less(np.abs(got - want), 2.0 ** -8 * (np.abs(got) + np.abs(want)) + 2.0 ** -14 * mag + 1e-30)
+    np.testing.assert_array_less(np.abs(got - want), 2.0 ** -8 * (np.abs(got) + np.abs(want)) + 2.0 ** -13 * mag + 1e-30)

@@ -84,7 +84,9 @@ def test_verify_workload_shapes(name):
         g = _run(vi, wl.temperature, dtype)
         o = _oracle(vi, wl.temperature, dtype)
         nflag = check_verify(g["out_tokens"], g["n_accepted"], o, wl.K)
-        assert nflag <= max(1, wl.batch // 8)
+        # on these seeded inputs the oracle flags at most one sequence (the large-vocabulary
+        # float32 logits; none elsewhere), so every other one is compared bit for bit
+        assert nflag <= 1
         np.testing.assert_allclose(g["probs"][..., 0], o["p_x"], atol=1e-5)
         # greedy on the same logits
         g0 = _run(vi, 0.0, dtype)
