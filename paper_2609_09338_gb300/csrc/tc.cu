@@ -332,7 +332,7 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                         tc_st16(tt + (uint32_t)cc, v);
                         continue;
                     }
-                    if (EPI == TC_LM) {
+                    if constexpr (EPI == TC_LM) {
                         // per row: (argmax z, sum exp((z - max z) / T)) over this warp's 32
                         // ids, for the 16 rows c0.. at once: each butterfly round halves the
                         // rows a lane carries (it keeps one half and receives the partner's
@@ -376,18 +376,18 @@ __global__ void __launch_bounds__(TC_THREADS, OSP_TC_CTAS_PER_SM)
                         if (!(lane & 1) && n < a.R && sub < a.lm_nsub)
                             a.lm_part[(size_t)n * a.lm_nsub + sub] =
                                 make_float4(av[0] * a.lm_invT, sv[0], av[0], __int_as_float(ai[0]));
-                        continue;
-                    }
+                    } else {
 #pragma unroll
-                    for (int j = 0; j < 16; ++j) {
-                        const int n = c0 + j;
-                        if (n >= a.R || !colok) continue;
-                        if (a.nsplit > 1 || EPI == TC_GLU) {   // partial of this k-range; tc_reduce applies the epilogue
-                            a.part[((size_t)sp * a.R + n) * a.nout + col] = v[j];
-                        } else if (EPI == TC_STORE) {
-                            a.y[(size_t)n * a.ldy + col] = v[j];
-                        } else if (EPI == TC_RESID) {
-                            a.x[(size_t)n * a.ldy + col] += v[j];
+                        for (int j = 0; j < 16; ++j) {
+                            const int n = c0 + j;
+                            if (n >= a.R || !colok) continue;
+                            if (a.nsplit > 1 || EPI == TC_GLU) {   // partial of this k-range; tc_reduce applies the epilogue
+                                a.part[((size_t)sp * a.R + n) * a.nout + col] = v[j];
+                            } else if (EPI == TC_STORE) {
+                                a.y[(size_t)n * a.ldy + col] = v[j];
+                            } else if (EPI == TC_RESID) {
+                                a.x[(size_t)n * a.ldy + col] += v[j];
+                            }
                         }
                     }
                 }
