@@ -258,7 +258,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
     const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
-    size_t o_lz = take(4ull * B * D.V);   // the streamed LM head's logits row (rows <= 2)
+    size_t o_lz = take(8ull * B * lmp.blocks * lmp.nsup);   // the streamed LM head's run statistics (rows <= 2)
     size_t o_lc = take(16ull * B * lmp.blocks);
     // tensor-core path: bf16 operand planes, QKV output, row-sampler partials
     const long long tc_rows = std::min<long long>(std::max<long long>(R_ext, B), TC_MAX_ROWS);
@@ -304,7 +304,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->attn_out = (float *)(p + o_ao);
         ws->ffn_h = (float *)(p + o_fh);
         ws->lm_stats = (float4 *)(p + o_ls);
-        ws->lm_z = (float *)(p + o_lz);
+        ws->lm_sup = (float2 *)(p + o_lz);
         ws->lm_cta_stats = (float4 *)(p + o_lc);
         ws->tc_xq = (uint16_t *)(p + o_xq);
         ws->tc_yq = (float *)(p + o_yq);
@@ -841,7 +841,10 @@ static int draft_step_impl(osprey_ctx *ctx, const osprey_kv *kv, int B, int K, i
             sa.qx = draft_qx;
             sa.stats = draft_stats;
             sa.logits = draft_logits;
-            sa.z = ws.lm_z;
+            sa.sup = ws.lm_sup;
+            const StreamPlan lp = stream_plan(G_LM, D, ctx->sms);
+            sa.nsup = lp.nsup;
+            sa.run = lp.run;
             sa.cta_stats = ws.lm_cta_stats;
             sa.ticket = ws.lm_ticket;
             if ((e = launch_stream(G_LM, sa, B, s)) != cudaSuccess) return cuda_fail(e, "lm head launch");

@@ -29,7 +29,7 @@ struct DraftWs {
     float *attn_out;                       // [R_ext][Hq*hd]
     float *ffn_h;                          // [R_ext][F]
     float4 *lm_stats;                      // [B][lm_warps]
-    float *lm_z;                           // [B][V] logits of the chain step (streamed LM head)
+    float2 *lm_sup;                        // [B][blocks][nsup] run statistics of the streamed LM head
     float4 *lm_cta_stats;                  // [B][sms]
     // tensor-core path (rows padded to np <= 80): bf16 operand planes [TC_PLANES][np][...]
     uint16_t *tc_xq;                       // [P][np][2d]    [s; RMSNorm(x)] for QKV
@@ -164,8 +164,9 @@ struct StreamArgs {
     float temperature;
     const float *u_draft;
     int32_t *tokens;
-    float *qx, *stats, *logits;
-    float *z;                     // [B][V] logits of the chain step (when logits is null)
+    float *qx, *stats, *logits;   // logits: the caller's draft_logits (optional output)
+    float2 *sup;                  // [B][blocks][nsup] (max, sum exp) of logits/T per run of `run` stages
+    int nsup, run;                // runs per block (entries reserved per block in sup), stages per run
     float4 *cta_stats;            // [B][blocks]
     int *ticket;                  // [groups]
     int32_t *status;
@@ -175,6 +176,8 @@ struct StreamArgs {
 
 struct StreamPlan {
     int items, n_items, n_stages, stage_bytes, blocks;
+    int nsup;   // LM head: runs of stages per block (second sampling level, <= 32)
+    int run;    // LM head: stages per run
     size_t smem;
 };
 

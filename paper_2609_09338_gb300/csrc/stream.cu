@@ -14,9 +14,11 @@
 //   QKV     [q;k;v] = W~_qkv [s; RMSNorm(x)], rotary on q,k; k,v -> pages
 //   OPROJ   x += W_o attn              DOWN  x += W_down h
 //   GATEUP  h = silu(W_gate n) * (W_up n), n = RMSNorm(x)
-//   LM      logits = W_lm RMSNorm(x_L); per-stage (tile) and per-block
-//           (max, sum exp, argmax); the last block draws the token by inverse
-//           CDF: block -> tile -> recompute that tile's logits -> id.
+//   LM      logits = W_lm RMSNorm(x_L), never written out (unless the caller
+//           asks for draft_logits): per-block (max, sum exp, argmax), and per
+//           run of stages (at most 32 runs a block: max, sum exp); the last block draws the token
+//           by inverse CDF: block -> run -> that run's logits, recomputed from
+//           W_lm with the main pass's arithmetic (bitwise equal) -> id.
 #include <math.h>
 
 #include "common.cuh"
@@ -319,12 +321,66 @@ __device__ int cdf_pick_regs(const float (&w)[PER], int e0, int n, float target_
 }
 
 constexpr int SG_PICK_PER = 2;    // block entries per thread in the first pick (blocks <= 2 x 288)
-constexpr int SG_PICK2_PER = 4;   // ids per thread in the second pick (ids per block <= 4 x 288)
+constexpr int SG_LM_MAXLOC = 1024;   // stages per block at most (per-stage statistics in shared memory)
+constexpr int SG_RUN_IDS = 32;    // ids of one run at most (stages per run x items)
 
-// Logits of row b at the current chain step: the caller's draft_logits when
-// given, else the workspace row.
-__device__ __forceinline__ float *lm_zrow(const StreamArgs &a, int b) {
-    return a.logits ? a.logits + ((size_t)b * a.K + a.step) * a.dim.V : a.z + (size_t)b * a.dim.V;
+
+// Inverse CDF over one weight per lane (in lane order) at `target`: the first
+// lane whose cumulative weight passes it (the last lane with weight when
+// rounding leaves the target past the total); *before = the weight before it.
+__device__ __forceinline__ int warp_cdf_pick(float c, bool valid, float target, float *before) {
+    const int lane = threadIdx.x & 31;
+    const float incl = warp_incl_scan(c);
+    const unsigned hit = __ballot_sync(0xffffffffu, valid && c > 0.f && target < incl);
+    const unsigned pos = __ballot_sync(0xffffffffu, valid && c > 0.f);
+    const int l = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+    *before = __shfl_sync(0xffffffffu, incl - c, l);
+    return l;
+}
+
+// Logits of ids [lo, hi) (at most SG_RUN_IDS) into z, each computed as
+// global_dot computes it (so bitwise equal to the main pass): warp w takes ids
+// lo + w, lo + w + SG_CW + 1, ...; the loads of all its ids for a 1024-wide
+// stretch of the row are issued before any is used.
+__device__ __forceinline__ void lm_recompute_run(const StreamArgs &a, int lo, int hi, const float *x, float *z) {
+    constexpr int NW = SG_THREADS / 32, PW = (SG_RUN_IDS + NW - 1) / NW;
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31, d = a.dim.d;
+    float acc[PW];
+#pragma unroll
+    for (int i = 0; i < PW; ++i) acc[i] = 0.f;
+    for (int b0 = 0; b0 < d; b0 += 1024) {
+        uint4 wv[PW][4];
+#pragma unroll
+        for (int i = 0; i < PW; ++i) {
+            const int id = lo + warp + i * NW;
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                const int base = b0 + 256 * c;
+                wv[i][c] = id < hi && base < d ? ld_stream(a.W + (size_t)id * d + base + lane * 8) : make_uint4(0, 0, 0, 0);
+            }
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const int base = b0 + 256 * c;
+            if (base >= d) break;
+            const float4 x0 = *(const float4 *)(x + base + lane * 8);
+            const float4 x1 = *(const float4 *)(x + base + lane * 8 + 4);
+            const float xf[8] = {x0.x, x0.y, x0.z, x0.w, x1.x, x1.y, x1.z, x1.w};
+#pragma unroll
+            for (int i = 0; i < PW; ++i) {
+                float wf[8];
+                unpack8(wv[i][c], wf);
+#pragma unroll
+                for (int e = 0; e < 8; ++e) acc[i] = fmaf(wf[e], xf[e], acc[i]);
+            }
+        }
+    }
+#pragma unroll
+    for (int i = 0; i < PW; ++i) {
+        const float v = warp_sum(acc[i]);
+        const int id = lo + warp + i * NW;
+        if (lane == 0 && id < hi) z[id - lo] = v;
+    }
 }
 
 template <int RG>
@@ -333,7 +389,9 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
     __shared__ MS shm[SG_CW + 1];
     __shared__ AM sha[SG_CW + 1];
     __shared__ float sh_scan[33];
-    __shared__ float s_e;
+    __shared__ float s_e, s_pickb;
+    __shared__ int s_pick[2];
+    __shared__ float s_run[SG_RUN_IDS];
     const Dims &D = a.dim;
     const bool greedy = a.temperature == 0.f;
     const float invT = greedy ? 1.f : 1.f / a.temperature;
@@ -374,27 +432,36 @@ __device__ void lm_sample_stream(const StreamArgs &a, int b, int rr, int src_row
         float before1;
         const int blk = cdf_pick_regs<SG_PICK_PER>(c1, e0, nblk, u, true, &before1, &S, sh_scan);
         const float target = u * S;
-        // level 2: every logit of that block's id range, written by the main
-        // pass (one load each, all in flight together)
+        // level 2: the chosen block's runs of a.run stages (at most 32: one warp)
+        const float2 *sp = a.sup + ((size_t)b * nblk + blk) * a.nsup;
         const int st0 = (int)((long long)a.n_stages * blk / nblk);
         const int st1 = (int)((long long)a.n_stages * (blk + 1) / nblk);
-        const int lo = st0 * a.items, hi = min(D.V, st1 * a.items);
-        const float *zr = lm_zrow(a, b);
-        const int f0 = t * SG_PICK2_PER;
-        float c2[SG_PICK2_PER];
-#pragma unroll
-        for (int k = 0; k < SG_PICK2_PER; ++k) {
-            const int n = lo + f0 + k;
-            c2[k] = n < hi ? __ldcg(zr + n) : -INFINITY;
+        const int nrun = (st1 - st0 + a.run - 1) / a.run;
+        const int warp = t >> 5, lane = t & 31;
+        if (warp == 0) {
+            const float2 e = lane < nrun ? __ldcg(sp + lane) : make_float2(-INFINITY, 0.f);
+            const float c = e.x == -INFINITY ? 0.f : e.y * __expf(e.x - M);
+            float bef;
+            const int run = warp_cdf_pick(c, lane < nrun, target - before1, &bef);
+            if (lane == 0) { s_pick[0] = run; s_pickb = bef; }
         }
-#pragma unroll
-        for (int k = 0; k < SG_PICK2_PER; ++k) c2[k] = c2[k] == -INFINITY ? 0.f : __expf(c2[k] * invT - M);
-        float before2, S2;
-        const int idx = cdf_pick_regs<SG_PICK2_PER>(c2, f0, hi - lo, target - before1, false, &before2, &S2, sh_scan);
-#pragma unroll
-        for (int k = 0; k < SG_PICK2_PER; ++k)
-            if (f0 + k == idx) s_e = c2[k];
         __syncthreads();
+        const int run = s_pick[0];
+        const float before2 = s_pickb;
+        // level 3: that run's logits, recomputed with the main pass's arithmetic
+        const int lo = (st0 + run * a.run) * a.items;
+        const int hi = min(D.V, min(st1, st0 + (run + 1) * a.run) * a.items);
+        lm_recompute_run(a, lo, hi, xs + (size_t)rr * D.d, s_run);
+        __syncthreads();
+        if (warp == 0) {
+            const float c = lane < hi - lo ? __expf(s_run[lane] * invT - M) : 0.f;
+            float bef;
+            const int id = warp_cdf_pick(c, lane < hi - lo, target - before1 - before2, &bef);
+            if (lane == id) s_e = c;
+            if (lane == 0) s_pick[1] = id;
+        }
+        __syncthreads();
+        const int idx = s_pick[1];
         token = lo + idx;
         qx = s_e / S;
     }
@@ -433,6 +500,7 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_MIN_BLOCKS) stream_kernel(c
     __shared__ float red[33];
     __shared__ int s_b[RG], s_pos[RG], s_act[RG], s_src[RG], s_abort;
     __shared__ float4 s_wstats[SG_CW][RG];
+    __shared__ float2 s_stst[MODE == G_LM ? SG_LM_MAXLOC : 1][RG];   // LM: (max, sum exp) of each local stage
     const Dims &D = a.dim;
     const int Kd = sg_kd(a);
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -616,7 +684,8 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_MIN_BLOCKS) stream_kernel(c
 #pragma unroll
                     for (int rr = 0; rr < RG; ++rr) {
                         const float z = acc[i][rr];
-                        if (lane == 0 && s_act[rr]) lm_zrow(a, r0 + rr)[item] = z;
+                        if (lane == 0 && s_act[rr] && a.logits)
+                            a.logits[((size_t)(r0 + rr) * a.K + a.step) * D.V + item] = z;
                         const float y = z * invT;
                         if (y > tm[rr]) { ts[rr] = ts[rr] * __expf(tm[rr] - y) + 1.f; tm[rr] = y; }
                         else ts[rr] += __expf(y - tm[rr]);
@@ -625,6 +694,7 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_MIN_BLOCKS) stream_kernel(c
                 }
 #pragma unroll
                 for (int rr = 0; rr < RG; ++rr) {
+                    if (lane == 0) s_stst[st - st0][rr] = make_float2(tm[rr], ts[rr]);
                     const MS c = ms_combine(MS{wm[rr], ws[rr]}, MS{tm[rr], ts[rr]});
                     wm[rr] = c.m;
                     ws[rr] = c.s;
@@ -648,6 +718,16 @@ __global__ void __launch_bounds__(SG_THREADS, OSP_SG_MIN_BLOCKS) stream_kernel(c
     }
     if (MODE != G_LM) return;
     __syncthreads();
+    if (warp > 0) {   // the block's runs of a.run stages
+        const int nrun = (nloc + a.run - 1) / a.run;
+        for (int e = threadIdx.x - 32; e < nrun * RG; e += SG_THREADS - 32) {
+            const int k = e / RG, rr = e - k * RG;
+            MS m{-INFINITY, 0.f};
+            for (int q = k * a.run; q < min(nloc, (k + 1) * a.run); ++q)
+                m = ms_combine(m, MS{s_stst[q][rr].x, s_stst[q][rr].y});
+            if (r0 + rr < a.B) a.sup[((size_t)(r0 + rr) * nblk + blockIdx.x) * a.nsup + k] = make_float2(m.m, m.s);
+        }
+    }
     if (warp == 0) {
 #pragma unroll
         for (int rr = 0; rr < RG; ++rr) {
@@ -706,6 +786,10 @@ StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms) {
     p.n_stages = (p.n_items + p.items - 1) / p.items;
     const int bps = mode == G_LM ? OSP_SG_BLOCKS_PER_SM : OSP_SG_GEMV_BPS;
     p.blocks = p.n_stages < sms * bps ? p.n_stages : sms * bps;
+    // LM head runs: the fewest stages per run that leave at most 32 runs a block
+    const int maxloc = (p.n_stages + p.blocks - 1) / p.blocks;
+    p.run = (maxloc + 31) / 32;
+    p.nsup = (maxloc + p.run - 1) / p.run;
     p.smem = (size_t)SG_NST * p.stage_bytes;
     return p;
 }
@@ -719,10 +803,15 @@ bool stream_supported(GemvMode mode, const Dims &D, int rg, int sms) {
     if (rg < 1 || rg > 2 || mode == G_FEAT) return false;
     const StreamPlan p = stream_plan(mode, D, sms);
     if (stream_smem(mode, D, rg, p) > 200 * 1024) return false;
-    // the LM head's sampler holds at most SG_PICK_PER entries per thread at each level
-    if (mode == G_LM && (p.blocks > SG_PICK_PER * SG_THREADS ||
-                         (long long)((p.n_stages + p.blocks - 1) / p.blocks) * p.items > SG_PICK2_PER * SG_THREADS))
-        return false;
+    // the LM head's sampler: blocks at most SG_PICK_PER per thread; a block's
+    // stages within its statistics array; a run's ids within the recompute buffer
+    // (the plan keeps the runs of a block at most 32)
+    if (mode == G_LM) {
+        const int maxloc = (p.n_stages + p.blocks - 1) / p.blocks;
+        if (p.blocks > SG_PICK_PER * SG_THREADS || maxloc > SG_LM_MAXLOC ||
+            p.run * p.items > SG_RUN_IDS)
+            return false;
+    }
     return true;
 }
 
@@ -761,7 +850,7 @@ static cudaError_t launch_stream_nrs(const StreamArgs &a, int nrs, int groups, i
 cudaError_t launch_stream(GemvMode mode, const StreamArgs &a, int rg, cudaStream_t s) {
     const int rows = mode == G_LM ? a.B : a.R;
     const int groups = (rows + rg - 1) / rg;
-    StreamPlan p{a.items, a.n_items, a.n_stages, a.stage_bytes, a.blocks, 0};
+    StreamPlan p{a.items, a.n_items, a.n_stages, a.stage_bytes, a.blocks, 0, 0};
     const size_t smem = stream_smem(mode, a.dim, rg, p);
     const int blocks = a.n_stages < a.blocks ? a.n_stages : a.blocks;
     const bool pair = mode == G_QKV || mode == G_GATEUP;
