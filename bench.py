@@ -36,12 +36,12 @@ sys.path.insert(0, ROOT)
 from paper_2609_09338_gb300 import synthetic as syn  # noqa: E402
 from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: E402
 
-# dram__bytes_read.sum + dram__bytes_write.sum of one LM-head launch of this
-# workload (the first LM head of a bench run, ncu --set full); valid only for
-# the stream.cu it was taken on.
+# dram__bytes_read.sum + dram__bytes_write.sum of one streamed LM-head launch
+# at batch 1 (qwen3-8b-d1024-v151936-b1-k7: the first LM head of a bench run,
+# ncu --set full); valid only for the stream.cu it was taken on.
 LM_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/stream.cu",
-              "sha256": "90d10a609dc3cdd6796755d7c6ff7213e7e7ddeb5064fcb5779e04778e7230de",
-              "bytes_per_launch": 314_359_808}
+              "sha256": "a4f2882b1b34ce368a59d87ad9d0b5db7b24847fc69e9b08247be5cbbd02cebe",
+              "bytes_per_launch": 311_286_528 + 2_934_016}
 # DRAM bytes (read + write) of one attention launch at the large-vocabulary
 # workload, from one ncu capture of this source (profiles/attn_large-vocab-*.md)
 ATTN_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/draft.cu",
