@@ -768,7 +768,8 @@ StreamPlan stream_plan(GemvMode mode, const Dims &D, int sms) {
     const int Kd = host_kd(mode, D);
     const int row_bytes = Kd * 2;
     const int target = mode == G_LM ? OSP_SG_LM_STAGE : OSP_SG_STAGE;   // bytes per stage
-    int rows = target / row_bytes;
+    // the LM head rounds to the nearest whole row (d 2560: two 5 KB rows, not one)
+    int rows = mode == G_LM ? (target + row_bytes / 2) / row_bytes : target / row_bytes;
     const bool pair = mode == G_QKV || mode == G_GATEUP;
     rows = rows < (pair ? 2 : 1) ? (pair ? 2 : 1) : rows;
     rows = rows > SG_MAXR ? SG_MAXR : (!pair && rows >= 6 ? 6 : pow2_floor(rows));
