@@ -40,7 +40,7 @@ from paper_2609_09338_gb300.workloads import BENCH_WORKLOAD, WORKLOADS  # noqa: 
 # at batch 1 (qwen3-8b-d1024-v151936-b1-k7: the first LM head of a bench run,
 # ncu --set full); valid only for the stream.cu it was taken on.
 LM_TRAFFIC = {"source": "paper_2609_09338_gb300/csrc/stream.cu",
-              "sha256": "a4f2882b1b34ce368a59d87ad9d0b5db7b24847fc69e9b08247be5cbbd02cebe",
+              "sha256": "52f460bbc3c87bb8a826df02e23cb78a1374cbd91b4bcbe4cc2ebfcecdf7d6bd",
               "bytes_per_launch": 311_286_528 + 2_934_016}
 # DRAM bytes (read + write) of one attention launch at the large-vocabulary
 # workload, from one ncu capture of this source (profiles/attn_large-vocab-*.md)
