@@ -231,7 +231,7 @@ static cudaError_t probe_record(cudaEvent_t ev, cudaStream_t s) {
 
 // ------------------------------------------------------------------ workspace
 // block: the layout of a block-drafting call (every extend row is sampled, so
-// the logits and sampler buffers hold B * max_new rows instead of B)
+// the sampler buffers hold B * max_new rows instead of B)
 static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int max_pages,
                            DraftWs *ws, void *base, bool block = false) {
     const Dims &D = ctx->dim;
@@ -258,7 +258,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
     size_t o_fh = take(4ull * R_ext * D.F);
     size_t o_ls = take(16ull * B * lm_warps);
     const StreamPlan lmp = stream_plan(G_LM, D, ctx->sms);
-    size_t o_lz = take(8ull * B * lmp.blocks * lmp.nsup);   // the streamed LM head's run statistics (rows <= 2)
+    size_t o_lsup = take(8ull * B * lmp.blocks * lmp.nsup);   // the streamed LM head's run statistics (rows <= 2)
     size_t o_lc = take(16ull * B * lmp.blocks);
     // tensor-core path: bf16 operand planes, QKV output, row-sampler partials
     const long long tc_rows = std::min<long long>(std::max<long long>(R_ext, B), TC_MAX_ROWS);
@@ -304,7 +304,7 @@ static size_t draft_layout(const osprey_ctx *ctx, int B, int K, int max_new, int
         ws->attn_out = (float *)(p + o_ao);
         ws->ffn_h = (float *)(p + o_fh);
         ws->lm_stats = (float4 *)(p + o_ls);
-        ws->lm_sup = (float2 *)(p + o_lz);
+        ws->lm_sup = (float2 *)(p + o_lsup);
         ws->lm_cta_stats = (float4 *)(p + o_lc);
         ws->tc_xq = (uint16_t *)(p + o_xq);
         ws->tc_yq = (float *)(p + o_yq);
