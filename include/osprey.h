@@ -110,7 +110,9 @@ const char *osprey_last_error(void);
  * The context picks the kernels a draft call uses:
  *   rows <= 2 per chain step: TMA-streamed GEMVs (weights read once per step);
  *   3..80 rows: tcgen05 tensor-core GEMMs, float32 activations split into three
- *     bf16 planes (24 mantissa bits) so results match the GEMV path's;
+ *     bf16 planes (24 mantissa bits) so results match the GEMV path's (the LM
+ *     head's operand into two planes, 16 bits: its logits differ from the
+ *     GEMV path's by rounding of the operand's last bits);
  *   attention: clusters merged on chip while they fit one wave, else global
  *     partials.
  * Two environment variables, read here, select the alternatives for testing:
