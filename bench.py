@@ -235,16 +235,19 @@ def _blas():
 
 def oracle_sequence_step(wl, ctx, w, W, kv, di, vi, b):
     """One sequence's share of a step, run by the oracle: its draft call (extend
-    rows + K-token chain) and its verification."""
+    rows + K-token chain) and its verification.  Returns the seconds each took."""
     from oracle import drafter as od
     from oracle import verify as ov
     offs = np.concatenate([[0], np.cumsum(ctx)]).astype(np.int64)
     sl = slice(int(offs[b]), int(offs[b + 1]))
+    t0 = time.perf_counter()
     od.draft_step(w, wl.shape, kv["k_rows"][:, sl], kv["v_rows"][:, sl], ctx[b:b + 1], di["tokens"][b:b + 1],
                   di["feats"][b:b + 1], di["n_new"][b:b + 1], wl.K, wl.temperature, di["u_draft"][b:b + 1],
                   widened=W)
+    t1 = time.perf_counter()
     ov.verify(vi["target_logits"][b:b + 1], vi["draft_logits"][b:b + 1], vi["draft_tokens"][b:b + 1],
               wl.temperature, vi["u_accept"][b:b + 1], vi["u_sample"][b:b + 1])
+    return t1 - t0, time.perf_counter() - t1
 
 
 def cpu_baseline(wl, ctx, w, kv, di, vi, budget_s=8.0):
@@ -260,27 +263,32 @@ def cpu_baseline(wl, ctx, w, kv, di, vi, budget_s=8.0):
     threads = blas[0]() if blas else None
 
     def sample(budget):
-        n, t_run = 0, 0.0
+        n, t_run, phases = 0, 0.0, []
         while True:
             b = n % wl.batch
             t1 = time.perf_counter()
-            oracle_sequence_step(wl, ctx, w, W, kv, di, vi, b)
+            phases.append(oracle_sequence_step(wl, ctx, w, W, kv, di, vi, b))
             t_run += time.perf_counter() - t1
             n += 1
             if t_run > budget or n >= 4 * wl.batch:
-                return n, t_run
-    n, t_run = sample(budget_s)
+                return n, t_run, phases
+    n, t_run, phases = sample(budget_s)
     res = {"value": n / t_run / wl.batch, "unit": "steps/s", "cores": threads, "kind": "oracle",
            "sample": f"{n} sequence(s) of {wl.name} (draft call K={wl.K} + verify each, float64 numpy), "
                      f"scaled to steps of {wl.batch} sequences; weights widened once ({setup:.1f}s, untimed); "
-                     f"cores = numpy BLAS threads; {os.cpu_count()} host cores visible"}
+                     f"cores = numpy BLAS threads; {os.cpu_count()} host cores visible",
+           # per sequence, over the sample: the draft call and the verification apart
+           "draft_call_s_median": float(np.median([p[0] for p in phases])),
+           "verify_s_median": float(np.median([p[1] for p in phases]))}
     if blas and threads and threads > 1:
         blas[1](1)
         try:
-            n1, t1 = sample(budget_s / 2)
+            n1, t1, phases1 = sample(budget_s / 2)
         finally:
             blas[1](threads)
-        res["one_core"] = {"value": n1 / t1 / wl.batch, "cores": 1, "sample": f"{n1} sequence(s)"}
+        res["one_core"] = {"value": n1 / t1 / wl.batch, "cores": 1, "sample": f"{n1} sequence(s)",
+                           "draft_call_s_median": float(np.median([p[0] for p in phases1])),
+                           "verify_s_median": float(np.median([p[1] for p in phases1]))}
     return res
 
 
